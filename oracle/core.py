@@ -1,0 +1,208 @@
+"""Oracle core: prior, fusion, greedy decode, verification, statistics.
+
+Test infrastructure only (see the package docstring). Plain fp64 numpy.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+
+# ----------------------------------------------------------------------------
+# data decoding (the oracle reads stored tensors itself; no shared helpers)
+# ----------------------------------------------------------------------------
+
+def to_f64(t) -> np.ndarray:
+    """Exact float64 copy of a torch tensor or numpy array (f32, bf16, ints).
+
+    bf16 is decoded from its bit pattern: the 16 stored bits are the upper
+    half of an IEEE float32.
+    """
+    try:
+        import torch
+    except ImportError:  # pragma: no cover
+        torch = None
+    if torch is not None and isinstance(t, torch.Tensor):
+        t = t.detach().cpu()
+        if t.dtype == torch.bfloat16:
+            bits = t.contiguous().view(torch.int16).numpy().view(np.uint16)
+            return (bits.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+        return t.numpy().astype(np.float64)
+    return np.asarray(t, dtype=np.float64)
+
+
+def round_bf16(x: np.ndarray) -> np.ndarray:
+    """Round to bf16 (round-to-nearest-even) through float32; returns float64.
+
+    This is the precision contract for activations that feed a bf16 product.
+    """
+    f = np.asarray(x, dtype=np.float32)
+    if not np.all(np.isfinite(f)):
+        raise ValueError("round_bf16: non-finite activation")
+    u = f.view(np.uint32).astype(np.uint64)
+    lsb = (u >> 16) & 1
+    u = ((u + 0x7FFF + lsb) >> 16) << 16
+    return u.astype(np.uint32).view(np.float32).astype(np.float64)
+
+
+# ----------------------------------------------------------------------------
+# unigram prior (Appendix A, "Unigram Prior Estimation")
+# ----------------------------------------------------------------------------
+
+def log_prior(counts, lam: float = 1.0) -> np.ndarray:
+    """l_P(v) = log( (c(v) + lambda) / sum_v' (c(v') + lambda) ), lambda = 1 by default."""
+    c = to_f64(counts)
+    if c.ndim != 1 or c.size == 0:
+        raise ValueError("counts must be a non-empty vector")
+    if np.any(c < 0) or lam <= 0:
+        raise ValueError("counts must be >= 0 and lambda > 0")
+    p = (c + lam) / np.sum(c + lam)
+    return np.log(p)
+
+
+# ----------------------------------------------------------------------------
+# fusion and decode (Section 4.3 equation; Algorithm 1, Decode at T = 0)
+# ----------------------------------------------------------------------------
+
+def lse(x: np.ndarray) -> float:
+    """log sum_v exp(x_v) for one row (textbook max-shifted form)."""
+    x = np.asarray(x, dtype=np.float64)
+    m = np.max(x)
+    if m == -np.inf:
+        raise ValueError("all entries are -inf")
+    return float(m + np.log(np.sum(np.exp(x - m))))
+
+
+def fuse(long, short, prior, alpha: float, beta: float) -> np.ndarray:
+    """l = l_L + alpha * l_S - beta * l_P (Section 4.3). ``short``/``prior`` may be None
+    (then that term is absent)."""
+    out = np.array(long, dtype=np.float64, copy=True)
+    if short is not None:
+        out = out + alpha * np.asarray(short, dtype=np.float64)
+    if prior is not None:
+        out = out - beta * np.asarray(prior, dtype=np.float64)
+    return out
+
+
+def greedy_decode(l: np.ndarray):
+    """Temperature-0 Decode(softmax(l)) of one row.
+
+    Returns (x, logp, gap): x = argmax with the lowest index on exact ties,
+    logp = log softmax(l)[x] = l[x] - LSE(l), gap = l[x] - max_{v != x} l[v]
+    (+inf for a one-entry row).
+    """
+    l = np.asarray(l, dtype=np.float64)
+    if np.any(np.isnan(l)) or np.any(l == np.inf):
+        raise ValueError("non-finite logits")
+    x = int(np.argmax(l))              # first occurrence of the maximum
+    logp = float(l[x] - lse(l))
+    if l.size == 1:
+        gap = np.inf
+    else:
+        rest = np.concatenate([l[:x], l[x + 1:]])
+        gap = float(l[x] - np.max(rest))
+    return x, logp, gap
+
+
+def combine_argmax(long, short, prior, alpha: float, beta: float):
+    """Row-wise fuse + greedy decode of [rows, V] logits.
+
+    Returns int64 tokens [rows], float64 logp [rows], float64 gap [rows].
+    """
+    L = to_f64(long)
+    S = None if short is None else to_f64(short)
+    P = None if prior is None else np.asarray(prior, dtype=np.float64)
+    rows = L.shape[0]
+    tok = np.zeros(rows, np.int64)
+    lp = np.zeros(rows)
+    gap = np.zeros(rows)
+    for i in range(rows):
+        f = fuse(L[i], None if S is None else S[i], P, alpha, beta)
+        tok[i], lp[i], gap[i] = greedy_decode(f)
+    return tok, lp, gap
+
+
+# ----------------------------------------------------------------------------
+# verification (Algorithm 1, greedy verification by one target forward)
+# ----------------------------------------------------------------------------
+
+def verify_greedy(draft, target):
+    """Greedy verification of a drafted block against target logits.
+
+    draft [B, n] tokens x_0..x_{n-1}; target [B, n+1, V] logits. Row j of the
+    target gives its own choice t_j = argmax_v target[b, j, v] (lowest index on
+    ties) for draft position j; row n is the bonus row. The accepted length a
+    is the number of leading positions with x_j == t_j (0..n) and the bonus
+    token is t_a. Returns (accept [B] int64, bonus [B] int64, t [B, n+1] int64).
+    """
+    D = np.asarray(draft, dtype=np.int64)
+    T = to_f64(target)
+    B, n = D.shape
+    if T.shape[:2] != (B, n + 1):
+        raise ValueError("target must be [B, n+1, V]")
+    t = np.zeros((B, n + 1), np.int64)
+    for b in range(B):
+        for j in range(n + 1):
+            row = T[b, j]
+            if np.any(np.isnan(row)):
+                raise ValueError("NaN target logits")
+            t[b, j] = int(np.argmax(row))
+    accept = np.zeros(B, np.int64)
+    bonus = np.zeros(B, np.int64)
+    for b in range(B):
+        a = 0
+        while a < n and D[b, a] == t[b, a]:
+            a += 1
+        accept[b] = a
+        bonus[b] = t[b, a]
+    return accept, bonus, t
+
+
+# ----------------------------------------------------------------------------
+# acceptance statistics (Appendix D)
+# ----------------------------------------------------------------------------
+
+def acceptance_rates(accept, n: int):
+    """rate_i = P(acceptance length >= i), i = 1..n+1, and tau = E[length].
+
+    The acceptance length counts the bonus token, L = a + 1, so rate_1 = 1
+    (the first position is always produced). Returns (rates [n+1], tau).
+    """
+    a = np.asarray(accept, dtype=np.int64)
+    if a.size == 0:
+        raise ValueError("no blocks")
+    L = a + 1
+    rates = np.array([np.mean(L >= i) for i in range(1, n + 2)], dtype=np.float64)
+    return rates, float(np.mean(L))
+
+
+# ----------------------------------------------------------------------------
+# exact factorisation (Section 4.1; proof in Appendix B)
+# ----------------------------------------------------------------------------
+
+def poe_factors(joint: np.ndarray):
+    """Factors of p(x | y, z) for a joint table p[x, y, z] > 0.
+
+    Returns (p_x_given_yz, poe, context, residual), each indexed [x, y, z]:
+      poe      = p(x|y) p(x|z) / p(x)
+      context  = p(y) p(z) / p(y, z)            (independent of x)
+      residual = p(y, z | x) / (p(y|x) p(z|x))
+    so that p(x|y,z) = poe * context * residual.
+    """
+    p = np.asarray(joint, dtype=np.float64)
+    p = p / p.sum()
+    px = p.sum(axis=(1, 2))
+    py = p.sum(axis=(0, 2))
+    pz = p.sum(axis=(0, 1))
+    pxy = p.sum(axis=2)
+    pxz = p.sum(axis=1)
+    pyz = p.sum(axis=0)
+    p_x_given_yz = p / pyz[None, :, :]
+    p_x_given_y = pxy / py[None, :]
+    p_x_given_z = pxz / pz[None, :]
+    poe = p_x_given_y[:, :, None] * p_x_given_z[:, None, :] / px[:, None, None]
+    context = (py[:, None] * pz[None, :] / pyz)[None, :, :] * np.ones_like(p)
+    p_yz_given_x = p / px[:, None, None]
+    p_y_given_x = pxy / px[:, None]
+    p_z_given_x = pxz / px[:, None]
+    residual = p_yz_given_x / (p_y_given_x[:, :, None] * p_z_given_x[:, None, :])
+    return p_x_given_yz, poe, context, residual
