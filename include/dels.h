@@ -1,0 +1,214 @@
+/*
+ * dels.h — C ABI of the DeLS-Spec per-block drafting hot path on GB300 (sm_103a).
+ *
+ * DeLS-Spec ("Decoupled Long-Short Contexts for Parallel Speculative
+ * Drafting") keeps a block-parallel drafter (DFlash) fixed as the
+ * long-context expert, adds a small autoregressive local head over the tokens
+ * already drafted in the block as the short-context expert, and fuses the
+ * two with a unigram prior correction (Section 4.3):
+ *
+ *     l(x) = l_L(x | y) + alpha * l_S(x | z) - beta * l_P(x)
+ *
+ * Each block position is decoded from softmax(l) and fed back to the local
+ * head; the finished block is verified by the target model (Algorithm 1).
+ * This library runs that loop at temperature 0 (Decode = argmax, lowest
+ * vocabulary index on exact ties) as hand-written CUDA kernels.
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ * - Pointers marked [device] are CUDA device pointers owned by the caller;
+ *   tensors are contiguous, row-major, the vocabulary dimension innermost,
+ *   and 16-byte aligned. Pointers marked [host] are ordinary host memory.
+ * - Calls are asynchronous on the given stream (a cudaStream_t; NULL is the
+ *   legacy default stream) and never synchronise, except dels_read_status.
+ * - The library allocates no memory and keeps no state between calls. Every
+ *   call takes a caller-owned device workspace of at least the size its
+ *   *_workspace_bytes function returns for the same arguments on the current
+ *   device. A workspace must be zero-filled once before its first use (for
+ *   example with cudaMemset); every call leaves it ready for the next call.
+ *   Calls that share a workspace must be ordered on one stream.
+ * - Return value: DELS_OK (0) or a negative DELS_ERR_* code detected on the
+ *   host, in which case nothing was enqueued. Errors detected on the device
+ *   (non-finite logits, an out-of-range token, a timed-out wait) are OR-ed
+ *   into a status word inside the workspace; read and clear it with
+ *   dels_read_status.
+ * - dtype codes: DELS_F32 (IEEE float32) or DELS_BF16 (bfloat16 bit pattern).
+ */
+#ifndef DELS_H_
+#define DELS_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Binary-compatible with cudaStream_t (struct CUstream_st*). */
+typedef struct CUstream_st* dels_stream_t;
+
+/* ---- status codes ------------------------------------------------------ */
+enum {
+  DELS_OK = 0,
+  /* detected on the host; nothing was enqueued */
+  DELS_ERR_NULL_POINTER = -1,      /* a required pointer is NULL */
+  DELS_ERR_BAD_SHAPE = -2,         /* a size is out of the supported range */
+  DELS_ERR_BAD_DTYPE = -3,         /* unknown or unsupported dtype code */
+  DELS_ERR_ALIGNMENT = -4,         /* a pointer or row pitch is not 16-byte aligned */
+  DELS_ERR_WORKSPACE = -5,         /* workspace NULL or smaller than required */
+  DELS_ERR_UNSUPPORTED = -6,       /* head kind / dims this build does not run */
+  DELS_ERR_CUDA = -7,              /* a CUDA runtime or driver call failed */
+  /* detected on the device; bits of the workspace status word */
+  DELS_STATUS_NONFINITE = 1,       /* NaN or +inf logit, or a row that is all -inf */
+  DELS_STATUS_TIMEOUT = 2,         /* a bounded device-side wait expired */
+  DELS_STATUS_BAD_TOKEN = 4        /* a draft token outside [0, V) */
+};
+
+typedef enum { DELS_F32 = 0, DELS_BF16 = 1 } dels_dtype;
+
+typedef enum {
+  DELS_HEAD_GRU = 0,    /* Appendix A RNN head (the paper's default)      */
+  DELS_HEAD_MLP = 1,    /* window MLP over the last `window` drafted tokens */
+  DELS_HEAD_XFMR = 2,   /* 1-layer causal transformer over the block prefix */
+  DELS_HEAD_MARKOV = 3  /* Appendix A Markov head                        */
+} dels_head_kind;
+
+/*
+ * Local head (short-context expert) weights. All matrices are [device],
+ * row-major [out, in] like a Linear layer, dtype `wdtype` (bf16 heads run the
+ * matrix products on tcgen05 tensor cores; f32 heads on CUDA cores). V is the
+ * vocabulary size of the call. Weight slots by kind:
+ *
+ * DELS_HEAD_GRU  (Appendix A): emb = E_tgt [V, d_model];
+ *     w[0] = W_ih [3*d_hidden, d_model], gate rows ordered (r, z, n);
+ *     w[1] = W_hh [3*d_hidden, d_hidden]; w[2] = W_rank [d_rank, d_hidden];
+ *     w_vocab = W_vocab [V, d_rank].
+ *     h_j = GRU(E_tgt[x_{j-1}], h_{j-1}) bias-free (PyTorch gate form),
+ *     h_0 = 0; r_j = SiLU(W_rank h_j); l_S = W_vocab r_j.
+ * DELS_HEAD_MLP: emb = E [V, d_model]; w[0] = W_1 [d_hidden, window*d_model];
+ *     w[1] = W_2 [d_hidden, d_hidden] when n_layers == 2; w_vocab [V, d_hidden];
+ *     d_rank must equal d_hidden. u = [E x_{j-1}; ...; E x_{j-window}] with
+ *     zero blocks before the block start; h = GELU(W_1 u) (then GELU(W_2 h)).
+ * DELS_HEAD_XFMR: emb = E [V, d_model]; w[0] = P [max_pos, d_model] position
+ *     table; w[1..4] = W_q, W_k, W_v, W_o [d_model, d_model];
+ *     w[5] = W_1 [d_hidden, d_model]; w[6] = W_2 [d_model, d_hidden];
+ *     w_vocab [V, d_model]; d_rank must equal d_model. Pre-RMSNorm block
+ *     (eps 1e-6, unit gain), n_heads causal heads, GELU FFN, final RMSNorm.
+ * DELS_HEAD_MARKOV (Appendix A): emb = E_M [V, d_rank]; w_vocab = W_M [V, d_rank];
+ *     l_S = W_M E_M[x_{j-1}].
+ *
+ * Activations that feed a bf16 product are rounded to bf16 (round to nearest
+ * even); accumulation and the recurrent GRU state are float32.
+ */
+typedef struct {
+  dels_head_kind kind;
+  dels_dtype wdtype;
+  int d_model;
+  int d_hidden;
+  int d_rank;
+  int window;
+  int n_layers;
+  int n_heads;
+  int max_pos;
+  const void* emb;
+  const void* w[8];
+  const void* w_vocab;
+} dels_local_head;
+
+/* ---- per-block drafting (Algorithm 1, temperature 0) --------------------- */
+
+/* Workspace bytes for dels_draft_block with these arguments on the current
+ * device; 0 if the arguments are not supported. */
+size_t dels_draft_workspace_bytes(const dels_local_head* head, int B, int n, int V);
+
+/*
+ * Drafts one block of n tokens for each of B independent requests
+ * (Algorithm 1; fusion of Section 4.3):
+ *   x_0 = argmax_v l_L[b,0,v]                          (no head, no prior)
+ *   for j = 1..n-1:  l_S = head(x_{0:j-1});
+ *                    x_j = argmax_v l_L[b,j,v] + alpha*l_S[v] - beta*l_P[v]
+ * long_logits  [device] [B, n, V] of logit_dtype (DFlash logits l_L).
+ * log_prior    [device] [V] float32 log unigram prior l_P (finite).
+ * out_tokens   [device] [B, n] int32 drafted tokens.
+ * out_logprob  [device] [B, n] float32 log softmax of the fused row at x_j.
+ * out_top2_gap [device] [B, n] float32 top-1 minus top-2 fused value; may be NULL.
+ * Limits: 1 <= B <= 128, 1 <= n <= 32, 8 <= V < 2^31, V % 8 == 0; bf16 heads
+ * need d_model, d_hidden, d_rank multiples of 16 (d_rank <= 4096); the
+ * transformer head needs n <= max_pos and d_model % n_heads == 0.
+ * B == 0 is a no-op.
+ */
+int dels_draft_block(const dels_local_head* head, const void* long_logits, dels_dtype logit_dtype,
+                     const float* log_prior, float alpha, float beta, int B, int n, int V,
+                     int32_t* out_tokens, float* out_logprob, float* out_top2_gap, void* workspace,
+                     size_t workspace_bytes, dels_stream_t stream);
+
+/* ---- fused combine + argmax over independent rows ---------------------- */
+
+size_t dels_combine_workspace_bytes(int rows, int V, dels_dtype dtype);
+
+/*
+ * For each of `rows` independent rows: l = l_L + alpha*l_S - beta*l_P
+ * (Section 4.3), then x = argmax l (lowest index on ties),
+ * logprob = l[x] - logsumexp(l), gap = l[x] - max_{v != x} l[v]
+ * (+inf when V == 1). One pass over the inputs; no [rows, V] intermediate
+ * is written.
+ * long_logits, short_logits [device] [rows, V] of `dtype`; short_logits may
+ * be NULL (then the alpha term is absent). log_prior [device] [V] float32,
+ * may be NULL (then the beta term is absent).
+ * out_token [device] [rows] int32; out_logprob [device] [rows] float32 (may
+ * be NULL); out_top2_gap [device] [rows] float32 (may be NULL).
+ * Limits: 0 <= rows < 2^31, 1 <= V < 2^31. Any V works; V % 8 == 0 (bf16) or
+ * V % 4 == 0 (f32) takes the 128-bit vector path.
+ */
+int dels_combine_argmax(const void* long_logits, const void* short_logits, dels_dtype dtype,
+                        const float* log_prior, float alpha, float beta, int rows, int V,
+                        int32_t* out_token, float* out_logprob, float* out_top2_gap, void* workspace,
+                        size_t workspace_bytes, dels_stream_t stream);
+
+/* ---- greedy verification (Algorithm 1, last two steps) ------------------ */
+
+size_t dels_verify_workspace_bytes(int B, int n, int V, dels_dtype dtype);
+
+/*
+ * Greedy verification of drafted blocks against the target's logits.
+ * draft_tokens  [device] [B, n] int32 x_0..x_{n-1}.
+ * target_logits [device] [B, n+1, V] of `dtype`: row j is the target's
+ *               distribution for draft position j; row n is the bonus row.
+ * t_j = argmax_v target[b,j,v] (lowest index on ties);
+ * out_accept_len [device] [B] int32: a = number of leading j with x_j == t_j (0..n);
+ * out_bonus      [device] [B] int32: t_a (the token the target adds);
+ * out_target_argmax [device] [B, n+1] int32 t_j, may be NULL.
+ * Limits: 0 <= B, 1 <= n <= 1024, 1 <= V < 2^31.
+ */
+int dels_verify_block(const int32_t* draft_tokens, const void* target_logits, dels_dtype dtype, int B, int n,
+                      int V, int32_t* out_accept_len, int32_t* out_bonus, int32_t* out_target_argmax,
+                      void* workspace, size_t workspace_bytes, dels_stream_t stream);
+
+/* ---- helpers ------------------------------------------------------------ */
+
+/*
+ * Reads the device status word of `workspace` into *out_status (an OR of
+ * DELS_STATUS_* bits, 0 when every call since the last read succeeded) and
+ * clears it. Synchronises `stream`.
+ */
+int dels_read_status(void* workspace, dels_stream_t stream, int32_t* out_status);
+
+/*
+ * Unigram log prior of Appendix A on the host:
+ *   l_P(v) = log( (counts[v] + lambda) / sum_u (counts[u] + lambda) ), in float64,
+ * stored as float32. counts [host] [V] int64 >= 0; lambda > 0 (the paper uses 1);
+ * out_log_prior [host] [V] float32.
+ */
+int dels_prior_from_counts(const int64_t* counts, int V, double lambda, float* out_log_prior);
+
+/* Human-readable name of a status or error code. */
+const char* dels_status_string(int code);
+
+/* Library ABI version (major * 10000 + minor * 100 + patch). */
+int dels_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* DELS_H_ */

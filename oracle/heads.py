@@ -219,6 +219,7 @@ class DraftResult:
     gap: np.ndarray           # [B, n] top-1 minus top-2 fused value
     argmax: np.ndarray        # [B, n] argmax of the fused logits at each position
     fused_at: Optional[np.ndarray] = None   # [B, n] fused value at the forced token
+    fused_max: Optional[np.ndarray] = None  # [B, n] maximum fused value (forced mode)
     logp_at: Optional[np.ndarray] = None    # [B, n] log softmax at the forced token
     short_rows: Optional[Dict] = None       # {(b, j): l_S row} when requested
 
@@ -244,6 +245,7 @@ def draft_block(head, long, prior, alpha, beta, forced=None, keep_short=()):
     logp = np.zeros((B, n))
     gap = np.zeros((B, n))
     fused_at = np.zeros((B, n)) if forced is not None else None
+    fused_max = np.zeros((B, n)) if forced is not None else None
     logp_at = np.zeros((B, n)) if forced is not None else None
     forced = None if forced is None else np.asarray(forced, dtype=np.int64)
     kept = {}
@@ -258,6 +260,7 @@ def draft_block(head, long, prior, alpha, beta, forced=None, keep_short=()):
             xf = int(forced[b, j])
             tokens[b, j] = xf
             fused_at[b, j] = f[xf]
+            fused_max[b, j] = f[x]
             logp_at[b, j] = f[xf] - lse(f)
         else:
             tokens[b, j] = x
@@ -274,4 +277,4 @@ def draft_block(head, long, prior, alpha, beta, forced=None, keep_short=()):
             if (b, j) in keep_short:
                 kept[(b, j)] = S[b].copy()
             record(b, j, f)
-    return DraftResult(tokens, logp, gap, amax, fused_at, logp_at, kept or None)
+    return DraftResult(tokens, logp, gap, amax, fused_at, fused_max, logp_at, kept or None)

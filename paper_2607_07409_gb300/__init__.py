@@ -1,0 +1,247 @@
+"""Python binding of ``libdels.so``, the DeLS-Spec drafting hot path on GB300.
+
+Argument marshalling only: every step of the drafting loop, the combine and
+the verification runs in the library's CUDA kernels. Functions named
+``dels_*`` mirror the C ABI in ``include/dels.h`` one to one and take torch
+tensors (or raw integer device pointers) in place of the C pointers. The
+``Drafter`` helper keeps a local head's weight pointers and a workspace for
+repeated calls. There is no CPU fallback: if ``libdels.so`` has not been
+built, every call raises ``RuntimeError``.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Dict, Optional
+
+import torch
+
+__all__ = [
+    "DELS_OK", "DELS_F32", "DELS_BF16",
+    "DELS_HEAD_GRU", "DELS_HEAD_MLP", "DELS_HEAD_XFMR", "DELS_HEAD_MARKOV",
+    "DELS_STATUS_NONFINITE", "DELS_STATUS_TIMEOUT", "DELS_STATUS_BAD_TOKEN",
+    "DelsError", "LocalHead", "lib", "library_path", "exported_symbols",
+    "dels_draft_workspace_bytes", "dels_draft_block",
+    "dels_combine_workspace_bytes", "dels_combine_argmax",
+    "dels_verify_workspace_bytes", "dels_verify_block",
+    "dels_read_status", "dels_prior_from_counts", "dels_status_string", "dels_version",
+    "make_head", "Drafter", "dtype_code",
+]
+
+DELS_OK = 0
+DELS_F32, DELS_BF16 = 0, 1
+DELS_HEAD_GRU, DELS_HEAD_MLP, DELS_HEAD_XFMR, DELS_HEAD_MARKOV = 0, 1, 2, 3
+DELS_STATUS_NONFINITE, DELS_STATUS_TIMEOUT, DELS_STATUS_BAD_TOKEN = 1, 2, 4
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_LIB_PATH = os.path.join(_HERE, "libdels.so")
+_lib = None
+
+# name -> (restype, argtypes); the C ABI of include/dels.h
+_vp, _i, _f, _d, _sz = ctypes.c_void_p, ctypes.c_int, ctypes.c_float, ctypes.c_double, ctypes.c_size_t
+
+
+class LocalHead(ctypes.Structure):
+    """Mirror of ``dels_local_head``."""
+
+    _fields_ = [
+        ("kind", ctypes.c_int), ("wdtype", ctypes.c_int),
+        ("d_model", ctypes.c_int), ("d_hidden", ctypes.c_int), ("d_rank", ctypes.c_int),
+        ("window", ctypes.c_int), ("n_layers", ctypes.c_int), ("n_heads", ctypes.c_int),
+        ("max_pos", ctypes.c_int),
+        ("emb", ctypes.c_void_p), ("w", ctypes.c_void_p * 8), ("w_vocab", ctypes.c_void_p),
+    ]
+
+
+_SIGS = {
+    "dels_draft_workspace_bytes": (_sz, [ctypes.POINTER(LocalHead), _i, _i, _i]),
+    "dels_draft_block": (_i, [ctypes.POINTER(LocalHead), _vp, _i, _vp, _f, _f, _i, _i, _i, _vp, _vp, _vp, _vp, _sz,
+                              _vp]),
+    "dels_combine_workspace_bytes": (_sz, [_i, _i, _i]),
+    "dels_combine_argmax": (_i, [_vp, _vp, _i, _vp, _f, _f, _i, _i, _vp, _vp, _vp, _vp, _sz, _vp]),
+    "dels_verify_workspace_bytes": (_sz, [_i, _i, _i, _i]),
+    "dels_verify_block": (_i, [_vp, _vp, _i, _i, _i, _i, _vp, _vp, _vp, _vp, _sz, _vp]),
+    "dels_read_status": (_i, [_vp, _vp, ctypes.POINTER(ctypes.c_int32)]),
+    "dels_prior_from_counts": (_i, [_vp, _i, _d, _vp]),
+    "dels_status_string": (ctypes.c_char_p, [_i]),
+    "dels_version": (_i, []),
+}
+
+
+def exported_symbols():
+    """Names of the C ABI entry points this binding expects the library to export."""
+    return list(_SIGS)
+
+
+class DelsError(RuntimeError):
+    def __init__(self, code: int, where: str):
+        self.code = code
+        super().__init__(f"{where}: {dels_status_string(code)} ({code})")
+
+
+def library_path() -> str:
+    return _LIB_PATH
+
+
+def lib():
+    """The loaded ``libdels.so`` (raises if it has not been built)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(_LIB_PATH):
+            raise RuntimeError(
+                f"{_LIB_PATH} not found: build it with `python -c 'import __graft_entry__ as g; g.build()'`")
+        L = ctypes.CDLL(_LIB_PATH)
+        for name, (res, args) in _SIGS.items():
+            fn = getattr(L, name)
+            fn.restype = res
+            fn.argtypes = args
+        _lib = L
+    return _lib
+
+
+# ----------------------------------------------------------------------------- marshalling helpers
+
+def _ptr(x) -> Optional[int]:
+    if x is None:
+        return None
+    if isinstance(x, torch.Tensor):
+        return x.data_ptr()
+    return int(x)
+
+
+def _stream(stream) -> Optional[int]:
+    if stream is None:
+        return torch.cuda.current_stream().cuda_stream if torch.cuda.is_available() else None
+    if isinstance(stream, torch.cuda.Stream):
+        return stream.cuda_stream
+    return int(stream)
+
+
+def dtype_code(t) -> int:
+    if isinstance(t, torch.Tensor):
+        t = t.dtype
+    if t == torch.float32:
+        return DELS_F32
+    if t == torch.bfloat16:
+        return DELS_BF16
+    raise ValueError(f"unsupported dtype {t}")
+
+
+def _check(code: int, where: str):
+    if code != DELS_OK:
+        raise DelsError(code, where)
+
+
+# ----------------------------------------------------------------------------- the C ABI, by name
+
+def dels_version() -> int:
+    return lib().dels_version()
+
+
+def dels_status_string(code: int) -> str:
+    return lib().dels_status_string(int(code)).decode()
+
+
+def dels_draft_workspace_bytes(head: LocalHead, B: int, n: int, V: int) -> int:
+    return lib().dels_draft_workspace_bytes(ctypes.byref(head), B, n, V)
+
+
+def dels_draft_block(head: LocalHead, long_logits, logit_dtype: int, log_prior, alpha: float, beta: float,
+                     B: int, n: int, V: int, out_tokens, out_logprob, out_top2_gap, workspace,
+                     workspace_bytes: int, stream=None) -> int:
+    r = lib().dels_draft_block(ctypes.byref(head), _ptr(long_logits), logit_dtype, _ptr(log_prior), alpha, beta,
+                               B, n, V, _ptr(out_tokens), _ptr(out_logprob), _ptr(out_top2_gap),
+                               _ptr(workspace), workspace_bytes, _stream(stream))
+    return r
+
+
+def dels_combine_workspace_bytes(rows: int, V: int, dtype: int) -> int:
+    return lib().dels_combine_workspace_bytes(rows, V, dtype)
+
+
+def dels_combine_argmax(long_logits, short_logits, dtype: int, log_prior, alpha: float, beta: float, rows: int,
+                        V: int, out_token, out_logprob, out_top2_gap, workspace, workspace_bytes: int,
+                        stream=None) -> int:
+    return lib().dels_combine_argmax(_ptr(long_logits), _ptr(short_logits), dtype, _ptr(log_prior), alpha, beta,
+                                     rows, V, _ptr(out_token), _ptr(out_logprob), _ptr(out_top2_gap),
+                                     _ptr(workspace), workspace_bytes, _stream(stream))
+
+
+def dels_verify_workspace_bytes(B: int, n: int, V: int, dtype: int) -> int:
+    return lib().dels_verify_workspace_bytes(B, n, V, dtype)
+
+
+def dels_verify_block(draft_tokens, target_logits, dtype: int, B: int, n: int, V: int, out_accept_len, out_bonus,
+                      out_target_argmax, workspace, workspace_bytes: int, stream=None) -> int:
+    return lib().dels_verify_block(_ptr(draft_tokens), _ptr(target_logits), dtype, B, n, V, _ptr(out_accept_len),
+                                   _ptr(out_bonus), _ptr(out_target_argmax), _ptr(workspace), workspace_bytes,
+                                   _stream(stream))
+
+
+def dels_read_status(workspace, stream=None) -> int:
+    out = ctypes.c_int32(0)
+    _check(lib().dels_read_status(_ptr(workspace), _stream(stream), ctypes.byref(out)), "dels_read_status")
+    return out.value
+
+
+def dels_prior_from_counts(counts: torch.Tensor, lam: float = 1.0) -> torch.Tensor:
+    """Host helper: float32 log prior [V] from int64 counts [V] (both CPU tensors)."""
+    c = counts.detach().to("cpu", torch.int64).contiguous()
+    out = torch.empty(c.numel(), dtype=torch.float32)
+    _check(lib().dels_prior_from_counts(c.data_ptr(), c.numel(), float(lam), out.data_ptr()),
+           "dels_prior_from_counts")
+    return out
+
+
+# ----------------------------------------------------------------------------- conveniences
+
+_KIND = {"gru": DELS_HEAD_GRU, "mlp": DELS_HEAD_MLP, "xfmr": DELS_HEAD_XFMR, "markov": DELS_HEAD_MARKOV}
+_SLOTS = {
+    "gru": ["w_ih", "w_hh", "w_rank"],
+    "mlp": ["w1", "w2"],
+    "xfmr": ["pos", "wq", "wk", "wv", "wo", "w1", "w2"],
+    "markov": [],
+}
+
+
+def make_head(spec, weights: Dict[str, torch.Tensor]) -> LocalHead:
+    """LocalHead for a head spec (``kind``, ``wdtype``, dims) and a dict of device weight tensors
+    (keys emb, w_vocab and the kind's slot names). The caller keeps the tensors alive."""
+    h = LocalHead()
+    h.kind = _KIND[spec.kind]
+    h.wdtype = DELS_BF16 if spec.wdtype == "bf16" else DELS_F32
+    h.d_model, h.d_hidden, h.d_rank = spec.d_model, spec.d_hidden, spec.d_rank
+    h.window, h.n_layers, h.n_heads, h.max_pos = spec.window, spec.n_layers, spec.n_heads, spec.max_pos
+    h.emb = _ptr(weights["emb"])
+    h.w_vocab = _ptr(weights["w_vocab"])
+    for i, name in enumerate(_SLOTS[spec.kind]):
+        if name in weights:
+            h.w[i] = _ptr(weights[name])
+    return h
+
+
+class Drafter:
+    """One local head + one workspace for repeated dels_draft_block calls."""
+
+    def __init__(self, spec, weights: Dict[str, torch.Tensor], B: int, n: int, V: int, device=None):
+        self.spec, self.weights = spec, weights
+        self.head = make_head(spec, weights)
+        self.B, self.n, self.V = B, n, V
+        self.device = device or weights["w_vocab"].device
+        nbytes = dels_draft_workspace_bytes(self.head, B, n, V)
+        if nbytes == 0:
+            raise DelsError(-2, "dels_draft_workspace_bytes")
+        self.ws_bytes = nbytes
+        self.workspace = torch.zeros(nbytes, dtype=torch.uint8, device=self.device)
+        self.tokens = torch.empty(B, n, dtype=torch.int32, device=self.device)
+        self.logprob = torch.empty(B, n, dtype=torch.float32, device=self.device)
+        self.gap = torch.empty(B, n, dtype=torch.float32, device=self.device)
+
+    def __call__(self, long_logits: torch.Tensor, log_prior: torch.Tensor, alpha: float, beta: float, stream=None):
+        _check(dels_draft_block(self.head, long_logits, dtype_code(long_logits), log_prior, alpha, beta, self.B,
+                                self.n, self.V, self.tokens, self.logprob, self.gap, self.workspace, self.ws_bytes,
+                                stream), "dels_draft_block")
+        return self.tokens, self.logprob, self.gap
+
+    def status(self, stream=None) -> int:
+        return dels_read_status(self.workspace, stream)

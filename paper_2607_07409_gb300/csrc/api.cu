@@ -1,0 +1,856 @@
+// C ABI of the drafting hot path: argument validation, workspace layout,
+// TMA descriptor encoding, and the per-block orchestration of Algorithm 1
+// (position 0 from the long logits alone, then local head -> vocabulary
+// projection + fused combine -> merge/feedback for positions 1..n-1).
+#include <algorithm>
+#include <cmath>
+#include <cstring>
+#include <mutex>
+#include <vector>
+
+#include "dels_internal.h"
+
+namespace dels {
+
+// ---------------------------------------------------------------- utilities
+
+int device_sm_count() {
+  int dev = 0, v = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+  if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+  return v;
+}
+
+int device_max_smem_optin() {
+  int dev = 0, v = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+  if (cudaDeviceGetAttribute(&v, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess) return 0;
+  return v;
+}
+
+namespace {
+
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn get_encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q{};
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  });
+  return fn;
+}
+
+inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+inline size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+}  // namespace
+
+bool encode_tmap_2d(CUtensorMap* m, const void* base, CUtensorMapDataType dt, int elem_bytes, uint64_t inner,
+                    uint64_t outer, uint64_t row_pitch_bytes, uint32_t box_inner, uint32_t box_outer,
+                    CUtensorMapSwizzle swz) {
+  EncodeTiledFn fn = get_encode_fn();
+  if (!fn) return false;
+  (void)elem_bytes;
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {row_pitch_bytes};
+  cuuint32_t box[2] = {box_inner, box_outer};
+  cuuint32_t es[2] = {1, 1};
+  return fn(m, dt, 2, const_cast<void*>(base), dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, swz,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+bool encode_tmap_3d(CUtensorMap* m, const void* base, CUtensorMapDataType dt, int elem_bytes, uint64_t d0,
+                    uint64_t d1, uint64_t d2, uint64_t pitch1_bytes, uint64_t pitch2_bytes, uint32_t b0, uint32_t b1,
+                    uint32_t b2, CUtensorMapSwizzle swz) {
+  EncodeTiledFn fn = get_encode_fn();
+  if (!fn) return false;
+  (void)elem_bytes;
+  cuuint64_t dims[3] = {d0, d1, d2};
+  cuuint64_t strides[2] = {pitch1_bytes, pitch2_bytes};
+  cuuint32_t box[3] = {b0, b1, b2};
+  cuuint32_t es[3] = {1, 1, 1};
+  return fn(m, dt, 3, const_cast<void*>(base), dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, swz,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+namespace {
+
+// ------------------------------------------------------------- tcgen05 plans
+
+struct Gemm {
+  TcGemmArgs a{};
+  CUtensorMap mA0{}, mB0{}, mA1{}, mB1{}, mL{};
+  int grid = 0;
+  size_t smem = 0;
+};
+
+constexpr int kSmemReserve = 512 + 2 * 128 * 16 + 1024 + 256;   // barriers, reduction scratch, alignment slack
+
+// A = X [B, K] bf16 (row pitch K*2); W = [O, K] bf16.
+bool map_x(CUtensorMap* m, const void* X, int B, int K) {
+  return encode_tmap_2d(m, X, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (uint64_t)K, (uint64_t)B, (uint64_t)K * 2, 64,
+                        128, CU_TENSOR_MAP_SWIZZLE_128B);
+}
+bool map_w(CUtensorMap* m, const void* W, int O, int K, int n_tile) {
+  return encode_tmap_2d(m, W, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (uint64_t)K, (uint64_t)O, (uint64_t)K * 2, 64,
+                        (uint32_t)n_tile, CU_TENSOR_MAP_SWIZZLE_128B);
+}
+
+int pick_stages(const TcGemmArgs& a, int per_stage, int fixed) {
+  const int budget = device_max_smem_optin() - kSmemReserve - fixed;
+  int st = budget / per_stage;
+  return std::max(2, std::min(st, 12));
+}
+
+// Y = act(X0 W0^T) over K split into `splits` pieces (segment 1 optional:
+// + X1 W1^T with its own splits, written as separate partials).
+bool plan_store(Gemm& g, int B, int O, const void* X0, const void* W0, int K0, const void* X1, const void* W1,
+                int K1, int n_tile, int splits0, int splits1, int act, float* out_f32, uint16_t* out_bf16,
+                int ldo_bf16, int* status, int sms) {
+  TcGemmArgs& a = g.a;
+  a.B = B;
+  a.O = O;
+  a.n_tile = n_tile;
+  a.num_o_tiles = (O + n_tile - 1) / n_tile;
+  a.seg_chunks[0] = (K0 + 63) / 64;
+  a.seg_chunks[1] = K1 > 0 ? (K1 + 63) / 64 : 0;
+  // make every split non-empty
+  auto fix = [](int nch, int s) {
+    if (nch == 0) return 0;
+    s = std::max(1, std::min(s, nch));
+    const int per = (nch + s - 1) / s;
+    return (nch + per - 1) / per;
+  };
+  a.seg_splits[0] = fix(a.seg_chunks[0], splits0);
+  a.seg_splits[1] = fix(a.seg_chunks[1], splits1);
+  a.total_splits = a.seg_splits[0] + a.seg_splits[1];
+  a.epi = EPI_STORE;
+  a.a_resident = 0;
+  a.act = act;
+  a.out_f32 = out_f32;
+  a.out_split_stride = (long long)B * O;
+  a.ldo = O;
+  a.out_bf16 = out_bf16;
+  a.ldo_bf16 = ldo_bf16;
+  a.status = status;
+  a.stages = pick_stages(a, 128 * 128 + n_tile * 128, 0);
+  if (!map_x(&g.mA0, X0, B, K0) || !map_w(&g.mB0, W0, O, K0, n_tile)) return false;
+  if (K1 > 0) {
+    if (!map_x(&g.mA1, X1, B, K1) || !map_w(&g.mB1, W1, O, K1, n_tile)) return false;
+  } else {
+    g.mA1 = g.mA0;
+    g.mB1 = g.mB0;
+  }
+  g.mL = g.mA0;
+  const int items = a.num_o_tiles * a.total_splits;
+  g.grid = std::min(items, std::max(1, sms));
+  g.smem = tc_gemm_smem_bytes(a);
+  return true;
+}
+
+// Splits so that tiles x splits roughly fills the GPU once.
+int splits_for(int O, int n_tile, int K, int sms) {
+  const int tiles = (O + n_tile - 1) / n_tile;
+  const int nch = (K + 63) / 64;
+  int s = std::max(1, sms / std::max(1, tiles));
+  return std::min(s, nch);
+}
+
+// Vocabulary projection fused with the combine (l_L tile of position j).
+bool plan_combine(Gemm& g, int B, int V, int n, const void* X, int K, const void* Wv, const void* longp,
+                  dels_dtype ldt, const float* prior, float alpha, float beta, void* partials, int partial_ld,
+                  int* status, int sms) {
+  TcGemmArgs& a = g.a;
+  const int n_tile = 128;
+  a.B = B;
+  a.O = V;
+  a.V = V;
+  a.n_tile = n_tile;
+  a.num_o_tiles = (V + n_tile - 1) / n_tile;
+  a.seg_chunks[0] = (K + 63) / 64;
+  a.seg_chunks[1] = 0;
+  a.seg_splits[0] = 1;
+  a.seg_splits[1] = 0;
+  a.total_splits = 1;
+  a.epi = EPI_COMBINE;
+  a.prior = prior;
+  a.alpha = alpha;
+  a.beta = beta;
+  a.long_f32 = (ldt == DELS_F32);
+  a.l_box_cols = a.long_f32 ? 32 : 64;
+  a.l_box_rows = std::min(128, (B + 7) / 8 * 8);
+  a.l_boxes = n_tile / a.l_box_cols;
+  a.partials = partials;
+  a.partial_ld = partial_ld;
+  a.status = status;
+  const int l_fixed = 2 * a.l_boxes * a.l_box_rows * 128;
+  a.a_resident = (a.seg_chunks[0] <= 4) ? 1 : 0;
+  if (a.a_resident) {
+    a.stages = pick_stages(a, n_tile * 128, a.seg_chunks[0] * 128 * 128 + l_fixed);
+  } else {
+    a.stages = pick_stages(a, 128 * 128 + n_tile * 128, l_fixed);
+  }
+  const int es = a.long_f32 ? 4 : 2;
+  if (!map_x(&g.mA0, X, B, K) || !map_w(&g.mB0, Wv, V, K, n_tile)) return false;
+  if (!encode_tmap_3d(&g.mL, longp, a.long_f32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16,
+                      es, (uint64_t)V, (uint64_t)n, (uint64_t)B, (uint64_t)V * es, (uint64_t)n * V * es,
+                      (uint32_t)a.l_box_cols, 1, (uint32_t)a.l_box_rows, CU_TENSOR_MAP_SWIZZLE_128B))
+    return false;
+  g.mA1 = g.mA0;
+  g.mB1 = g.mB0;
+  g.grid = std::min(a.num_o_tiles, std::max(1, sms));
+  g.smem = tc_gemm_smem_bytes(a);
+  return true;
+}
+
+cudaError_t run(const Gemm& g, cudaStream_t s) {
+  return launch_tc_gemm(g.a, &g.mA0, &g.mB0, &g.mA1, &g.mB1, &g.mL, g.grid, g.smem, s);
+}
+
+// ------------------------------------------------------------ draft layout
+
+struct Carve {
+  size_t off = kHeaderBytes;
+  size_t take(size_t bytes) {
+    const size_t o = off;
+    off = round_up(off + bytes, 256);
+    return o;
+  }
+};
+
+struct DraftLayout {
+  bool ok = false;
+  int sms = 0;
+  int partial_ld = 0;
+  size_t partials = 0;
+  // GRU
+  size_t eg = 0, h = 0, hb = 0, gpart = 0, r = 0;
+  int gru_s0 = 0, gru_s1 = 0;
+  // MLP
+  size_t u = 0, mpart = 0, h1 = 0, h2 = 0;
+  int mlp_s1 = 0, mlp_s2 = 0;
+  // XFMR
+  size_t ex = 0, t = 0, ab = 0, q = 0, kc = 0, vc = 0, xpart = 0, ob = 0, uu = 0, anb = 0, fb = 0, y = 0, feat = 0;
+  int xs_qkv = 0, xs_o = 0, xs_1 = 0, xs_2 = 0;
+  // MARKOV
+  size_t mk = 0;
+  size_t total = 0;
+};
+
+int head_es(const dels_local_head* h) { return h->wdtype == DELS_F32 ? 4 : 2; }
+
+DraftLayout draft_layout(const dels_local_head* hd, int B, int n, int V) {
+  DraftLayout L;
+  L.sms = device_sm_count();
+  if (L.sms <= 0) return L;
+  const int sms = L.sms;
+  Carve c;
+  L.partial_ld = std::max(sms, 16 * sms / std::max(1, B) + 1);
+  L.partials = c.take((size_t)B * L.partial_ld * 16);
+  const int es = head_es(hd);
+  const bool bf = hd->wdtype == DELS_BF16;
+  switch (hd->kind) {
+    case DELS_HEAD_GRU: {
+      const int D = hd->d_model, H = hd->d_hidden, R = hd->d_rank;
+      L.eg = c.take((size_t)B * D * es);
+      L.h = c.take((size_t)B * H * 4);
+      L.hb = c.take((size_t)B * H * 2);
+      if (bf) {
+        L.gru_s0 = std::max(1, std::min((D + 63) / 64, sms / std::max(1, (3 * H + 127) / 128) - 1));
+        L.gru_s1 = 1;
+      } else {
+        L.gru_s0 = 1;
+        L.gru_s1 = 1;
+      }
+      L.gpart = c.take((size_t)(L.gru_s0 + L.gru_s1) * B * 3 * H * 4);
+      L.r = c.take((size_t)B * R * es);
+      break;
+    }
+    case DELS_HEAD_MLP: {
+      const int D = hd->d_model, Hd = hd->d_hidden, W = hd->window;
+      L.u = c.take((size_t)B * W * D * es);
+      L.mlp_s1 = bf ? splits_for(Hd, 128, W * D, sms) : 1;
+      L.mlp_s2 = bf ? splits_for(Hd, 128, Hd, sms) : 1;
+      L.mpart = c.take((size_t)std::max(L.mlp_s1, L.mlp_s2) * B * Hd * 4);
+      L.h1 = c.take((size_t)B * Hd * es);
+      L.h2 = c.take((size_t)B * Hd * es);
+      break;
+    }
+    case DELS_HEAD_XFMR: {
+      const int D = hd->d_model, F = hd->d_hidden, P = hd->max_pos;
+      L.ex = c.take((size_t)B * D * 2);
+      L.t = c.take((size_t)B * D * 4);
+      L.ab = c.take((size_t)B * D * 2);
+      L.q = c.take((size_t)B * D * 4);
+      L.kc = c.take((size_t)B * P * D * 4);
+      L.vc = c.take((size_t)B * P * D * 4);
+      L.xs_qkv = splits_for(D, 128, D, sms);
+      L.xs_o = splits_for(D, 128, D, sms);
+      L.xs_1 = splits_for(F, 128, D, sms);
+      L.xs_2 = splits_for(D, 128, F, sms);
+      const int smax = std::max(std::max(L.xs_qkv, L.xs_o), std::max(L.xs_1, L.xs_2));
+      L.xpart = c.take((size_t)smax * B * std::max(D, F) * 4);
+      L.ob = c.take((size_t)B * D * 2);
+      L.uu = c.take((size_t)B * D * 4);
+      L.anb = c.take((size_t)B * D * 2);
+      L.fb = c.take((size_t)B * F * 2);
+      L.y = c.take((size_t)B * D * 4);
+      L.feat = c.take((size_t)B * D * 2);
+      break;
+    }
+    case DELS_HEAD_MARKOV: {
+      L.mk = c.take((size_t)B * hd->d_rank * es);
+      break;
+    }
+    default:
+      return L;
+  }
+  L.total = c.off;
+  L.ok = true;
+  return L;
+}
+
+int validate_head(const dels_local_head* h, int n) {
+  if (!h) return DELS_ERR_NULL_POINTER;
+  if (h->wdtype != DELS_F32 && h->wdtype != DELS_BF16) return DELS_ERR_BAD_DTYPE;
+  const bool bf = h->wdtype == DELS_BF16;
+  auto dim_ok = [&](int d) { return d > 0 && d <= 65536 && (!bf || d % 16 == 0) && (bf || d % 4 == 0); };
+  if (!h->emb || !h->w_vocab) return DELS_ERR_NULL_POINTER;
+  if (!aligned16(h->emb) || !aligned16(h->w_vocab)) return DELS_ERR_ALIGNMENT;
+  for (int i = 0; i < 8; ++i)
+    if (h->w[i] && !aligned16(h->w[i])) return DELS_ERR_ALIGNMENT;
+  switch (h->kind) {
+    case DELS_HEAD_GRU:
+      if (!h->w[0] || !h->w[1] || !h->w[2]) return DELS_ERR_NULL_POINTER;
+      if (!dim_ok(h->d_model) || !dim_ok(h->d_hidden) || !dim_ok(h->d_rank)) return DELS_ERR_BAD_SHAPE;
+      if (h->d_rank > 4096) return DELS_ERR_BAD_SHAPE;
+      return DELS_OK;
+    case DELS_HEAD_MLP:
+      if (!h->w[0] || (h->n_layers == 2 && !h->w[1])) return DELS_ERR_NULL_POINTER;
+      if (h->n_layers != 1 && h->n_layers != 2) return DELS_ERR_BAD_SHAPE;
+      if (h->window < 1 || h->window > 32) return DELS_ERR_BAD_SHAPE;
+      if (!dim_ok(h->d_model) || !dim_ok(h->d_hidden) || h->d_rank != h->d_hidden) return DELS_ERR_BAD_SHAPE;
+      return DELS_OK;
+    case DELS_HEAD_XFMR:
+      if (!bf) return DELS_ERR_UNSUPPORTED;
+      for (int i = 0; i < 7; ++i)
+        if (!h->w[i]) return DELS_ERR_NULL_POINTER;
+      if (!dim_ok(h->d_model) || !dim_ok(h->d_hidden) || h->d_rank != h->d_model) return DELS_ERR_BAD_SHAPE;
+      if (h->n_heads < 1 || h->d_model % h->n_heads != 0 || h->max_pos < n) return DELS_ERR_BAD_SHAPE;
+      return DELS_OK;
+    case DELS_HEAD_MARKOV:
+      if (!dim_ok(h->d_rank)) return DELS_ERR_BAD_SHAPE;
+      return DELS_OK;
+    default:
+      return DELS_ERR_UNSUPPORTED;
+  }
+}
+
+int validate_draft(const dels_local_head* head, const void* long_logits, dels_dtype ldt, const float* prior, int B,
+                   int n, int V, const int32_t* tok, const float* lp, const float* gap) {
+  if (B < 0 || B > kMaxBatchTile) return DELS_ERR_BAD_SHAPE;
+  if (n < 1 || n > 32) return DELS_ERR_BAD_SHAPE;
+  if (V < 8 || V % 8 != 0) return DELS_ERR_BAD_SHAPE;
+  if (ldt != DELS_F32 && ldt != DELS_BF16) return DELS_ERR_BAD_DTYPE;
+  int r = validate_head(head, n);
+  if (r != DELS_OK) return r;
+  if (B == 0) return DELS_OK;
+  if (!long_logits || !prior || !tok || !lp) return DELS_ERR_NULL_POINTER;
+  if (!aligned16(long_logits) || !aligned16(prior) || !aligned16(tok) || !aligned16(lp) || (gap && !aligned16(gap)))
+    return DELS_ERR_ALIGNMENT;
+  return DELS_OK;
+}
+
+#define DELS_CUDA(call)                        \
+  do {                                         \
+    cudaError_t e__ = (call);                  \
+    if (e__ != cudaSuccess) return DELS_ERR_CUDA; \
+  } while (0)
+
+template <typename T>
+T* at(void* ws, size_t off) {
+  return reinterpret_cast<T*>(static_cast<uint8_t*>(ws) + off);
+}
+
+// Position 0: x_0 = argmax l_L[b, 0, :], partials then merge (+ gather).
+int draft_position0(const void* long_logits, dels_dtype ldt, int B, int n, int V, void* partials, int partial_ld,
+                    int* status, const MergeArgs& merge_base, int sms, cudaStream_t s) {
+  RowsArgs a{};
+  const int es = ldt == DELS_F32 ? 4 : 2;
+  RowsPlan p = plan_rows(B, V, es, sms, true, partial_ld);
+  a.longp = long_logits;
+  a.rows = B;
+  a.V = V;
+  a.ld_long = (long long)n * V;
+  a.chunk_cols = p.chunk_cols;
+  a.nchunks = p.nchunks;
+  a.rows_per_cta = 1;
+  a.partials = partials;
+  a.partial_ld = partial_ld;
+  a.status = status;
+  DELS_CUDA(launch_combine_rows(a, ldt, true, false, s));
+  MergeArgs m = merge_base;
+  m.count = p.nchunks;
+  m.j = 0;
+  DELS_CUDA(launch_draft_merge(m, s));
+  return DELS_OK;
+}
+
+}  // namespace
+}  // namespace dels
+
+using namespace dels;
+
+extern "C" {
+
+int dels_version(void) { return 100; }
+
+const char* dels_status_string(int code) {
+  switch (code) {
+    case DELS_OK: return "ok";
+    case DELS_ERR_NULL_POINTER: return "null pointer";
+    case DELS_ERR_BAD_SHAPE: return "size out of supported range";
+    case DELS_ERR_BAD_DTYPE: return "unsupported dtype";
+    case DELS_ERR_ALIGNMENT: return "pointer or pitch not 16-byte aligned";
+    case DELS_ERR_WORKSPACE: return "workspace missing or too small";
+    case DELS_ERR_UNSUPPORTED: return "unsupported head configuration";
+    case DELS_ERR_CUDA: return "CUDA call failed";
+    case DELS_STATUS_NONFINITE: return "device: non-finite logits";
+    case DELS_STATUS_TIMEOUT: return "device: bounded wait expired";
+    case DELS_STATUS_BAD_TOKEN: return "device: draft token out of range";
+    default: return "unknown status";
+  }
+}
+
+int dels_prior_from_counts(const int64_t* counts, int V, double lambda, float* out_log_prior) {
+  if (!counts || !out_log_prior) return DELS_ERR_NULL_POINTER;
+  if (V < 1 || !(lambda > 0.0)) return DELS_ERR_BAD_SHAPE;
+  long double total = 0.0L;
+  for (int v = 0; v < V; ++v) {
+    if (counts[v] < 0) return DELS_ERR_BAD_SHAPE;
+    total += (long double)counts[v] + (long double)lambda;
+  }
+  for (int v = 0; v < V; ++v) {
+    const double p = (double)(((long double)counts[v] + (long double)lambda) / total);
+    out_log_prior[v] = (float)std::log(p);
+  }
+  return DELS_OK;
+}
+
+int dels_read_status(void* workspace, dels_stream_t stream, int32_t* out_status) {
+  if (!workspace || !out_status) return DELS_ERR_NULL_POINTER;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  int32_t v = 0;
+  if (cudaMemcpyAsync(&v, workspace, sizeof(v), cudaMemcpyDeviceToHost, s) != cudaSuccess) return DELS_ERR_CUDA;
+  if (cudaStreamSynchronize(s) != cudaSuccess) return DELS_ERR_CUDA;
+  if (cudaMemsetAsync(workspace, 0, sizeof(v), s) != cudaSuccess) return DELS_ERR_CUDA;
+  *out_status = v;
+  return DELS_OK;
+}
+
+// ----------------------------------------------------------------- combine
+
+size_t dels_combine_workspace_bytes(int rows, int V, dels_dtype dtype) {
+  if (rows < 0 || V < 1 || (dtype != DELS_F32 && dtype != DELS_BF16)) return 0;
+  const int sms = device_sm_count();
+  if (sms <= 0) return 0;
+  const int es = dtype == DELS_F32 ? 4 : 2;
+  const bool vec = (V % (16 / es)) == 0;
+  RowsPlan p = plan_rows(rows, V, 2 * es, sms, vec, 1 << 20);
+  const size_t groups = ((size_t)rows + p.rows_per_cta - 1) / p.rows_per_cta;
+  size_t off = kHeaderBytes;
+  off = round_up(off + groups * 4, 256);
+  off = round_up(off + (size_t)rows * p.nchunks * 16, 256);
+  return off;
+}
+
+int dels_combine_argmax(const void* long_logits, const void* short_logits, dels_dtype dtype, const float* log_prior,
+                        float alpha, float beta, int rows, int V, int32_t* out_token, float* out_logprob,
+                        float* out_top2_gap, void* workspace, size_t workspace_bytes, dels_stream_t stream) {
+  if (dtype != DELS_F32 && dtype != DELS_BF16) return DELS_ERR_BAD_DTYPE;
+  if (rows < 0 || V < 1) return DELS_ERR_BAD_SHAPE;
+  if (!workspace) return DELS_ERR_WORKSPACE;
+  if (rows == 0) return DELS_OK;
+  if (!long_logits || !out_token) return DELS_ERR_NULL_POINTER;
+  if (!aligned16(long_logits) || (short_logits && !aligned16(short_logits)) || (log_prior && !aligned16(log_prior)) ||
+      !aligned16(workspace))
+    return DELS_ERR_ALIGNMENT;
+  const size_t need = dels_combine_workspace_bytes(rows, V, dtype);
+  if (need == 0) return DELS_ERR_CUDA;
+  if (workspace_bytes < need) return DELS_ERR_WORKSPACE;
+  const int sms = device_sm_count();
+  const int es = dtype == DELS_F32 ? 4 : 2;
+  const bool vec = (V % (16 / es)) == 0;
+  RowsPlan p = plan_rows(rows, V, 2 * es, sms, vec, 1 << 20);
+  const size_t groups = ((size_t)rows + p.rows_per_cta - 1) / p.rows_per_cta;
+  RowsArgs a{};
+  a.longp = long_logits;
+  a.shortp = short_logits;
+  a.prior = log_prior;
+  a.alpha = alpha;
+  a.beta = beta;
+  a.rows = rows;
+  a.V = V;
+  a.ld_long = V;
+  a.ld_short = V;
+  a.chunk_cols = p.chunk_cols;
+  a.nchunks = p.nchunks;
+  a.rows_per_cta = p.rows_per_cta;
+  a.counters = at<int>(workspace, kHeaderBytes);
+  a.partials = at<void>(workspace, round_up(kHeaderBytes + groups * 4, 256));
+  a.partial_ld = p.nchunks;
+  a.out_token = out_token;
+  a.out_lp = out_logprob;
+  a.out_gap = out_top2_gap;
+  a.status = at<int>(workspace, 0);
+  if (launch_combine_rows(a, dtype, vec, true, reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess)
+    return DELS_ERR_CUDA;
+  return DELS_OK;
+}
+
+// ------------------------------------------------------------------ verify
+
+size_t dels_verify_workspace_bytes(int B, int n, int V, dels_dtype dtype) {
+  if (B < 0 || n < 1 || n > 1024 || V < 1 || (dtype != DELS_F32 && dtype != DELS_BF16)) return 0;
+  const int sms = device_sm_count();
+  if (sms <= 0) return 0;
+  const int es = dtype == DELS_F32 ? 4 : 2;
+  const bool vec = (V % (16 / es)) == 0;
+  const size_t rows = (size_t)B * (n + 1);
+  RowsPlan p = plan_rows((int)std::min<size_t>(rows, INT32_MAX), V, es, sms, vec, 1 << 20);
+  size_t off = kHeaderBytes;
+  off = round_up(off + rows * 4, 256);        // per-row tickets
+  off = round_up(off + (size_t)B * 4, 256);   // per-request tickets
+  off = round_up(off + rows * 4, 256);        // target argmax scratch
+  off = round_up(off + rows * p.nchunks * 16, 256);
+  return off;
+}
+
+int dels_verify_block(const int32_t* draft_tokens, const void* target_logits, dels_dtype dtype, int B, int n, int V,
+                      int32_t* out_accept_len, int32_t* out_bonus, int32_t* out_target_argmax, void* workspace,
+                      size_t workspace_bytes, dels_stream_t stream) {
+  if (dtype != DELS_F32 && dtype != DELS_BF16) return DELS_ERR_BAD_DTYPE;
+  if (B < 0 || n < 1 || n > 1024 || V < 1) return DELS_ERR_BAD_SHAPE;
+  if ((long long)B * (n + 1) > INT32_MAX) return DELS_ERR_BAD_SHAPE;
+  if (!workspace) return DELS_ERR_WORKSPACE;
+  if (B == 0) return DELS_OK;
+  if (!draft_tokens || !target_logits || !out_accept_len || !out_bonus) return DELS_ERR_NULL_POINTER;
+  if (!aligned16(target_logits) || !aligned16(workspace)) return DELS_ERR_ALIGNMENT;
+  const size_t need = dels_verify_workspace_bytes(B, n, V, dtype);
+  if (need == 0) return DELS_ERR_CUDA;
+  if (workspace_bytes < need) return DELS_ERR_WORKSPACE;
+  const int sms = device_sm_count();
+  const int es = dtype == DELS_F32 ? 4 : 2;
+  const bool vec = (V % (16 / es)) == 0;
+  const size_t rows = (size_t)B * (n + 1);
+  RowsPlan p = plan_rows((int)rows, V, es, sms, vec, 1 << 20);
+  RowsArgs a{};
+  a.longp = target_logits;
+  a.rows = (int)rows;
+  a.V = V;
+  a.ld_long = V;
+  a.chunk_cols = p.chunk_cols;
+  a.nchunks = p.nchunks;
+  a.rows_per_cta = 1;
+  size_t off = kHeaderBytes;
+  a.counters = at<int>(workspace, off);
+  off = round_up(off + rows * 4, 256);
+  a.counters_b = at<int>(workspace, off);
+  off = round_up(off + (size_t)B * 4, 256);
+  a.targ_scratch = at<int32_t>(workspace, off);
+  off = round_up(off + rows * 4, 256);
+  a.partials = at<void>(workspace, off);
+  a.partial_ld = p.nchunks;
+  a.out_token = out_target_argmax;
+  a.draft = draft_tokens;
+  a.n = n;
+  a.out_accept = out_accept_len;
+  a.out_bonus = out_bonus;
+  a.status = at<int>(workspace, 0);
+  if (launch_verify_rows(a, dtype, vec, reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess) return DELS_ERR_CUDA;
+  return DELS_OK;
+}
+
+// ------------------------------------------------------------------- draft
+
+size_t dels_draft_workspace_bytes(const dels_local_head* head, int B, int n, int V) {
+  if (validate_head(head, n) != DELS_OK || B < 0 || B > kMaxBatchTile || n < 1 || n > 32 || V < 8 || V % 8)
+    return 0;
+  DraftLayout L = draft_layout(head, std::max(B, 1), n, V);
+  return L.ok ? L.total : 0;
+}
+
+int dels_draft_block(const dels_local_head* head, const void* long_logits, dels_dtype logit_dtype,
+                     const float* log_prior, float alpha, float beta, int B, int n, int V, int32_t* out_tokens,
+                     float* out_logprob, float* out_top2_gap, void* workspace, size_t workspace_bytes,
+                     dels_stream_t stream) {
+  int r = validate_draft(head, long_logits, logit_dtype, log_prior, B, n, V, out_tokens, out_logprob, out_top2_gap);
+  if (r != DELS_OK) return r;
+  if (!workspace) return DELS_ERR_WORKSPACE;
+  if (B == 0) return DELS_OK;
+  if (!aligned16(workspace)) return DELS_ERR_ALIGNMENT;
+  DraftLayout L = draft_layout(head, B, n, V);
+  if (!L.ok) return DELS_ERR_CUDA;
+  if (workspace_bytes < L.total) return DELS_ERR_WORKSPACE;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const int sms = L.sms;
+  const bool bf = head->wdtype == DELS_BF16;
+  const int es = bf ? 2 : 4;
+  int* status = at<int>(workspace, 0);
+  void* partials = at<void>(workspace, L.partials);
+
+  MergeArgs mb{};
+  mb.partials = partials;
+  mb.partial_ld = L.partial_ld;
+  mb.B = B;
+  mb.n = n;
+  mb.tokens = out_tokens;
+  mb.out_lp = out_logprob;
+  mb.out_gap = out_top2_gap;
+  mb.status = status;
+  mb.table = head->emb;
+  mb.table_f32 = bf ? 0 : 1;
+  mb.window = 1;
+
+  switch (head->kind) {
+    case DELS_HEAD_GRU: {
+      const int D = head->d_model, H = head->d_hidden, R = head->d_rank;
+      void* eg = at<void>(workspace, L.eg);
+      float* h = at<float>(workspace, L.h);
+      uint16_t* hb = at<uint16_t>(workspace, L.hb);
+      float* gpart = at<float>(workspace, L.gpart);
+      void* rr = at<void>(workspace, L.r);
+      mb.D = D;
+      mb.dest = eg;
+      DELS_CUDA(cudaMemsetAsync(h, 0, (size_t)B * H * 4, s));
+      DELS_CUDA(cudaMemsetAsync(hb, 0, (size_t)B * H * 2, s));
+      r = draft_position0(long_logits, logit_dtype, B, n, V, partials, L.partial_ld, status, mb, sms, s);
+      if (r != DELS_OK || n == 1) return r;
+      if (bf) {
+        Gemm gg, gr, gv;
+        if (!plan_store(gg, B, 3 * H, eg, head->w[0], D, hb, head->w[1], H, 128, L.gru_s0, L.gru_s1, ACT_NONE,
+                        gpart, nullptr, 0, status, sms))
+          return DELS_ERR_CUDA;
+        if (!plan_store(gr, B, R, hb, head->w[2], H, nullptr, nullptr, 0, 32, 1, 0, ACT_SILU, nullptr,
+                        static_cast<uint16_t*>(rr), R, status, sms))
+          return DELS_ERR_CUDA;
+        if (!plan_combine(gv, B, V, n, rr, R, head->w_vocab, long_logits, logit_dtype, log_prior, alpha, beta,
+                          partials, L.partial_ld, status, sms))
+          return DELS_ERR_CUDA;
+        for (int j = 1; j < n; ++j) {
+          DELS_CUDA(run(gg, s));
+          DELS_CUDA(launch_gru_gates(gpart, gg.a.seg_splits[0], gg.a.seg_splits[1], B, H, h, hb, s));
+          DELS_CUDA(run(gr, s));
+          gv.a.j = j;
+          DELS_CUDA(run(gv, s));
+          MergeArgs m = mb;
+          m.count = gv.grid;
+          m.j = j;
+          if (j == n - 1) m.table = nullptr;
+          DELS_CUDA(launch_draft_merge(m, s));
+        }
+      } else {
+        const float* E = static_cast<const float*>(eg);
+        const float* Wih = static_cast<const float*>(head->w[0]);
+        const float* Whh = static_cast<const float*>(head->w[1]);
+        const float* Wr = static_cast<const float*>(head->w[2]);
+        float* feat = static_cast<float*>(rr);
+        const int nch = std::max(1, std::min(L.partial_ld, (V + 255) / 256));
+        for (int j = 1; j < n; ++j) {
+          DELS_CUDA(launch_gemv_f32(E, D, Wih, B, 3 * H, D, ACT_NONE, gpart, 3 * H, s));
+          DELS_CUDA(launch_gemv_f32(h, H, Whh, B, 3 * H, H, ACT_NONE, gpart + (size_t)B * 3 * H, 3 * H, s));
+          DELS_CUDA(launch_gru_gates(gpart, 1, 1, B, H, h, hb, s));
+          DELS_CUDA(launch_gemv_f32(h, H, Wr, B, R, H, ACT_SILU, feat, R, s));
+          DELS_CUDA(launch_vocab_combine_f32(feat, R, static_cast<const float*>(head->w_vocab),
+                                             static_cast<const uint8_t*>(long_logits) +
+                                                 (size_t)j * V * (logit_dtype == DELS_F32 ? 4 : 2),
+                                             logit_dtype == DELS_F32, (long long)n * V, log_prior, alpha, beta, B, V,
+                                             partials, L.partial_ld, nch, status, s));
+          MergeArgs m = mb;
+          m.count = nch;
+          m.j = j;
+          if (j == n - 1) m.table = nullptr;
+          DELS_CUDA(launch_draft_merge(m, s));
+        }
+      }
+      return DELS_OK;
+    }
+    case DELS_HEAD_MLP: {
+      const int D = head->d_model, Hd = head->d_hidden, W = head->window, K1 = W * D;
+      void* u = at<void>(workspace, L.u);
+      float* mpart = at<float>(workspace, L.mpart);
+      void* h1 = at<void>(workspace, L.h1);
+      void* h2 = at<void>(workspace, L.h2);
+      void* feat = head->n_layers == 2 ? h2 : h1;
+      mb.D = D;
+      mb.window = W;
+      mb.dest = u;
+      r = draft_position0(long_logits, logit_dtype, B, n, V, partials, L.partial_ld, status, mb, sms, s);
+      if (r != DELS_OK || n == 1) return r;
+      if (bf) {
+        Gemm g1, g2, gv;
+        if (!plan_store(g1, B, Hd, u, head->w[0], K1, nullptr, nullptr, 0, 128, L.mlp_s1, 0, ACT_NONE, mpart,
+                        nullptr, 0, status, sms))
+          return DELS_ERR_CUDA;
+        if (head->n_layers == 2 &&
+            !plan_store(g2, B, Hd, h1, head->w[1], Hd, nullptr, nullptr, 0, 128, L.mlp_s2, 0, ACT_NONE, mpart,
+                        nullptr, 0, status, sms))
+          return DELS_ERR_CUDA;
+        if (!plan_combine(gv, B, V, n, feat, Hd, head->w_vocab, long_logits, logit_dtype, log_prior, alpha, beta,
+                          partials, L.partial_ld, status, sms))
+          return DELS_ERR_CUDA;
+        for (int j = 1; j < n; ++j) {
+          DELS_CUDA(run(g1, s));
+          DELS_CUDA(launch_splitk_finish(mpart, g1.a.total_splits, B, Hd, nullptr, ACT_GELU, nullptr, 0,
+                                         static_cast<uint16_t*>(h1), Hd, s));
+          if (head->n_layers == 2) {
+            DELS_CUDA(run(g2, s));
+            DELS_CUDA(launch_splitk_finish(mpart, g2.a.total_splits, B, Hd, nullptr, ACT_GELU, nullptr, 0,
+                                           static_cast<uint16_t*>(h2), Hd, s));
+          }
+          gv.a.j = j;
+          DELS_CUDA(run(gv, s));
+          MergeArgs m = mb;
+          m.count = gv.grid;
+          m.j = j;
+          if (j == n - 1) m.table = nullptr;
+          DELS_CUDA(launch_draft_merge(m, s));
+        }
+      } else {
+        const int nch = std::max(1, std::min(L.partial_ld, (V + 255) / 256));
+        for (int j = 1; j < n; ++j) {
+          DELS_CUDA(launch_gemv_f32(static_cast<const float*>(u), K1, static_cast<const float*>(head->w[0]), B, Hd,
+                                    K1, ACT_GELU, static_cast<float*>(h1), Hd, s));
+          if (head->n_layers == 2)
+            DELS_CUDA(launch_gemv_f32(static_cast<const float*>(h1), Hd, static_cast<const float*>(head->w[1]), B,
+                                      Hd, Hd, ACT_GELU, static_cast<float*>(h2), Hd, s));
+          DELS_CUDA(launch_vocab_combine_f32(static_cast<const float*>(feat), Hd,
+                                             static_cast<const float*>(head->w_vocab),
+                                             static_cast<const uint8_t*>(long_logits) +
+                                                 (size_t)j * V * (logit_dtype == DELS_F32 ? 4 : 2),
+                                             logit_dtype == DELS_F32, (long long)n * V, log_prior, alpha, beta, B, V,
+                                             partials, L.partial_ld, nch, status, s));
+          MergeArgs m = mb;
+          m.count = nch;
+          m.j = j;
+          if (j == n - 1) m.table = nullptr;
+          DELS_CUDA(launch_draft_merge(m, s));
+        }
+      }
+      return DELS_OK;
+    }
+    case DELS_HEAD_XFMR: {
+      const int D = head->d_model, F = head->d_hidden, P = head->max_pos, NH = head->n_heads;
+      uint16_t* ex = at<uint16_t>(workspace, L.ex);
+      float* t = at<float>(workspace, L.t);
+      uint16_t* ab = at<uint16_t>(workspace, L.ab);
+      float* q = at<float>(workspace, L.q);
+      float* kc = at<float>(workspace, L.kc);
+      float* vc = at<float>(workspace, L.vc);
+      float* xpart = at<float>(workspace, L.xpart);
+      uint16_t* ob = at<uint16_t>(workspace, L.ob);
+      float* uu = at<float>(workspace, L.uu);
+      uint16_t* anb = at<uint16_t>(workspace, L.anb);
+      uint16_t* fb = at<uint16_t>(workspace, L.fb);
+      float* y = at<float>(workspace, L.y);
+      uint16_t* feat = at<uint16_t>(workspace, L.feat);
+      mb.D = D;
+      mb.dest = ex;
+      r = draft_position0(long_logits, logit_dtype, B, n, V, partials, L.partial_ld, status, mb, sms, s);
+      if (r != DELS_OK || n == 1) return r;
+      Gemm gq, gk, gvv, go, g1, g2, gv;
+      bool ok = plan_store(gq, B, D, ab, head->w[1], D, nullptr, nullptr, 0, 128, L.xs_qkv, 0, ACT_NONE, xpart,
+                           nullptr, 0, status, sms) &&
+                plan_store(gk, B, D, ab, head->w[2], D, nullptr, nullptr, 0, 128, L.xs_qkv, 0, ACT_NONE, xpart,
+                           nullptr, 0, status, sms) &&
+                plan_store(gvv, B, D, ab, head->w[3], D, nullptr, nullptr, 0, 128, L.xs_qkv, 0, ACT_NONE, xpart,
+                           nullptr, 0, status, sms) &&
+                plan_store(go, B, D, ob, head->w[4], D, nullptr, nullptr, 0, 128, L.xs_o, 0, ACT_NONE, xpart,
+                           nullptr, 0, status, sms) &&
+                plan_store(g1, B, F, anb, head->w[5], D, nullptr, nullptr, 0, 128, L.xs_1, 0, ACT_NONE, xpart,
+                           nullptr, 0, status, sms) &&
+                plan_store(g2, B, D, fb, head->w[6], F, nullptr, nullptr, 0, 128, L.xs_2, 0, ACT_NONE, xpart,
+                           nullptr, 0, status, sms) &&
+                plan_combine(gv, B, V, n, feat, D, head->w_vocab, long_logits, logit_dtype, log_prior, alpha, beta,
+                             partials, L.partial_ld, status, sms);
+      if (!ok) return DELS_ERR_CUDA;
+      const uint16_t* pos = static_cast<const uint16_t*>(head->w[0]);
+      for (int j = 1; j < n; ++j) {
+        const int p = j - 1;   // position of the newest drafted token x_{j-1}
+        DELS_CUDA(launch_xfmr_embed(ex, pos, p, B, D, t, ab, s));
+        DELS_CUDA(run(gq, s));
+        DELS_CUDA(launch_splitk_finish(xpart, gq.a.total_splits, B, D, nullptr, ACT_NONE, q, D, nullptr, 0, s));
+        DELS_CUDA(run(gk, s));
+        DELS_CUDA(launch_splitk_finish(xpart, gk.a.total_splits, B, D, nullptr, ACT_NONE, kc + (size_t)p * D, P * D,
+                                       nullptr, 0, s));
+        DELS_CUDA(run(gvv, s));
+        DELS_CUDA(launch_splitk_finish(xpart, gvv.a.total_splits, B, D, nullptr, ACT_NONE, vc + (size_t)p * D, P * D,
+                                       nullptr, 0, s));
+        DELS_CUDA(launch_attention(q, kc, vc, B, D, NH, p + 1, P, ob, s));
+        DELS_CUDA(run(go, s));
+        DELS_CUDA(launch_splitk_finish(xpart, go.a.total_splits, B, D, t, ACT_NONE, uu, D, nullptr, 0, s));
+        DELS_CUDA(launch_rmsnorm_bf16(uu, B, D, D, anb, s));
+        DELS_CUDA(run(g1, s));
+        DELS_CUDA(launch_splitk_finish(xpart, g1.a.total_splits, B, F, nullptr, ACT_GELU, nullptr, 0, fb, F, s));
+        DELS_CUDA(run(g2, s));
+        DELS_CUDA(launch_splitk_finish(xpart, g2.a.total_splits, B, D, uu, ACT_NONE, y, D, nullptr, 0, s));
+        DELS_CUDA(launch_rmsnorm_bf16(y, B, D, D, feat, s));
+        gv.a.j = j;
+        DELS_CUDA(run(gv, s));
+        MergeArgs m = mb;
+        m.count = gv.grid;
+        m.j = j;
+        if (j == n - 1) m.table = nullptr;
+        DELS_CUDA(launch_draft_merge(m, s));
+      }
+      return DELS_OK;
+    }
+    case DELS_HEAD_MARKOV: {
+      const int R = head->d_rank;
+      void* feat = at<void>(workspace, L.mk);
+      mb.D = R;
+      mb.dest = feat;
+      r = draft_position0(long_logits, logit_dtype, B, n, V, partials, L.partial_ld, status, mb, sms, s);
+      if (r != DELS_OK || n == 1) return r;
+      Gemm gv;
+      if (bf && !plan_combine(gv, B, V, n, feat, R, head->w_vocab, long_logits, logit_dtype, log_prior, alpha, beta,
+                              partials, L.partial_ld, status, sms))
+        return DELS_ERR_CUDA;
+      const int nch = std::max(1, std::min(L.partial_ld, (V + 255) / 256));
+      for (int j = 1; j < n; ++j) {
+        int count;
+        if (bf) {
+          gv.a.j = j;
+          DELS_CUDA(run(gv, s));
+          count = gv.grid;
+        } else {
+          DELS_CUDA(launch_vocab_combine_f32(static_cast<const float*>(feat), R,
+                                             static_cast<const float*>(head->w_vocab),
+                                             static_cast<const uint8_t*>(long_logits) +
+                                                 (size_t)j * V * (logit_dtype == DELS_F32 ? 4 : 2),
+                                             logit_dtype == DELS_F32, (long long)n * V, log_prior, alpha, beta, B, V,
+                                             partials, L.partial_ld, nch, status, s));
+          count = nch;
+        }
+        MergeArgs m = mb;
+        m.count = count;
+        m.j = j;
+        if (j == n - 1) m.table = nullptr;
+        DELS_CUDA(launch_draft_merge(m, s));
+      }
+      return DELS_OK;
+    }
+    default:
+      return DELS_ERR_UNSUPPORTED;
+  }
+}
+
+}  // extern "C"

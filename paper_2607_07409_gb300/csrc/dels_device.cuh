@@ -1,0 +1,324 @@
+// Device-side building blocks for the DeLS-Spec drafting kernels (sm_103a).
+//
+// * RowAcc: one-pass state of a fused-logit row: running maximum (which is
+//   also the top-1 value), its lowest index, the runner-up value, and the
+//   sum of exp(l - max) rescaled online (Milakov & Gimelshein's online
+//   normaliser). Log-softmax of the argmax is -log(sum); the top-2 gap is
+//   max - second. This is the temperature-0 Decode of Algorithm 1.
+// * Thin inline-PTX wrappers for mbarrier, TMA (cp.async.bulk.tensor),
+//   tcgen05 (alloc / mma / commit / ld) and the async-proxy fences.
+//   Every mbarrier wait is bounded by a global-timer deadline; on expiry the
+//   CTA-wide abort flag is raised and the caller unwinds without hanging.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+#include <cuda.h>
+
+#include "dels_internal.h"
+
+namespace dels {
+
+// ----------------------------------------------------------------------------
+// status word
+// ----------------------------------------------------------------------------
+__device__ __forceinline__ void raise_status(int* status, int code) {
+  if (status) atomicOr(status, code);
+}
+
+__device__ __forceinline__ uint64_t globaltimer_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %globaltimer;" : "=l"(t));
+  return t;
+}
+
+// ----------------------------------------------------------------------------
+// bf16 <-> f32 (bit level; the 16 stored bits are the top half of an f32)
+// ----------------------------------------------------------------------------
+__device__ __forceinline__ float bf16lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+
+__device__ __forceinline__ uint16_t f32_to_bf16_rne(float f) {
+  uint32_t u = __float_as_uint(f);
+  u += 0x7FFFu + ((u >> 16) & 1u);
+  return (uint16_t)(u >> 16);
+}
+
+// ----------------------------------------------------------------------------
+// RowAcc: top-1 / top-2 / online log-sum-exp of one row
+// ----------------------------------------------------------------------------
+struct RowAcc {
+  float m;       // running max == top-1 value
+  float s;       // sum exp(l - m)
+  float second;  // runner-up value (equal to m on an exact tie)
+  int idx;       // lowest index attaining m
+};
+static_assert(sizeof(RowAcc) == 16, "RowAcc is one 16-byte record");
+
+__device__ __forceinline__ RowAcc rowacc_init() {
+  RowAcc a;
+  a.m = -INFINITY; a.s = 0.f; a.second = -INFINITY; a.idx = 0x7FFFFFFF;
+  return a;
+}
+
+// Top-2 update for one element, visited in increasing index order within a
+// thread (so a strict '>' keeps the lowest index on ties).
+__device__ __forceinline__ void top2_push(float x, int v, float& best, float& second, int& idx) {
+  const bool gt = x > best;
+  second = gt ? best : fmaxf(second, x);
+  idx = gt ? v : idx;
+  best = gt ? x : best;
+}
+
+// Online-normaliser update for a chunk of K values whose top-2 has already
+// been pushed (so `best` is the new running max); `m` is the old max.
+template <int K>
+__device__ __forceinline__ void lse_chunk(const float (&x)[K], float best, float& m, float& s) {
+  if (best == -INFINITY) return;               // chunk and history all -inf
+  s *= __expf(m - best);                       // m == -inf -> 0 (s was 0)
+  m = best;
+  float acc = 0.f;
+#pragma unroll
+  for (int i = 0; i < K; ++i) acc += __expf(x[i] - best);   // -inf -> 0; NaN/+inf -> NaN
+  s += acc;
+}
+
+// Merge two partial states (any index order). Ties on the value go to the
+// lower index; the runner-up becomes the larger of the loser's top-1 and the
+// winner's runner-up.
+__device__ __forceinline__ RowAcc rowacc_merge(const RowAcc& a, const RowAcc& b) {
+  const bool b_wins = (b.m > a.m) || (b.m == a.m && b.idx < a.idx);
+  const RowAcc& w = b_wins ? b : a;
+  const RowAcc& l = b_wins ? a : b;
+  RowAcc r;
+  r.m = w.m;
+  r.idx = w.idx;
+  r.second = fmaxf(w.second, l.m);
+  if (r.m == -INFINITY) {
+    r.s = (a.s != a.s || b.s != b.s) ? NAN : 0.f;
+  } else {
+    const float sa = (a.m == -INFINITY) ? (a.s != a.s ? NAN : 0.f) : a.s * __expf(a.m - r.m);
+    const float sb = (b.m == -INFINITY) ? (b.s != b.s ? NAN : 0.f) : b.s * __expf(b.m - r.m);
+    r.s = sa + sb;
+  }
+  return r;
+}
+
+__device__ __forceinline__ RowAcc rowacc_shfl_down(const RowAcc& a, int delta) {
+  RowAcc r;
+  r.m = __shfl_down_sync(0xFFFFFFFFu, a.m, delta);
+  r.s = __shfl_down_sync(0xFFFFFFFFu, a.s, delta);
+  r.second = __shfl_down_sync(0xFFFFFFFFu, a.second, delta);
+  r.idx = __shfl_down_sync(0xFFFFFFFFu, a.idx, delta);
+  return r;
+}
+
+// Warp-level merge in a fixed tree order; lane 0 holds the result.
+__device__ __forceinline__ RowAcc rowacc_warp_reduce(RowAcc a) {
+#pragma unroll
+  for (int d = 16; d > 0; d >>= 1) a = rowacc_merge(a, rowacc_shfl_down(a, d));
+  return a;
+}
+
+// A finished row is valid when it had at least one finite entry and no
+// NaN / +inf (either of which turns s into NaN).
+__device__ __forceinline__ bool rowacc_valid(const RowAcc& a) {
+  return a.m > -INFINITY && a.m < INFINITY && a.s == a.s && a.s > 0.5f && a.s < INFINITY;
+}
+
+// Argmax-only update (verification): value and lowest index.
+__device__ __forceinline__ void argmax_push(float x, int v, float& best, int& idx, bool& nan_seen) {
+  const bool gt = x > best;
+  idx = gt ? v : idx;
+  best = gt ? x : best;
+  nan_seen |= (x != x);
+}
+
+// ----------------------------------------------------------------------------
+// shared-memory address helpers
+// ----------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+// ----------------------------------------------------------------------------
+// mbarrier
+// ----------------------------------------------------------------------------
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void fence_mbarrier_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Bounded wait: returns false (and raises the CTA abort flag) if the barrier
+// phase has not completed by `deadline_ns`, or if another role of the CTA
+// already aborted.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint64_t deadline_ns,
+                                          volatile int* abort_flag) {
+  uint32_t polls = 0;
+  while (!mbar_try_wait(bar, parity)) {
+    if ((++polls & 63u) == 0u) {
+      if (*abort_flag) return false;
+      if (globaltimer_ns() > deadline_ns) {
+        *abort_flag = 1;
+        return false;
+      }
+    }
+  }
+  return true;
+}
+
+// ----------------------------------------------------------------------------
+// TMA (tiled tensor copies global -> shared, completion on an mbarrier)
+// ----------------------------------------------------------------------------
+__device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* map) {
+  asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+}
+
+__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, uint64_t* bar, int x, int y,
+                                            uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1, {%3, %4}], [%2], %5;" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(x), "r"(y), "l"(policy)
+      : "memory");
+}
+
+__device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, uint64_t* bar, int x, int y,
+                                            int z, uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1, {%3, %4, %5}], [%2], %6;" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(x), "r"(y), "r"(z), "l"(policy)
+      : "memory");
+}
+
+// L2 eviction-priority policies for the cache hints above.
+__device__ __forceinline__ uint64_t l2_policy_evict_first() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+__device__ __forceinline__ uint64_t l2_policy_evict_last() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+__device__ __forceinline__ uint64_t l2_policy_evict_normal() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_normal.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+
+// ----------------------------------------------------------------------------
+// tcgen05 (5th-generation tensor cores, tensor memory)
+// ----------------------------------------------------------------------------
+__device__ __forceinline__ void tmem_alloc(uint32_t* smem_dst, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(smem_dst)),
+               "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+// D[tmem] (+)= A[smem] * B[smem]^T, kind::f16 (bf16 inputs, f32 accumulate).
+__device__ __forceinline__ void tc_mma_f16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                           uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// Arrive once on `bar` when all previously issued tcgen05 ops of this thread complete.
+__device__ __forceinline__ void tc_commit(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+                   smem_u32(bar))
+               : "memory");
+}
+
+// 32 lanes x 32 consecutive 32-bit columns: thread i of the warp receives
+// row (lane base + i), columns [col, col + 32).
+__device__ __forceinline__ void tmem_ld_32x32b_x32(uint32_t taddr, float (&r)[32]) {
+  uint32_t* u = reinterpret_cast<uint32_t*>(r);
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : "=r"(u[0]), "=r"(u[1]), "=r"(u[2]), "=r"(u[3]), "=r"(u[4]), "=r"(u[5]), "=r"(u[6]), "=r"(u[7]),
+        "=r"(u[8]), "=r"(u[9]), "=r"(u[10]), "=r"(u[11]), "=r"(u[12]), "=r"(u[13]), "=r"(u[14]), "=r"(u[15]),
+        "=r"(u[16]), "=r"(u[17]), "=r"(u[18]), "=r"(u[19]), "=r"(u[20]), "=r"(u[21]), "=r"(u[22]), "=r"(u[23]),
+        "=r"(u[24]), "=r"(u[25]), "=r"(u[26]), "=r"(u[27]), "=r"(u[28]), "=r"(u[29]), "=r"(u[30]), "=r"(u[31])
+      : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_ld_wait() {
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// Shared-memory matrix descriptor for a K-major bf16 operand stored in the
+// 128-byte-swizzled layout that TMA writes with CU_TENSOR_MAP_SWIZZLE_128B:
+// rows of 64 elements (128 B), 8-row groups 1024 B apart. `addr` must lie in
+// a 1024-byte-aligned buffer; stepping K by 16 elements adds 32 B to it.
+__device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t addr) {
+  uint64_t d = 0;
+  d |= (uint64_t)((addr & 0x3FFFFu) >> 4);          // start address
+  d |= (uint64_t)(16u >> 4) << 16;                   // leading byte offset (unused for SW128 K-major)
+  d |= (uint64_t)(1024u >> 4) << 32;                 // stride byte offset: 8 rows x 128 B
+  d |= (uint64_t)1 << 46;                            // descriptor version (fixed 0b001)
+  d |= (uint64_t)2 << 61;                            // swizzle: 128 B
+  return d;
+}
+
+// Instruction descriptor, kind::f16: bf16 A and B, f32 accumulator, both
+// operands K-major, shape M x N.
+__host__ __device__ __forceinline__ uint32_t idesc_bf16_f32(int M, int N) {
+  return (1u << 4)                      // D format: f32
+         | (1u << 7)                    // A format: bf16
+         | (1u << 10)                   // B format: bf16
+         | ((uint32_t)(N >> 3) << 17)   // N / 8
+         | ((uint32_t)(M >> 4) << 24);  // M / 16
+}
+
+// Named barrier among a subset of warps (id 1..15, an immediate so that the
+// compiler reserves it).
+template <int ID>
+__device__ __forceinline__ void named_bar_sync(int nthreads) {
+  asm volatile("bar.sync %0, %1;" ::"n"(ID), "r"(nthreads) : "memory");
+}
+
+}  // namespace dels

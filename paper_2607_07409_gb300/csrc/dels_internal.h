@@ -1,0 +1,140 @@
+// Internal declarations shared by the library's translation units (host side
+// launchers and the parameter blocks their kernels take).
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+#include <cuda_runtime.h>
+#include <cuda.h>
+
+#include "../../include/dels.h"
+
+namespace dels {
+
+constexpr int kHeaderBytes = 256;          // workspace: status word + padding
+constexpr int kRowsThreads = 256;          // row-reduction kernels
+constexpr int kMaxBatchTile = 128;         // tcgen05 M: batch rows per tile
+constexpr uint64_t kWaitBudgetNs = 2000000000ull;   // bounded device waits: 2 s
+
+struct RowAcc;
+
+// ---- row reductions (combine / verify / draft position 0) -------------------
+struct RowsArgs {
+  const void* longp;
+  const void* shortp;
+  const float* prior;
+  float alpha, beta;
+  int rows, V;
+  long long ld_long, ld_short;   // row pitch in elements
+  int chunk_cols;                // columns per chunk (multiple of 8)
+  int nchunks;                   // chunks per row
+  int rows_per_cta;              // R
+  void* partials;                // [rows][partial_ld] 16-byte records
+  int partial_ld;
+  int* counters;                 // per row group (combine) / per row (verify)
+  int* counters_b;               // verify: per request
+  int32_t* out_token;
+  float* out_lp;
+  float* out_gap;
+  // verify
+  const int32_t* draft;
+  int n;                         // draft positions (verify)
+  int32_t* out_accept;
+  int32_t* out_bonus;
+  int32_t* targ_scratch;         // [rows] target argmax (workspace)
+  int* status;
+};
+
+struct RowsPlan {
+  int nchunks, chunk_cols, rows_per_cta, grid;
+};
+
+RowsPlan plan_rows(int rows, int V, int bytes_per_col, int num_sms, bool vec, int max_chunks);
+cudaError_t launch_combine_rows(const RowsArgs& a, dels_dtype dt, bool vec, bool finalize, cudaStream_t s);
+cudaError_t launch_verify_rows(const RowsArgs& a, dels_dtype dt, bool vec, cudaStream_t s);
+
+// ---- draft merge + gather of the next local-head input ----------------------
+struct MergeArgs {
+  const void* partials;          // [B][partial_ld] RowAcc
+  int partial_ld, count;
+  int B, n, j;
+  int32_t* tokens;               // [B, n]
+  float* out_lp;                 // [B, n]
+  float* out_gap;                // [B, n] or null
+  int* status;
+  // gather: dest[b, k*D:(k+1)*D] = table[token(b, j-k)] or 0 for k < window
+  const void* table;             // [V, D] (bf16 or f32) or null
+  int table_f32;
+  int D, window;
+  void* dest;                    // [B, window*D] same dtype as table
+};
+cudaError_t launch_draft_merge(const MergeArgs& a, cudaStream_t s);
+
+// ---- tcgen05 GEMM (batched skinny products and the vocab projection) --------
+enum EpiKind { EPI_STORE = 0, EPI_COMBINE = 1 };
+enum ActKind { ACT_NONE = 0, ACT_SILU = 1, ACT_GELU = 2 };
+
+struct TcGemmArgs {
+  int B;                         // real batch rows (<= 128)
+  int O;                         // rows of W (outputs)
+  int n_tile;                    // N per tile (multiple of 16, <= 256)
+  int num_o_tiles;
+  int seg_chunks[2];             // K chunks of 64 per segment
+  int seg_splits[2];             // K splits per segment (0 splits: unused segment)
+  int total_splits;
+  int epi;
+  int a_resident;                // A (activations) loaded once per CTA
+  int stages;
+  // EPI_STORE
+  int act;
+  float* out_f32;                // [split][B][ldo] (or final when total_splits == 1)
+  long long out_split_stride;
+  int ldo;
+  uint16_t* out_bf16;            // [B][ldo_bf16] activation output (total_splits == 1)
+  int ldo_bf16;
+  // EPI_COMBINE
+  const float* prior;
+  float alpha, beta;
+  int V;
+  int j;                         // block position: coordinate into the long-logit map
+  int long_f32;
+  int l_box_cols, l_box_rows, l_boxes;   // long-logit tile = l_boxes boxes
+  void* partials;                // [B][partial_ld] RowAcc
+  int partial_ld;
+  int* status;
+  int debug_skip_producer;       // test hook: producer never fills (exercises the bounded waits)
+};
+
+cudaError_t launch_tc_gemm(const TcGemmArgs& a, const CUtensorMap* mA0, const CUtensorMap* mB0,
+                           const CUtensorMap* mA1, const CUtensorMap* mB1, const CUtensorMap* mL, int grid,
+                           size_t smem_bytes, cudaStream_t s);
+size_t tc_gemm_smem_bytes(const TcGemmArgs& a);
+
+// ---- small head kernels -------------------------------------------------------
+cudaError_t launch_gru_gates(const float* part, int S0, int S1, int B, int H, float* h, uint16_t* h_bf16,
+                             cudaStream_t s);
+cudaError_t launch_splitk_finish(const float* part, int S, int B, int O, const float* residual, int act,
+                                 float* out_f32, int ld_f32, uint16_t* out_bf16, int ld_bf16, cudaStream_t s);
+cudaError_t launch_rmsnorm_bf16(const float* x, int B, int D, int ld, uint16_t* out, cudaStream_t s);
+cudaError_t launch_xfmr_embed(const uint16_t* e_rows, const uint16_t* pos_table, int pos, int B, int D,
+                              float* t_out, uint16_t* a_bf16, cudaStream_t s);
+cudaError_t launch_attention(const float* q, const float* kcache, const float* vcache, int B, int D, int nh,
+                             int npos, int cache_ld_pos, uint16_t* o_bf16, cudaStream_t s);
+cudaError_t launch_gemv_f32(const float* X, int ldx, const float* W, int B, int O, int K, int act, float* Y,
+                            int ldy, cudaStream_t s);
+cudaError_t launch_vocab_combine_f32(const float* feat, int K, const float* Wv, const void* longp, int long_f32,
+                                     long long ld_long, const float* prior, float alpha, float beta, int B,
+                                     int V, void* partials, int partial_ld, int nchunks, int* status,
+                                     cudaStream_t s);
+
+// ---- host utilities ---------------------------------------------------------
+int device_sm_count();
+int device_max_smem_optin();
+bool encode_tmap_2d(CUtensorMap* m, const void* base, CUtensorMapDataType dt, int elem_bytes, uint64_t inner,
+                    uint64_t outer, uint64_t row_pitch_bytes, uint32_t box_inner, uint32_t box_outer,
+                    CUtensorMapSwizzle swz);
+bool encode_tmap_3d(CUtensorMap* m, const void* base, CUtensorMapDataType dt, int elem_bytes, uint64_t d0,
+                    uint64_t d1, uint64_t d2, uint64_t pitch1_bytes, uint64_t pitch2_bytes, uint32_t b0,
+                    uint32_t b1, uint32_t b2, CUtensorMapSwizzle swz);
+
+}  // namespace dels

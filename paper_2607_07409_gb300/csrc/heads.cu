@@ -1,0 +1,273 @@
+// Element-wise and small reduction kernels of the local heads (Appendix A
+// GRU head; the window-MLP and transformer heads of the synthetic
+// workloads), plus the float32 CUDA-core path used when the head's weights
+// are float32. The large matrix products of bf16 heads run in tc_gemm.cu.
+#include <climits>
+
+#include "dels_device.cuh"
+
+namespace dels {
+
+namespace {
+
+__device__ __forceinline__ float sigmoidf_(float x) { return 1.f / (1.f + __expf(-x)); }
+
+__device__ __forceinline__ float act_f(int act, float x) {
+  if (act == ACT_SILU) return x / (1.f + __expf(-x));
+  if (act == ACT_GELU) return 0.5f * x * (1.f + erff(x * 0.70710678118654752f));
+  return x;
+}
+
+__device__ __forceinline__ float bf16_to_f(uint16_t u) { return __uint_as_float((uint32_t)u << 16); }
+
+// GRU gates (PyTorch bias-free form; gate rows r, z, n):
+//   gi = sum of the S0 input-product partials, gh = sum of the S1 recurrent ones
+//   r = sigmoid(gi_r + gh_r), z = sigmoid(gi_z + gh_z)
+//   c = tanh(gi_n + r * gh_n), h' = (1 - z) * c + z * h
+__global__ void k_gru_gates(const float* __restrict__ part, int S0, int S1, int B, int H, float* __restrict__ h,
+                            uint16_t* __restrict__ h_bf16) {
+  const long long total = (long long)B * H;
+  const long long split_stride = (long long)B * 3 * H;
+  for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < total;
+       e += (long long)gridDim.x * blockDim.x) {
+    const int b = (int)(e / H), i = (int)(e % H);
+    const long long base = (long long)b * 3 * H + i;
+    float gir = 0.f, giz = 0.f, gin = 0.f, ghr = 0.f, ghz = 0.f, ghn = 0.f;
+    for (int s = 0; s < S0; ++s) {
+      const float* p = part + s * split_stride + base;
+      gir += p[0]; giz += p[H]; gin += p[2 * H];
+    }
+    for (int s = S0; s < S0 + S1; ++s) {
+      const float* p = part + s * split_stride + base;
+      ghr += p[0]; ghz += p[H]; ghn += p[2 * H];
+    }
+    const float r = sigmoidf_(gir + ghr);
+    const float z = sigmoidf_(giz + ghz);
+    const float c = tanhf(gin + r * ghn);
+    const float hp = h[e];
+    const float hn = (1.f - z) * c + z * hp;
+    h[e] = hn;
+    h_bf16[e] = f32_to_bf16_rne(hn);
+  }
+}
+
+// out[b, o] = act(sum_s part[s, b, o] (+ residual[b, o])); partials and the
+// residual are dense [.., B, O]; outputs have their own row pitch.
+__global__ void k_splitk_finish(const float* __restrict__ part, int S, int B, int O,
+                                const float* __restrict__ residual, int act, float* __restrict__ out_f32, int ld_f32,
+                                uint16_t* __restrict__ out_bf16, int ld_bf16) {
+  const long long total = (long long)B * O;
+  for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < total;
+       e += (long long)gridDim.x * blockDim.x) {
+    const int b = (int)(e / O), o = (int)(e % O);
+    float acc = 0.f;
+    for (int s = 0; s < S; ++s) acc += part[s * total + e];
+    if (residual) acc += residual[e];
+    acc = act_f(act, acc);
+    if (out_f32) out_f32[(long long)b * ld_f32 + o] = acc;
+    if (out_bf16) out_bf16[(long long)b * ld_bf16 + o] = f32_to_bf16_rne(acc);
+  }
+}
+
+__device__ __forceinline__ float block_sum(float v) {
+  __shared__ float red[32];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int d = 16; d > 0; d >>= 1) v += __shfl_down_sync(0xFFFFFFFFu, v, d);
+  __syncthreads();
+  if (lane == 0) red[warp] = v;
+  __syncthreads();
+  const int nw = (blockDim.x + 31) >> 5;
+  v = (threadIdx.x < nw) ? red[threadIdx.x] : 0.f;
+  if (warp == 0) {
+#pragma unroll
+    for (int d = 16; d > 0; d >>= 1) v += __shfl_down_sync(0xFFFFFFFFu, v, d);
+    if (lane == 0) red[0] = v;
+  }
+  __syncthreads();
+  return red[0];
+}
+
+// out = bf16( x / sqrt(mean(x^2) + 1e-6) ), one CTA per row
+__global__ void k_rmsnorm_bf16(const float* __restrict__ x, int D, int ld, uint16_t* __restrict__ out) {
+  const float* row = x + (long long)blockIdx.x * ld;
+  float ss = 0.f;
+  for (int i = threadIdx.x; i < D; i += blockDim.x) ss += row[i] * row[i];
+  ss = block_sum(ss);
+  const float inv = rsqrtf(ss / (float)D + 1e-6f);
+  for (int i = threadIdx.x; i < D; i += blockDim.x) out[(long long)blockIdx.x * ld + i] = f32_to_bf16_rne(row[i] * inv);
+}
+
+// t = E[x] + P[pos] (float32), a = bf16(RMSNorm(t)); one CTA per row
+__global__ void k_xfmr_embed(const uint16_t* __restrict__ e_rows, const uint16_t* __restrict__ pos_table, int pos,
+                             int D, float* __restrict__ t_out, uint16_t* __restrict__ a_bf16) {
+  const long long off = (long long)blockIdx.x * D;
+  float ss = 0.f;
+  for (int i = threadIdx.x; i < D; i += blockDim.x) {
+    const float t = bf16_to_f(e_rows[off + i]) + bf16_to_f(pos_table[(long long)pos * D + i]);
+    t_out[off + i] = t;
+    ss += t * t;
+  }
+  ss = block_sum(ss);
+  const float inv = rsqrtf(ss / (float)D + 1e-6f);
+  for (int i = threadIdx.x; i < D; i += blockDim.x) a_bf16[off + i] = f32_to_bf16_rne(t_out[off + i] * inv);
+}
+
+// Causal attention of the newest position over positions 0..npos-1 of the
+// block: one CTA per (row, head); o = softmax(q k^T / sqrt(dh)) v, stored bf16.
+__global__ void k_attention(const float* __restrict__ q, const float* __restrict__ kc, const float* __restrict__ vc,
+                            int D, int nh, int npos, int cache_ld_pos, uint16_t* __restrict__ o_bf16) {
+  const int b = blockIdx.x / nh, hd = blockIdx.x % nh;
+  const int dh = D / nh;
+  __shared__ float w[64];
+  const float* qv = q + (long long)b * D + hd * dh;
+  const float scale = rsqrtf((float)dh);
+  for (int p = 0; p < npos; ++p) {
+    const float* kv = kc + ((long long)b * cache_ld_pos + p) * D + hd * dh;
+    float d = 0.f;
+    for (int i = threadIdx.x; i < dh; i += blockDim.x) d += qv[i] * kv[i];
+    d = block_sum(d);
+    if (threadIdx.x == 0) w[p] = d * scale;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float m = -INFINITY;
+    for (int p = 0; p < npos; ++p) m = fmaxf(m, w[p]);
+    float s = 0.f;
+    for (int p = 0; p < npos; ++p) { w[p] = __expf(w[p] - m); s += w[p]; }
+    for (int p = 0; p < npos; ++p) w[p] /= s;
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < dh; i += blockDim.x) {
+    float o = 0.f;
+    for (int p = 0; p < npos; ++p) o += w[p] * vc[((long long)b * cache_ld_pos + p) * D + hd * dh + i];
+    o_bf16[(long long)b * D + hd * dh + i] = f32_to_bf16_rne(o);
+  }
+}
+
+// float32 skinny product on CUDA cores: Y[b, o] = act(sum_k X[b, k] W[o, k]);
+// one warp per output row o, lanes stride over k, all batch rows at once.
+template <int BMAX>
+__global__ void k_gemv_f32(const float* __restrict__ X, int ldx, const float* __restrict__ W, int B, int O, int K,
+                           int act, float* __restrict__ Y, int ldy) {
+  const int lane = threadIdx.x & 31;
+  const int o = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (o >= O) return;
+  const float* w = W + (long long)o * K;
+  for (int b0 = 0; b0 < B; b0 += BMAX) {
+    float acc[BMAX];
+#pragma unroll
+    for (int i = 0; i < BMAX; ++i) acc[i] = 0.f;
+    for (int k = lane; k < K; k += 32) {
+      const float wk = w[k];
+#pragma unroll
+      for (int i = 0; i < BMAX; ++i)
+        if (b0 + i < B) acc[i] = fmaf(wk, X[(long long)(b0 + i) * ldx + k], acc[i]);
+    }
+#pragma unroll
+    for (int i = 0; i < BMAX; ++i) {
+      float v = acc[i];
+#pragma unroll
+      for (int d = 16; d > 0; d >>= 1) v += __shfl_down_sync(0xFFFFFFFFu, v, d);
+      if (lane == 0 && b0 + i < B) Y[(long long)(b0 + i) * ldy + o] = act_f(act, v);
+    }
+  }
+}
+
+// float32 vocabulary projection fused with the combine: CTA (chunk, b)
+// computes l_S[v] = W_vocab[v] . feat[b] for its vocabulary chunk (one warp
+// per row v), fuses l = l_L + alpha l_S - beta l_P and reduces to one RowAcc.
+__global__ void __launch_bounds__(256) k_vocab_combine_f32(const float* __restrict__ feat, int K,
+                                                           const float* __restrict__ Wv, const void* longp,
+                                                           int long_f32, long long ld_long,
+                                                           const float* __restrict__ prior, float alpha, float beta,
+                                                           int V, void* partials, int partial_ld, int nchunks,
+                                                           int* status) {
+  const int chunk = blockIdx.x % nchunks, b = blockIdx.x / nchunks;
+  const int per = (V + nchunks - 1) / nchunks;
+  const int v0 = chunk * per, v1 = min(V, v0 + per);
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  const float* fb = feat + (long long)b * K;
+  float best = -INFINITY, second = -INFINITY, m = -INFINITY, s = 0.f;
+  int idx = INT_MAX;
+  for (int v = v0 + warp; v < v1; v += nw) {
+    const float* w = Wv + (long long)v * K;
+    float d = 0.f;
+    for (int k = lane; k < K; k += 32) d = fmaf(w[k], fb[k], d);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) d += __shfl_xor_sync(0xFFFFFFFFu, d, o);
+    const float l = long_f32 ? static_cast<const float*>(longp)[(long long)b * ld_long + v]
+                             : bf16_to_f(static_cast<const uint16_t*>(longp)[(long long)b * ld_long + v]);
+    float f[1] = {fmaf(-beta, prior[v], fmaf(alpha, d, l))};
+    top2_push(f[0], v, best, second, idx);
+    lse_chunk<1>(f, best, m, s);
+  }
+  RowAcc r;
+  r.m = best; r.s = s; r.second = second; r.idx = idx;
+  // lanes of a warp hold identical states; merge across warps
+  __shared__ RowAcc red[32];
+  if (lane == 0) red[warp] = r;
+  __syncthreads();
+  if (warp == 0) {
+    RowAcc x = lane < nw ? red[lane] : rowacc_init();
+    x = rowacc_warp_reduce(x);
+    if (lane == 0)
+      reinterpret_cast<float4*>(partials)[(long long)b * partial_ld + chunk] =
+          make_float4(x.m, x.s, x.second, __int_as_float(x.idx));
+  }
+  (void)status;
+}
+
+inline int grid_for(long long total, int threads) {
+  long long g = (total + threads - 1) / threads;
+  return (int)std::min<long long>(std::max<long long>(g, 1), 65535LL * 16);
+}
+
+}  // namespace
+
+cudaError_t launch_gru_gates(const float* part, int S0, int S1, int B, int H, float* h, uint16_t* h_bf16,
+                             cudaStream_t s) {
+  k_gru_gates<<<grid_for((long long)B * H, 256), 256, 0, s>>>(part, S0, S1, B, H, h, h_bf16);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_splitk_finish(const float* part, int S, int B, int O, const float* residual, int act,
+                                 float* out_f32, int ld_f32, uint16_t* out_bf16, int ld_bf16, cudaStream_t s) {
+  k_splitk_finish<<<grid_for((long long)B * O, 256), 256, 0, s>>>(part, S, B, O, residual, act, out_f32, ld_f32,
+                                                                  out_bf16, ld_bf16);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_rmsnorm_bf16(const float* x, int B, int D, int ld, uint16_t* out, cudaStream_t s) {
+  k_rmsnorm_bf16<<<B, 256, 0, s>>>(x, D, ld, out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_xfmr_embed(const uint16_t* e_rows, const uint16_t* pos_table, int pos, int B, int D,
+                              float* t_out, uint16_t* a_bf16, cudaStream_t s) {
+  k_xfmr_embed<<<B, 256, 0, s>>>(e_rows, pos_table, pos, D, t_out, a_bf16);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_attention(const float* q, const float* kcache, const float* vcache, int B, int D, int nh,
+                             int npos, int cache_ld_pos, uint16_t* o_bf16, cudaStream_t s) {
+  k_attention<<<B * nh, 128, 0, s>>>(q, kcache, vcache, D, nh, npos, cache_ld_pos, o_bf16);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gemv_f32(const float* X, int ldx, const float* W, int B, int O, int K, int act, float* Y, int ldy,
+                            cudaStream_t s) {
+  const int warps = 8;
+  k_gemv_f32<8><<<(O + warps - 1) / warps, warps * 32, 0, s>>>(X, ldx, W, B, O, K, act, Y, ldy);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_vocab_combine_f32(const float* feat, int K, const float* Wv, const void* longp, int long_f32,
+                                     long long ld_long, const float* prior, float alpha, float beta, int B, int V,
+                                     void* partials, int partial_ld, int nchunks, int* status, cudaStream_t s) {
+  k_vocab_combine_f32<<<B * nchunks, 256, 0, s>>>(feat, K, Wv, longp, long_f32, ld_long, prior, alpha, beta, V,
+                                                  partials, partial_ld, nchunks, status);
+  return cudaGetLastError();
+}
+
+}  // namespace dels

@@ -1,0 +1,447 @@
+// Row reductions over the vocabulary: the fused combine + argmax (Section 4.3
+// fusion, temperature-0 Decode of Algorithm 1), greedy verification against
+// target logits (Algorithm 1, verification step), and the per-position merge
+// of the drafting loop (which also gathers the next local-head input).
+//
+// These are pure HBM streams: every kernel reads each logit once with 128-bit
+// loads (streaming cache hint) and keeps its per-row state in registers; a
+// row split over several CTAs is finished by the last CTA to arrive (atomic
+// ticket, reset by that CTA), so no [rows, V] intermediate is ever written.
+#include <climits>
+
+#include "dels_device.cuh"
+
+namespace dels {
+
+namespace {
+
+__device__ __forceinline__ void load8(const uint16_t* p, float (&x)[8]) {
+  const uint4 w = __ldcs(reinterpret_cast<const uint4*>(p));
+  x[0] = bf16lo(w.x); x[1] = bf16hi(w.x); x[2] = bf16lo(w.y); x[3] = bf16hi(w.y);
+  x[4] = bf16lo(w.z); x[5] = bf16hi(w.z); x[6] = bf16lo(w.w); x[7] = bf16hi(w.w);
+}
+__device__ __forceinline__ void load8(const float* p, float (&x)[8]) {
+  const float4 a = __ldcs(reinterpret_cast<const float4*>(p));
+  const float4 b = __ldcs(reinterpret_cast<const float4*>(p) + 1);
+  x[0] = a.x; x[1] = a.y; x[2] = a.z; x[3] = a.w; x[4] = b.x; x[5] = b.y; x[6] = b.z; x[7] = b.w;
+}
+__device__ __forceinline__ float load1(const uint16_t* p) { return __uint_as_float((uint32_t)__ldcs(p) << 16); }
+__device__ __forceinline__ float load1(const float* p) { return __ldcs(p); }
+
+__device__ __forceinline__ RowAcc ld_rowacc_cg(const void* base, long long i) {
+  const float4 v = __ldcg(reinterpret_cast<const float4*>(base) + i);
+  RowAcc r;
+  r.m = v.x; r.s = v.y; r.second = v.z; r.idx = __float_as_int(v.w);
+  return r;
+}
+__device__ __forceinline__ void st_rowacc(void* base, long long i, const RowAcc& r) {
+  reinterpret_cast<float4*>(base)[i] = make_float4(r.m, r.s, r.second, __int_as_float(r.idx));
+}
+
+__device__ __forceinline__ void write_decode(const RowAcc& r, long long out_i, int32_t* tok, float* lp, float* gap,
+                                             int* status) {
+  const bool ok = rowacc_valid(r);
+  if (!ok) raise_status(status, DELS_STATUS_NONFINITE);
+  tok[out_i] = ok ? r.idx : -1;
+  if (lp) lp[out_i] = ok ? -logf(r.s) : NAN;
+  if (gap) gap[out_i] = ok ? (r.m - r.second) : NAN;
+}
+
+// Per-thread running state of one row.
+struct RowState {
+  float best, second, m, s;
+  int idx;
+  __device__ __forceinline__ void init() {
+    best = -INFINITY; second = -INFINITY; m = -INFINITY; s = 0.f; idx = INT_MAX;
+  }
+  template <int K>
+  __device__ __forceinline__ void push(const float (&f)[K], int c) {
+#pragma unroll
+    for (int i = 0; i < K; ++i) top2_push(f[i], c + i, best, second, idx);
+    lse_chunk<K>(f, best, m, s);
+  }
+  __device__ __forceinline__ RowAcc acc() const {
+    RowAcc r;
+    r.m = best; r.s = s; r.second = second; r.idx = idx;
+    return r;
+  }
+};
+
+// Merge each row's RowAcc across the CTA; the results are valid in warp 0.
+template <int R>
+__device__ __forceinline__ void block_reduce_rows(const RowAcc (&acc)[R], RowAcc (&out)[R]) {
+  __shared__ RowAcc red[kRowsThreads / 32][R];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int r = 0; r < R; ++r) {
+    RowAcc x = rowacc_warp_reduce(acc[r]);
+    if (lane == 0) red[warp][r] = x;
+  }
+  __syncthreads();
+  if (warp == 0) {
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      RowAcc x = lane < kRowsThreads / 32 ? red[lane][r] : rowacc_init();
+      out[r] = rowacc_warp_reduce(x);
+    }
+  }
+}
+
+// ----------------------------------------------------------------------------
+// fused combine: l = l_L + alpha l_S - beta l_P, then top-1/top-2/LSE per row
+// ----------------------------------------------------------------------------
+template <typename T, int R, bool VEC, bool SH, bool PR, bool FINAL>
+__global__ void __launch_bounds__(kRowsThreads) k_combine_rows(RowsArgs a) {
+  const int chunk = blockIdx.x % a.nchunks;
+  const int group = blockIdx.x / a.nchunks;
+  const int r0 = group * R;
+  const int nr = min(R, a.rows - r0);
+  const int c0 = chunk * a.chunk_cols;
+  const int c1 = min(a.V, c0 + a.chunk_cols);
+  const T* L = static_cast<const T*>(a.longp) + (long long)r0 * a.ld_long;
+  const T* S = SH ? static_cast<const T*>(a.shortp) + (long long)r0 * a.ld_short : nullptr;
+  const float alpha = a.alpha, nbeta = -a.beta;
+
+  RowState st[R];
+#pragma unroll
+  for (int r = 0; r < R; ++r) st[r].init();
+
+  if constexpr (VEC) {
+    constexpr int U = (R == 1) ? 4 : 1;        // 128-bit loads in flight per row
+    const int step = kRowsThreads * 8;
+    for (int cb = c0 + threadIdx.x * 8; cb < c1; cb += step * U) {
+      float lv[U][R][8];
+      float sv[U][R][8];
+      float pv[U][8];
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const int c = cb + u * step;
+        if (c < c1) {
+          if constexpr (PR) {
+            const float4 p0 = __ldg(reinterpret_cast<const float4*>(a.prior + c));
+            const float4 p1 = __ldg(reinterpret_cast<const float4*>(a.prior + c) + 1);
+            pv[u][0] = p0.x; pv[u][1] = p0.y; pv[u][2] = p0.z; pv[u][3] = p0.w;
+            pv[u][4] = p1.x; pv[u][5] = p1.y; pv[u][6] = p1.z; pv[u][7] = p1.w;
+          }
+#pragma unroll
+          for (int r = 0; r < R; ++r) {
+            if (r < nr) {
+              load8(L + (long long)r * a.ld_long + c, lv[u][r]);
+              if constexpr (SH) load8(S + (long long)r * a.ld_short + c, sv[u][r]);
+            }
+          }
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const int c = cb + u * step;
+        if (c < c1) {
+#pragma unroll
+          for (int r = 0; r < R; ++r) {
+            if (r < nr) {
+              float f[8];
+#pragma unroll
+              for (int i = 0; i < 8; ++i) {
+                float x = lv[u][r][i];
+                if constexpr (SH) x = fmaf(alpha, sv[u][r][i], x);
+                if constexpr (PR) x = fmaf(nbeta, pv[u][i], x);
+                f[i] = x;
+              }
+              st[r].push<8>(f, c);
+            }
+          }
+        }
+      }
+    }
+  } else {
+    for (int c = c0 + threadIdx.x; c < c1; c += kRowsThreads) {
+      const float p = PR ? __ldg(a.prior + c) : 0.f;
+#pragma unroll
+      for (int r = 0; r < R; ++r) {
+        if (r < nr) {
+          float x = load1(L + (long long)r * a.ld_long + c);
+          if constexpr (SH) x = fmaf(alpha, load1(S + (long long)r * a.ld_short + c), x);
+          if constexpr (PR) x = fmaf(nbeta, p, x);
+          float f[1] = {x};
+          st[r].push<1>(f, c);
+        }
+      }
+    }
+  }
+
+  RowAcc acc[R], res[R];
+#pragma unroll
+  for (int r = 0; r < R; ++r) acc[r] = st[r].acc();
+  block_reduce_rows<R>(acc, res);
+
+  __shared__ int s_last;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if (a.nchunks == 1 && FINAL) {
+    if (threadIdx.x == 0) {
+      for (int r = 0; r < nr; ++r) write_decode(res[r], r0 + r, a.out_token, a.out_lp, a.out_gap, a.status);
+    }
+    return;
+  }
+  if (threadIdx.x == 0) {
+    for (int r = 0; r < nr; ++r) st_rowacc(a.partials, (long long)(r0 + r) * a.partial_ld + chunk, res[r]);
+  }
+  if (!FINAL) return;
+  if (threadIdx.x == 0) {
+    __threadfence();
+    const int ticket = atomicAdd(&a.counters[group], 1);
+    s_last = (ticket == a.nchunks - 1);
+  }
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  if (warp < nr) {
+    const long long row = r0 + warp;
+    RowAcc x = rowacc_init();
+    for (int k = lane; k < a.nchunks; k += 32) x = rowacc_merge(x, ld_rowacc_cg(a.partials, row * a.partial_ld + k));
+    x = rowacc_warp_reduce(x);
+    if (lane == 0) write_decode(x, row, a.out_token, a.out_lp, a.out_gap, a.status);
+  }
+  if (threadIdx.x == 0) a.counters[group] = 0;
+}
+
+// ----------------------------------------------------------------------------
+// verification: t_j = argmax target[b, j, :]; accept = leading matches; bonus
+// ----------------------------------------------------------------------------
+struct ArgAcc {
+  float best;
+  int idx;
+  int nan;
+};
+
+__device__ __forceinline__ ArgAcc argacc_merge(const ArgAcc& a, const ArgAcc& b) {
+  const bool b_wins = (b.best > a.best) || (b.best == a.best && b.idx < a.idx);
+  ArgAcc r = b_wins ? b : a;
+  r.nan = a.nan | b.nan;
+  return r;
+}
+__device__ __forceinline__ ArgAcc argacc_shfl_down(const ArgAcc& a, int d) {
+  ArgAcc r;
+  r.best = __shfl_down_sync(0xFFFFFFFFu, a.best, d);
+  r.idx = __shfl_down_sync(0xFFFFFFFFu, a.idx, d);
+  r.nan = __shfl_down_sync(0xFFFFFFFFu, a.nan, d);
+  return r;
+}
+__device__ __forceinline__ ArgAcc argacc_warp_reduce(ArgAcc a) {
+#pragma unroll
+  for (int d = 16; d > 0; d >>= 1) a = argacc_merge(a, argacc_shfl_down(a, d));
+  return a;
+}
+
+template <typename T, bool VEC>
+__global__ void __launch_bounds__(kRowsThreads) k_verify_rows(RowsArgs a) {
+  const int chunk = blockIdx.x % a.nchunks;
+  const int row = blockIdx.x / a.nchunks;        // b * (n + 1) + j
+  const int c0 = chunk * a.chunk_cols;
+  const int c1 = min(a.V, c0 + a.chunk_cols);
+  const T* L = static_cast<const T*>(a.longp) + (long long)row * a.ld_long;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+
+  float best = -INFINITY;
+  int idx = INT_MAX;
+  bool nan_seen = false;
+  if constexpr (VEC) {
+    constexpr int U = 4;
+    const int step = kRowsThreads * 8;
+    for (int cb = c0 + threadIdx.x * 8; cb < c1; cb += step * U) {
+      float lv[U][8];
+#pragma unroll
+      for (int u = 0; u < U; ++u)
+        if (cb + u * step < c1) load8(L + cb + u * step, lv[u]);
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const int c = cb + u * step;
+        if (c < c1) {
+#pragma unroll
+          for (int i = 0; i < 8; ++i) argmax_push(lv[u][i], c + i, best, idx, nan_seen);
+        }
+      }
+    }
+  } else {
+    for (int c = c0 + threadIdx.x; c < c1; c += kRowsThreads) argmax_push(load1(L + c), c, best, idx, nan_seen);
+  }
+
+  __shared__ ArgAcc red[kRowsThreads / 32];
+  __shared__ int s_last;
+  ArgAcc x{best, idx, nan_seen ? 1 : 0};
+  x = argacc_warp_reduce(x);
+  if (lane == 0) red[warp] = x;
+  __syncthreads();
+  if (warp != 0) return;
+  x = lane < kRowsThreads / 32 ? red[lane] : ArgAcc{-INFINITY, INT_MAX, 0};
+  x = argacc_warp_reduce(x);
+
+  if (a.nchunks > 1) {
+    int last = 0;
+    if (lane == 0) {
+      reinterpret_cast<float4*>(a.partials)[(long long)row * a.partial_ld + chunk] =
+          make_float4(x.best, __int_as_float(x.idx), __int_as_float(x.nan), 0.f);
+      __threadfence();
+      last = (atomicAdd(&a.counters[row], 1) == a.nchunks - 1);
+    }
+    last = __shfl_sync(0xFFFFFFFFu, last, 0);
+    if (!last) return;
+    __threadfence();
+    ArgAcc y{-INFINITY, INT_MAX, 0};
+    for (int k = lane; k < a.nchunks; k += 32) {
+      const float4 v = __ldcg(reinterpret_cast<const float4*>(a.partials) + (long long)row * a.partial_ld + k);
+      y = argacc_merge(y, ArgAcc{v.x, __float_as_int(v.y), __float_as_int(v.z)});
+    }
+    x = argacc_warp_reduce(y);
+    if (lane == 0) a.counters[row] = 0;
+  }
+  if (lane != 0) return;
+  (void)s_last;
+
+  // this CTA holds the finished argmax of `row`
+  if (x.nan) raise_status(a.status, DELS_STATUS_NONFINITE);
+  const int t = (x.idx == INT_MAX) ? 0 : x.idx;   // an all -inf row: first index
+  const int n = a.n;
+  const int b = row / (n + 1);
+  a.targ_scratch[row] = t;
+  if (a.out_token) a.out_token[row] = t;
+  __threadfence();
+  if (atomicAdd(&a.counters_b[b], 1) != n) return;
+  __threadfence();
+  int acc = 0;
+  bool bad = false;
+  for (; acc < n; ++acc) {
+    const int xd = a.draft[(long long)b * n + acc];
+    bad |= (xd < 0 || xd >= a.V);
+    const int tj = __ldcg(a.targ_scratch + (long long)b * (n + 1) + acc);
+    if (xd != tj) break;
+  }
+  for (int k = acc; k < n && !bad; ++k) {
+    const int xd = a.draft[(long long)b * n + k];
+    bad |= (xd < 0 || xd >= a.V);
+  }
+  if (bad) raise_status(a.status, DELS_STATUS_BAD_TOKEN);
+  a.out_accept[b] = acc;
+  a.out_bonus[b] = __ldcg(a.targ_scratch + (long long)b * (n + 1) + acc);
+  a.counters_b[b] = 0;
+}
+
+// ----------------------------------------------------------------------------
+// drafting: merge the per-CTA partials of position j, emit x_j, and gather the
+// local head's next input rows
+// ----------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) k_draft_merge(MergeArgs a) {
+  const int b = blockIdx.x;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  __shared__ RowAcc red[8];
+  __shared__ int s_tok;
+  RowAcc x = rowacc_init();
+  for (int k = threadIdx.x; k < a.count; k += blockDim.x)
+    x = rowacc_merge(x, ld_rowacc_cg(a.partials, (long long)b * a.partial_ld + k));
+  x = rowacc_warp_reduce(x);
+  if (lane == 0) red[warp] = x;
+  __syncthreads();
+  if (warp == 0) {
+    x = lane < (int)(blockDim.x >> 5) ? red[lane] : rowacc_init();
+    x = rowacc_warp_reduce(x);
+    if (lane == 0) {
+      const long long o = (long long)b * a.n + a.j;
+      write_decode(x, o, a.tokens, a.out_lp, a.out_gap, a.status);
+      s_tok = rowacc_valid(x) ? x.idx : -1;
+    }
+  }
+  __syncthreads();
+  if (a.table == nullptr) return;
+  const int es = a.table_f32 ? 4 : 2;
+  const int vec_per_row = a.D * es / 16;                 // D * es is a multiple of 16
+  for (int k = 0; k < a.window; ++k) {
+    const int jj = a.j - k;
+    int tok = -1;
+    if (k == 0) tok = s_tok;
+    else if (jj >= 0) tok = a.tokens[(long long)b * a.n + jj];
+    uint4* dst = reinterpret_cast<uint4*>(static_cast<uint8_t*>(a.dest) +
+                                          ((long long)b * a.window + k) * (long long)a.D * es);
+    if (tok < 0) {
+      for (int i = threadIdx.x; i < vec_per_row; i += blockDim.x) dst[i] = make_uint4(0, 0, 0, 0);
+    } else {
+      const uint4* src = reinterpret_cast<const uint4*>(static_cast<const uint8_t*>(a.table) +
+                                                        (long long)tok * a.D * es);
+      for (int i = threadIdx.x; i < vec_per_row; i += blockDim.x) dst[i] = __ldg(src + i);
+    }
+  }
+}
+
+template <typename T, int R, bool VEC, bool SH, bool PR>
+cudaError_t launch_combine_t(const RowsArgs& a, bool finalize, cudaStream_t s) {
+  const int groups = (a.rows + R - 1) / R;
+  const long long grid = (long long)groups * a.nchunks;
+  if (grid == 0) return cudaSuccess;
+  if (finalize)
+    k_combine_rows<T, R, VEC, SH, PR, true><<<(unsigned)grid, kRowsThreads, 0, s>>>(a);
+  else
+    k_combine_rows<T, R, VEC, SH, PR, false><<<(unsigned)grid, kRowsThreads, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+template <typename T, int R, bool VEC>
+cudaError_t dispatch_sp(const RowsArgs& a, bool finalize, cudaStream_t s) {
+  const bool sh = a.shortp != nullptr, pr = a.prior != nullptr;
+  if (sh && pr) return launch_combine_t<T, R, VEC, true, true>(a, finalize, s);
+  if (sh) return launch_combine_t<T, R, VEC, true, false>(a, finalize, s);
+  if (pr) return launch_combine_t<T, R, VEC, false, true>(a, finalize, s);
+  return launch_combine_t<T, R, VEC, false, false>(a, finalize, s);
+}
+
+template <typename T>
+cudaError_t dispatch_rv(const RowsArgs& a, bool vec, bool finalize, cudaStream_t s) {
+  if (a.rows_per_cta == 4) {
+    return vec ? dispatch_sp<T, 4, true>(a, finalize, s) : dispatch_sp<T, 4, false>(a, finalize, s);
+  }
+  return vec ? dispatch_sp<T, 1, true>(a, finalize, s) : dispatch_sp<T, 1, false>(a, finalize, s);
+}
+
+}  // namespace
+
+RowsPlan plan_rows(int rows, int V, int bytes_per_col, int num_sms, bool vec, int max_chunks) {
+  RowsPlan p{};
+  const long long target_items = 16LL * num_sms;
+  int nchunks = 1;
+  if (rows > 0 && rows < target_items) nchunks = (int)((target_items + rows - 1) / rows);
+  const int min_cols = std::max(2048, 32768 / std::max(1, bytes_per_col));
+  nchunks = std::min(nchunks, std::max(1, V / min_cols));
+  nchunks = std::max(1, std::min(nchunks, max_chunks));
+  int chunk_cols = (V + nchunks - 1) / nchunks;
+  chunk_cols = (chunk_cols + 7) / 8 * 8;
+  nchunks = (V + chunk_cols - 1) / chunk_cols;
+  p.nchunks = std::max(1, nchunks);
+  p.chunk_cols = std::max(8, chunk_cols);
+  p.rows_per_cta = (vec && rows >= 64LL * num_sms && p.nchunks == 1) ? 4 : 1;
+  const long long groups = (rows + p.rows_per_cta - 1) / p.rows_per_cta;
+  p.grid = (int)std::min<long long>(groups * p.nchunks, INT_MAX);
+  return p;
+}
+
+cudaError_t launch_combine_rows(const RowsArgs& a, dels_dtype dt, bool vec, bool finalize, cudaStream_t s) {
+  if (dt == DELS_BF16) return dispatch_rv<uint16_t>(a, vec, finalize, s);
+  return dispatch_rv<float>(a, vec, finalize, s);
+}
+
+cudaError_t launch_verify_rows(const RowsArgs& a, dels_dtype dt, bool vec, cudaStream_t s) {
+  const long long grid = (long long)a.rows * a.nchunks;
+  if (grid == 0) return cudaSuccess;
+  if (dt == DELS_BF16) {
+    if (vec) k_verify_rows<uint16_t, true><<<(unsigned)grid, kRowsThreads, 0, s>>>(a);
+    else k_verify_rows<uint16_t, false><<<(unsigned)grid, kRowsThreads, 0, s>>>(a);
+  } else {
+    if (vec) k_verify_rows<float, true><<<(unsigned)grid, kRowsThreads, 0, s>>>(a);
+    else k_verify_rows<float, false><<<(unsigned)grid, kRowsThreads, 0, s>>>(a);
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_draft_merge(const MergeArgs& a, cudaStream_t s) {
+  if (a.B == 0) return cudaSuccess;
+  k_draft_merge<<<a.B, 256, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+}  // namespace dels

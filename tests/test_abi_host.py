@@ -1,0 +1,119 @@
+"""Host-side checks of the C-ABI library (no GPU needed).
+
+The library must load, export every entry point ``include/dels.h`` declares,
+and reject bad arguments on the host before touching a device.
+"""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def dels():
+    import paper_2607_07409_gb300 as m
+    if not os.path.exists(m.library_path()):
+        from paper_2607_07409_gb300 import build
+        build.build()
+    m.lib()
+    return m
+
+
+def _declared_functions():
+    src = open(os.path.join(ROOT, "include", "dels.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(dels_[a-z0-9_]+)\s*\(", src)))
+
+
+def test_library_exports_every_declared_symbol(dels):
+    declared = _declared_functions()
+    assert len(declared) >= 10
+    L = ctypes.CDLL(dels.library_path())
+    for name in declared:
+        assert hasattr(L, name), f"missing export {name}"
+    assert sorted(dels.exported_symbols()) == declared
+
+
+def test_version_and_status_strings(dels):
+    assert dels.dels_version() >= 100
+    assert dels.dels_status_string(0) == "ok"
+    assert "NaN" in dels.dels_status_string(1) or "non-finite" in dels.dels_status_string(1)
+    assert dels.dels_status_string(-4).startswith("pointer")
+
+
+def test_prior_from_counts_matches_oracle(dels):
+    c = synth.make_counts(synth.WORKLOADS["qwen3_8b_batched"])
+    got = dels.dels_prior_from_counts(c).numpy().astype(np.float64)
+    ref = oracle.log_prior(c)
+    np.testing.assert_allclose(got, ref, rtol=0, atol=2e-6)    # float32 storage of an fp64 value
+    got2 = dels.dels_prior_from_counts(torch.tensor([0, 1, 2]), lam=0.5).numpy()
+    np.testing.assert_allclose(got2, np.log(np.array([0.5, 1.5, 2.5]) / 4.5), atol=1e-7)
+
+
+def test_prior_rejects_bad_arguments(dels):
+    L = dels.lib()
+    out = torch.empty(3)
+    c = torch.tensor([1, -1, 2])
+    assert L.dels_prior_from_counts(c.data_ptr(), 3, 1.0, out.data_ptr()) == -2
+    c = torch.tensor([1, 1, 2])
+    assert L.dels_prior_from_counts(c.data_ptr(), 3, 0.0, out.data_ptr()) == -2
+    assert L.dels_prior_from_counts(None, 3, 1.0, out.data_ptr()) == -1
+
+
+def test_host_validation_rejects_before_device_work(dels):
+    L = dels.lib()
+    ws = ctypes.create_string_buffer(1024)
+    wsp = ctypes.addressof(ws)
+    # unknown dtype code
+    assert L.dels_combine_argmax(16, 16, 7, None, 0.0, 0.0, 1, 8, 16, None, None, wsp, 1024, None) == -3
+    # negative rows
+    assert L.dels_combine_argmax(16, 16, 0, None, 0.0, 0.0, -1, 8, 16, None, None, wsp, 1024, None) == -2
+    # missing output
+    assert L.dels_combine_argmax(16, None, 0, None, 0.0, 0.0, 1, 8, None, None, None, wsp, 1024, None) == -1
+    # misaligned logits
+    assert L.dels_combine_argmax(18, None, 0, None, 0.0, 0.0, 1, 8, 16, None, None, wsp, 1024, None) == -4
+    # no workspace
+    assert L.dels_combine_argmax(16, None, 0, None, 0.0, 0.0, 1, 8, 16, None, None, None, 0, None) == -5
+    # verify: n out of range
+    assert L.dels_verify_block(16, 16, 0, 1, 0, 8, 16, 16, None, wsp, 1024, None) == -2
+    assert L.dels_verify_block(16, 16, 0, 1, 2000, 8, 16, 16, None, wsp, 1024, None) == -2
+    # rows == 0 and B == 0 are no-ops
+    assert L.dels_combine_argmax(None, None, 0, None, 0.0, 0.0, 0, 8, None, None, None, wsp, 1024, None) == 0
+    assert L.dels_verify_block(None, None, 0, 0, 4, 8, None, None, None, wsp, 1024, None) == 0
+
+
+def test_draft_validation(dels):
+    L = dels.lib()
+    spec = synth.WORKLOADS["qwen3_8b_batched"].head
+    h = dels.LocalHead()
+    h.kind, h.wdtype = 0, 1
+    h.d_model, h.d_hidden, h.d_rank = spec.d_model, spec.d_hidden, spec.d_rank
+    h.emb, h.w_vocab = 4096, 8192
+    h.w[0], h.w[1], h.w[2] = 16, 32, 48
+    ws = 64
+    args = lambda B, n, V, dt=1: (ctypes.byref(h), 16, dt, 16, 0.3, 0.3, B, n, V, 16, 16, None, ws, 1 << 30, None)
+    assert L.dels_draft_block(*args(200, 16, 151936)) == -2          # B > 128
+    assert L.dels_draft_block(*args(4, 0, 151936)) == -2             # n < 1
+    assert L.dels_draft_block(*args(4, 33, 151936)) == -2            # n > 32
+    assert L.dels_draft_block(*args(4, 16, 1001)) == -2              # V % 8 != 0
+    assert L.dels_draft_block(*args(4, 16, 151936, dt=5)) == -3      # logit dtype
+    h.w[1] = None
+    assert L.dels_draft_block(*args(4, 16, 151936)) == -1            # missing W_hh
+    h.w[1] = 40
+    assert L.dels_draft_block(*args(4, 16, 151936)) == -4            # misaligned W_hh
+    h.w[1] = 32
+    h.d_rank = 100
+    assert L.dels_draft_block(*args(4, 16, 151936)) == -2            # bf16 dims must be multiples of 16
+    h.d_rank = 256
+    h.kind = 2
+    h.wdtype = 0
+    assert L.dels_draft_block(*args(4, 16, 151936)) == -6            # f32 transformer head unsupported
+    assert L.dels_draft_workspace_bytes(ctypes.byref(h), 4, 16, 151936) == 0

@@ -1,0 +1,233 @@
+"""GPU parity of the C-ABI library against the CPU oracle.
+
+Every call goes through libdels.so (via the ctypes binding); inputs are the
+seeded synthetic workloads of ``synth``; expected values come from ``oracle``
+only. Sizes are chosen so the oracle finishes in seconds while the device
+path still runs several tiles and a ragged tail.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+import paper_2607_07409_gb300 as dels
+from parity import LP_TOL_BF16, LP_TOL_F32, check_draft, check_rows
+
+pytestmark = pytest.mark.gpu
+
+DEV = "cuda:0"
+
+
+def _ws(nbytes):
+    assert nbytes > 0
+    return torch.zeros(nbytes, dtype=torch.uint8, device=DEV)
+
+
+def _status(ws):
+    return dels.dels_read_status(ws)
+
+
+# ------------------------------------------------------------------ combine
+
+def _combine(long, short, prior, alpha, beta):
+    rows, V = long.shape
+    dt = dels.dtype_code(long)
+    nbytes = dels.dels_combine_workspace_bytes(rows, V, dt)
+    ws = _ws(nbytes)
+    tok = torch.full((rows,), -7, dtype=torch.int32, device=DEV)
+    lp = torch.empty(rows, dtype=torch.float32, device=DEV)
+    gap = torch.empty(rows, dtype=torch.float32, device=DEV)
+    r = dels.dels_combine_argmax(long, short, dt, prior, alpha, beta, rows, V, tok, lp, gap, ws, nbytes)
+    assert r == 0, dels.dels_status_string(r)
+    torch.cuda.synchronize()
+    return tok.cpu().numpy(), lp.cpu().numpy(), gap.cpu().numpy(), _status(ws)
+
+
+@pytest.mark.parametrize("rows,V,dtype,w", [
+    (5, 1000, "bf16", 0.5),        # ragged tail, one chunk per row
+    (3, 1003, "f32", 1.0),         # V not a multiple of the vector width: scalar path
+    (7, 1001, "bf16", 0.5),
+    (64, 32000, "bf16", 0.0),      # w = 0: plain argmax, exact ties included
+    (2, 151936, "f32", 0.5),       # few rows: split over many CTAs + last-CTA merge
+    (1, 151936, "bf16", 1.0),
+    (33, 5000, "f32", 0.0),
+])
+def test_combine_matches_oracle(rows, V, dtype, w):
+    d = synth.make_combine_inputs(rows, V, dtype, seed=rows * 31 + V, device=DEV)
+    prior_cpu = dels.dels_prior_from_counts(d["counts"])
+    tok, lp, gap, st = _combine(d["long"], d["short"], prior_cpu.to(DEV), w, w)
+    assert st == 0
+    ref_prior = oracle.log_prior(d["counts"])
+    # the device consumes the library's float32 prior; the oracle uses its own fp64 prior
+    np.testing.assert_allclose(prior_cpu.numpy(), ref_prior, rtol=0, atol=2e-6)
+    rt, rl, rg = oracle.combine_argmax(d["long"], d["short"], prior_cpu.numpy().astype(np.float64), w, w)
+    fused = None
+    if rows * V < 5e6:
+        fused = oracle.fuse(oracle.to_f64(d["long"]), oracle.to_f64(d["short"]),
+                            prior_cpu.numpy().astype(np.float64), w, w)
+    check_rows(tok, lp, gap, rt, rl, rg, exact_ties=(w == 0.0), fused=fused)
+
+
+def test_combine_many_rows_grouped_path():
+    rows, V = 10000, 64                      # rows >= 64 * SMs: 4 rows per CTA
+    d = synth.make_combine_inputs(rows, V, "bf16", seed=11, device=DEV)
+    prior = dels.dels_prior_from_counts(d["counts"])
+    tok, lp, gap, st = _combine(d["long"], d["short"], prior.to(DEV), 0.5, 0.5)
+    assert st == 0
+    rt, rl, rg = oracle.combine_argmax(d["long"], d["short"], prior.numpy().astype(np.float64), 0.5, 0.5)
+    check_rows(tok, lp, gap, rt, rl, rg)
+
+
+def test_combine_optional_terms_absent():
+    d = synth.make_combine_inputs(4, 4096, "f32", seed=12, device=DEV)
+    tok, lp, gap, st = _combine(d["long"], None, None, 0.7, 0.7)
+    assert st == 0
+    rt, rl, rg = oracle.combine_argmax(d["long"], None, None, 0.7, 0.7)
+    check_rows(tok, lp, gap, rt, rl, rg, exact_ties=True)
+
+
+def test_combine_masked_and_nonfinite_rows():
+    V = 2048
+    long = torch.randn(4, V, device=DEV) * 3
+    long[0, :100] = -float("inf")            # masked entries are allowed
+    long[1, :] = -float("inf")               # all masked: error
+    long[2, 77] = float("nan")               # NaN: error
+    long[3, 5] = float("inf")                # +inf: error
+    tok, lp, gap, st = _combine(long, None, None, 0.0, 0.0)
+    assert st & dels.DELS_STATUS_NONFINITE
+    rt, rl, rg = oracle.combine_argmax(long[:1], None, None, 0.0, 0.0)
+    assert tok[0] == rt[0] and abs(lp[0] - rl[0]) < 1e-5
+    assert tok[1] == -1 and tok[2] == -1 and tok[3] == -1
+
+
+def test_combine_zero_rows_is_noop():
+    ws = _ws(4096)
+    r = dels.dels_combine_argmax(None, None, dels.DELS_F32, None, 0.0, 0.0, 0, 100, None, None, None, ws, 4096)
+    assert r == 0
+
+
+# ------------------------------------------------------------------- verify
+
+def _verify(draft, target):
+    B, n = draft.shape
+    V = target.shape[-1]
+    dt = dels.dtype_code(target)
+    nbytes = dels.dels_verify_workspace_bytes(B, n, V, dt)
+    ws = _ws(nbytes)
+    acc = torch.full((B,), -9, dtype=torch.int32, device=DEV)
+    bonus = torch.full((B,), -9, dtype=torch.int32, device=DEV)
+    targ = torch.full((B, n + 1), -9, dtype=torch.int32, device=DEV)
+    r = dels.dels_verify_block(draft, target, dt, B, n, V, acc, bonus, targ, ws, nbytes)
+    assert r == 0, dels.dels_status_string(r)
+    torch.cuda.synchronize()
+    return acc.cpu().numpy(), bonus.cpu().numpy(), targ.cpu().numpy(), _status(ws), (ws, nbytes)
+
+
+@pytest.mark.parametrize("B,n,V,dtype", [
+    (9, 6, 50, "bf16"), (5, 16, 151936, "bf16"), (3, 8, 32000, "f32"), (17, 4, 1003, "f32"), (2, 32, 4099, "bf16"),
+])
+def test_verify_planted_prefix(B, n, V, dtype):
+    t, draft, planted, accept = synth.make_planted_verify(B, n, V, dtype, seed=B * n, device=DEV)
+    acc, bonus, targ, st, _ = _verify(draft, t)
+    assert st == 0
+    np.testing.assert_array_equal(targ, planted.numpy())
+    np.testing.assert_array_equal(acc, accept.numpy())
+    np.testing.assert_array_equal(bonus, planted.numpy()[np.arange(B), accept.numpy()])
+
+
+def test_verify_random_ties_match_oracle():
+    B, n, V = 40, 5, 3000
+    g = torch.Generator().manual_seed(3)
+    T = torch.randint(-3, 3, (B, n + 1, V), generator=g).to(torch.bfloat16)     # many exact ties
+    draft = torch.randint(0, 2, (B, n), generator=g).to(torch.int32)
+    acc, bonus, targ, st, _ = _verify(draft.to(DEV), T.to(DEV))
+    ra, rb, rt = oracle.verify_greedy(draft.numpy(), T)
+    np.testing.assert_array_equal(targ, rt)
+    np.testing.assert_array_equal(acc, ra)
+    np.testing.assert_array_equal(bonus, rb)
+
+
+def test_verify_repeated_calls_reuse_workspace():
+    t, draft, planted, accept = synth.make_planted_verify(6, 7, 999, "f32", seed=5, device=DEV)
+    acc, bonus, targ, st, (ws, nbytes) = _verify(draft, t)
+    for _ in range(3):   # tickets must reset between calls
+        a2 = torch.empty(6, dtype=torch.int32, device=DEV)
+        b2 = torch.empty(6, dtype=torch.int32, device=DEV)
+        assert dels.dels_verify_block(draft, t, dels.DELS_F32, 6, 7, 999, a2, b2, None, ws, nbytes) == 0
+        torch.cuda.synchronize()
+        np.testing.assert_array_equal(a2.cpu().numpy(), accept.numpy())
+
+
+def test_verify_bad_draft_token_flags_status():
+    t, draft, planted, accept = synth.make_planted_verify(3, 4, 100, "f32", seed=6, device=DEV)
+    draft[2, 3] = 100
+    _, _, _, st, _ = _verify(draft, t)
+    assert st & dels.DELS_STATUS_BAD_TOKEN
+
+
+# ------------------------------------------------------------------ drafting
+
+def _draft(w, d):
+    W = {k[5:]: v for k, v in d.items() if k.startswith("head.")}
+    prior = dels.dels_prior_from_counts(d["counts"]).to(DEV)
+    drafter = dels.Drafter(w.head, W, w.B, w.n, w.V)
+    tok, lp, gap = drafter(d["long"], prior, w.alpha, w.beta)
+    torch.cuda.synchronize()
+    assert drafter.status() == 0
+    return tok.cpu().numpy(), lp.cpu().numpy(), gap.cpu().numpy(), W, prior.cpu().numpy().astype(np.float64)
+
+
+def _oracle_head(w, W):
+    return oracle.make_head(w.head, {k: v.cpu() for k, v in W.items()})
+
+
+SMALL = {
+    "tiny": synth.WORKLOADS["tiny"],
+    "gru": synth.with_sizes(synth.WORKLOADS["qwen3_8b_batched"], B=5, n=6, V=3000,
+                            head_d_model=256, head_d_hidden=128, head_d_rank=64),
+    "gru_b64": synth.with_sizes(synth.WORKLOADS["qwen3_8b_batched"], B=64, n=4, V=4096,
+                                head_d_model=512, head_d_hidden=256, head_d_rank=256),
+    "mlp2": synth.with_sizes(synth.WORKLOADS["qwen3_0p6b"], B=3, n=6, V=2000,
+                             head_d_model=128, head_d_hidden=192, head_d_rank=192),
+    "xfmr": synth.with_sizes(synth.WORKLOADS["qwen3_4b"], B=2, n=5, V=1536,
+                             head_d_model=256, head_d_hidden=512, head_d_rank=256, head_n_heads=4,
+                             head_max_pos=8),
+    "markov": synth.Workload("markov", B=4, n=6, V=2048, logit_dtype="bf16",
+                             head=synth.HeadSpec("markov", "bf16", 0, 0, 128), weight=0.5, seed=7),
+    "markov_f32": synth.Workload("markov_f32", B=2, n=5, V=1000, logit_dtype="f32",
+                                 head=synth.HeadSpec("markov", "f32", 0, 0, 64), weight=0.5, seed=8),
+    "gru_f32": synth.with_sizes(synth.WORKLOADS["qwen3_8b_batched"], B=3, n=5, V=1200, logit_dtype="f32",
+                                head_wdtype="f32", head_d_model=64, head_d_hidden=32, head_d_rank=16),
+}
+
+
+@pytest.mark.parametrize("stress", [False, True])
+@pytest.mark.parametrize("name", list(SMALL))
+def test_draft_small_matches_oracle(name, stress):
+    w = SMALL[name]
+    if stress:
+        w = synth.stress(w)
+    d = synth.make_inputs(w, device=DEV, target=False)
+    tok, lp, gap, W, prior = _draft(w, d)
+    tol = LP_TOL_F32 if w.head.wdtype == "f32" else LP_TOL_BF16
+    info = check_draft(tok, lp, gap, _oracle_head(w, W), d["long"].cpu(), prior, w.alpha, w.beta, tol)
+    print(name, stress, info)
+
+
+def test_draft_zero_weight_is_dflash_argmax():
+    w = synth.with_sizes(synth.stress(synth.WORKLOADS["qwen3_8b_batched"]), B=8, n=5, V=2048, weight=0.0,
+                         head_d_model=128, head_d_hidden=64, head_d_rank=64)
+    d = synth.make_inputs(w, device=DEV, target=False)
+    tok, lp, gap, W, prior = _draft(w, d)
+    L = oracle.to_f64(d["long"])
+    np.testing.assert_array_equal(tok, np.argmax(L, axis=2))
+
+
+def test_draft_block_of_one_position():
+    w = synth.with_sizes(synth.WORKLOADS["qwen3_8b_batched"], B=3, n=1, V=1024,
+                         head_d_model=64, head_d_hidden=32, head_d_rank=32)
+    d = synth.make_inputs(w, device=DEV, target=False)
+    tok, lp, gap, W, prior = _draft(w, d)
+    L = oracle.to_f64(d["long"])
+    np.testing.assert_array_equal(tok[:, 0], np.argmax(L[:, 0], axis=1))
