@@ -1,0 +1,421 @@
+#!/usr/bin/env python
+"""Throughput of the DeLS-Spec per-block drafting hot path on GB300.
+
+One step = one pass of the whole hot path over one batch: dels_draft_block
+(position 0 from the DFlash logits, then for each later position the GRU
+local head, the tcgen05 vocabulary projection fused with the Section 4.3
+combine, and the merge that feeds the token back) followed by
+dels_verify_block (greedy verification against the target logits).
+
+Workload: Qwen3-8B-shaped batched drafting — B = 64 requests, block n = 16,
+vocabulary V = 151936, the Appendix A GRU head (target embedding 4096, GRU
+hidden 1024, rank 256), bf16 weights N(0, 0.02), bf16 DFlash logits N(0, 3)
+plus a Zipf(1.1) bias, target logits = DFlash + N(0, 1). Synthetic data; the
+paper's checkpoints and benchmark prompts are not used.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Prints one JSON line (rank 0). N > 1 runs one independent replica per GPU
+(launched by torchrun): the drafting path has no cross-request exchange.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import re
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "drafted tokens/sec on 1 GB300; combine/argmax HBM GB/s vs 8 TB/s; oracle match"
+UNIT = "drafted tokens/s"
+WORKLOAD = "qwen3_8b_batched"
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse_args():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=200)
+    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    p.add_argument("--e2e-steps", type=int, default=20)
+    p.add_argument("--cpu-rows", type=int, default=4, help="requests in the CPU-oracle baseline sample")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    return p.parse_args()
+
+
+# ----------------------------------------------------------------------------- helpers
+
+def dist_setup(n_expected):
+    import torch
+    import torch.distributed as dist
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1 and not dist.is_initialized():
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        if backend == "nccl":
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend=backend)
+    return world, rank, local
+
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as fh:
+            d = json.load(fh)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def kernel_source_digest():
+    h = hashlib.sha256()
+    for name in ("tc_gemm.cu", "dels_device.cuh"):
+        with open(os.path.join(ROOT, "paper_2607_07409_gb300", "csrc", name), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def ncu_traffic(profile_name):
+    """Per-launch DRAM bytes of the dominant kernel from the committed ncu
+    summary, if it was captured on the current kernel source."""
+    path = os.path.join(ROOT, "profiles", profile_name)
+    try:
+        txt = open(path).read()
+    except OSError:
+        return None
+    m = re.search(r"traffic_bytes_per_launch:\s*([0-9.eE+]+)", txt)
+    s = re.search(r"kernel_source_digest:\s*([0-9a-f]+)", txt)
+    if not m or not s or s.group(1) != kernel_source_digest():
+        return None
+    return float(m.group(1))
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle-reason samples while the timed region runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id):
+        self.gpu_id = gpu_id
+        self.proc = None
+        self.out = None
+
+    def __enter__(self):
+        try:
+            self.out = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu_id), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=self.out, stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            time.sleep(0.15)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        if self.proc is None or self.out is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unavailable"]}
+        self.out.flush()
+        rows = []
+        with open(self.out.name) as fh:
+            for line in fh:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 9 and parts[1].replace(".", "").isdigit():
+                    rows.append(parts)
+        os.unlink(self.out.name)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        sm = [float(r[1]) for r in rows]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower() == "active"})
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": float(rows[0][2]), "reasons": reasons,
+                "samples": len(rows), "power_w_max": max(float(r[3]) for r in rows if _isnum(r[3]))}
+
+
+def _isnum(s):
+    try:
+        float(s)
+        return True
+    except ValueError:
+        return False
+
+
+def algorithmic_vocab_bytes(w):
+    """Bytes one vocabulary-projection + combine launch must move: W_vocab once,
+    the DFlash logits of one position for every request, the prior, and r."""
+    h = w.head
+    return w.V * h.d_rank * 2 + w.B * w.V * 2 + w.V * 4 + w.B * h.d_rank * 2
+
+
+def algorithmic_block_bytes(w):
+    """Bytes of one drafted block with every weight streamed once per position
+    (positions 1..n-1) plus the DFlash logits and prior."""
+    h = w.head
+    per_pos = (w.V * h.d_rank * 2 + 3 * h.d_hidden * (h.d_model + h.d_hidden) * 2 + h.d_rank * h.d_hidden * 2
+               + w.B * w.V * 2 + w.V * 4 + w.B * h.d_model * 2)
+    return (w.n - 1) * per_pos + w.B * w.V * 2
+
+
+# ----------------------------------------------------------------------------- CPU oracle leg
+
+def oracle_sample(w, d, rows, positions, gpu_tokens=None):
+    """Time the oracle on `rows` requests x `positions` positions of the block
+    (plus their greedy verification); optionally check the device's tokens."""
+    import numpy as np
+    import oracle
+    W = {k[5:]: v.cpu() for k, v in d.items() if k.startswith("head.")}
+    long = d["long"][:rows, :positions].cpu()
+    target = d["target"][:rows].cpu()
+    prior = oracle.log_prior(d["counts"])
+    t0 = time.perf_counter()
+    forced = None if gpu_tokens is None else gpu_tokens[:rows, :positions]
+    res = oracle.draft_block(oracle.make_head(w.head, W), long, prior, w.alpha, w.beta, forced=forced)
+    if positions == w.n:
+        oracle.verify_greedy(res.tokens, target)
+    dt = time.perf_counter() - t0
+    match = None
+    if forced is not None:
+        same = forced == res.argmax
+        near = (res.gap < 1e-3) & (res.fused_at >= res.fused_max - 1e-3)
+        match = {"rows": rows, "positions": positions, "tokens_equal": int(same.sum()),
+                 "tokens_total": int(same.size), "near_ties": int((res.gap < 1e-3).sum()),
+                 "ok": bool(np.all(same | near))}
+    return rows * positions, dt, match, res
+
+
+def cpu_cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except Exception:
+        return os.cpu_count()
+
+
+# ----------------------------------------------------------------------------- reference arm
+
+def run_reference(args):
+    world, rank, _ = dist_setup(args.gpus)
+    if rank != 0:
+        return 0
+    import torch
+    import synth
+    w = synth.WORKLOADS[WORKLOAD]
+    d = synth.make_inputs(w, device="cpu")
+    rows, positions = 1, 4
+    for _ in range(args.warmup):
+        oracle_sample(w, d, rows, positions)
+    times = []
+    tokens = 0
+    for _ in range(args.steps):
+        t, dt, _, _ = oracle_sample(w, d, rows, positions)
+        tokens += t
+        times.append(dt)
+    total = sum(times)
+    value = tokens / total
+    sample = f"{rows} of {w.B} requests x positions 0..{positions - 1} of {WORKLOAD} per step"
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * total / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": WORKLOAD, "B": w.B, "n": w.n, "V": w.V, "head": "gru 4096/1024/256"},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ----------------------------------------------------------------------------- our arm
+
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+    import synth
+    import paper_2607_07409_gb300 as dels
+
+    world, rank, local = dist_setup(args.gpus)
+    dev = torch.device(f"cuda:{local}")
+    torch.cuda.set_device(dev)
+    w = synth.WORKLOADS[WORKLOAD]
+    d = synth.make_inputs(w, device=dev)
+    W = {k[5:]: v for k, v in d.items() if k.startswith("head.")}
+    prior = dels.dels_prior_from_counts(d["counts"]).to(dev)
+    long, target = d["long"], d["target"]
+    drafter = dels.Drafter(w.head, W, w.B, w.n, w.V)
+    vbytes = dels.dels_verify_workspace_bytes(w.B, w.n, w.V, dels.DELS_BF16)
+    vws = torch.zeros(vbytes, dtype=torch.uint8, device=dev)
+    acc = torch.empty(w.B, dtype=torch.int32, device=dev)
+    bonus = torch.empty(w.B, dtype=torch.int32, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def step(long_in, target_in):
+        tok, lp, gap = drafter(long_in, prior, w.alpha, w.beta, stream)
+        r = dels.dels_verify_block(tok, target_in, dels.DELS_BF16, w.B, w.n, w.V, acc, bonus, None, vws, vbytes,
+                                   stream)
+        if r != 0:
+            raise dels.DelsError(r, "dels_verify_block")
+        return tok
+
+    for _ in range(max(3, args.warmup)):
+        step(long, target)
+    torch.cuda.synchronize()
+    if drafter.status() != 0 or dels.dels_read_status(vws) != 0:
+        raise RuntimeError("device status set during warm-up")
+
+    # ---- timed region: device-resident inputs (long 311 MB + target 331 MB per step > L2)
+    dels.dels_profile_reset()
+    dels.dels_profile_enable(True)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    gpu_id = local
+    try:
+        gpu_id = "GPU-" + str(torch.cuda.get_device_properties(dev).uuid)
+    except Exception:
+        pass
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(gpu_id) as clk:
+        e0.record(stream)
+        for _ in range(args.steps):
+            step(long, target)
+        e1.record(stream)
+        torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    dels.dels_profile_enable(False)
+    ms = e0.elapsed_time(e1)
+    t = torch.tensor([ms], dtype=torch.float64, device=dev)
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    ms_max = float(t.item())
+    kernels = {}
+    launches = 0
+    for name, cls in dels.KCLASS.items():
+        n_l, tot = dels.dels_profile_read(cls)
+        launches += n_l
+        if n_l:
+            kernels[name] = {"launches_per_step": n_l / args.steps, "ms_per_step": tot / args.steps,
+                             "us_per_launch": 1e3 * tot / n_l}
+    dels.dels_profile_reset()
+    if drafter.status() != 0 or dels.dels_read_status(vws) != 0:
+        raise RuntimeError("device status set during the timed region")
+    tokens_per_step = w.B * w.n
+    value = tokens_per_step * args.steps * world / (ms_max / 1e3)
+
+    # ---- roofline of the dominant kernel (vocabulary projection + combine)
+    peak, peak_kind = measured_peaks()
+    vc = kernels.get("vocab_combine")
+    roofline = None
+    if vc:
+        per_launch_s = vc["us_per_launch"] * 1e-6
+        achieved = algorithmic_vocab_bytes(w) / per_launch_s / 1e9
+        roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+                    "frac": round(achieved / peak, 4), "peak_source": peak_kind,
+                    "kernel": "k_tc_gemm (vocab projection + fused combine)",
+                    "algorithmic_bytes_per_launch": algorithmic_vocab_bytes(w),
+                    "traffic": ncu_traffic(f"vocab_combine_{WORKLOAD}.md")}
+    block_bytes = algorithmic_block_bytes(w)
+
+    # ---- end to end through the public API with host buffers
+    long_h = long.cpu().pin_memory()
+    target_h = target.cpu().pin_memory()
+    long_d = torch.empty_like(long)
+    target_d = torch.empty_like(target)
+    tok_h = torch.empty(w.B, w.n, dtype=torch.int32).pin_memory()
+    acc_h = torch.empty(w.B, dtype=torch.int32).pin_memory()
+    bonus_h = torch.empty(w.B, dtype=torch.int32).pin_memory()
+    k_e2e = max(1, min(args.e2e_steps, args.steps))
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    f0.record(stream)
+    for _ in range(k_e2e):
+        long_d.copy_(long_h, non_blocking=True)
+        target_d.copy_(target_h, non_blocking=True)
+        tok = step(long_d, target_d)
+        tok_h.copy_(tok, non_blocking=True)
+        acc_h.copy_(acc, non_blocking=True)
+        bonus_h.copy_(bonus, non_blocking=True)
+    f1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = f0.elapsed_time(f1)
+    te = torch.tensor([e2e_ms], dtype=torch.float64, device=dev)
+    if world > 1:
+        dist.all_reduce(te, op=dist.ReduceOp.MAX)
+    e2e_val = tokens_per_step * k_e2e * world / (float(te.item()) / 1e3)
+    h2d = long.numel() * long.element_size() + target.numel() * target.element_size()
+    d2h = tok_h.numel() * 4 + acc_h.numel() * 4 + bonus_h.numel() * 4
+
+    # ---- acceptance statistics of the drafted blocks (Appendix D rate_i)
+    a = acc.cpu().numpy()
+    rates = [float((a + 1 >= i).mean()) for i in range(1, w.n + 2)]
+
+    # ---- CPU oracle baseline + oracle match on a sample (rank 0, N = 1)
+    cpu = None
+    match = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        gpu_tok = drafter.tokens.cpu().numpy()
+        ntok, dt, match, _ = oracle_sample(w, d, args.cpu_rows, w.n, gpu_tokens=gpu_tok)
+        cpu = {"value": ntok / dt, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
+               "sample": f"{args.cpu_rows} of {w.B} requests x all {w.n} positions of {WORKLOAD} "
+                         f"(+ their verification), forced to the device's tokens"}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": max(3, args.warmup), "ms_per_step": ms_max / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": WORKLOAD, "B": w.B, "n": w.n, "V": w.V,
+                       "head": "gru emb 4096 / hidden 1024 / rank 256, bf16", "alpha": w.alpha, "beta": w.beta,
+                       "step": "dels_draft_block + dels_verify_block",
+                       "l2": "inputs larger than L2 (long 311 MB + target 331 MB per step, not flushed)",
+                       "parallelism": f"replicas x{world}"},
+            "roofline": roofline,
+            "block": {"algorithmic_bytes": block_bytes,
+                      "hbm_gbs_equiv": round(block_bytes / (ms_max / args.steps * 1e-3) / 1e9, 1)},
+            "kernels": kernels,
+            "gpu_launches": launches,
+            "e2e": {"value": e2e_val, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                    "steps": k_e2e},
+            "clocks": clk.summary(),
+            "cpu_baseline": cpu,
+            "oracle_match": match,
+            "acceptance": {"tau": float((a + 1).mean()), "rate": rates[:6]},
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -201,6 +201,32 @@ int dels_read_status(void* workspace, dels_stream_t stream, int32_t* out_status)
  */
 int dels_prior_from_counts(const int64_t* counts, int V, double lambda, float* out_log_prior);
 
+/* ---- instrumentation (not part of the method) ---------------------------- */
+
+/* Kernel classes timed by the optional per-kernel profiler. */
+enum {
+  DELS_KCLASS_VOCAB_COMBINE = 0, /* tcgen05 vocabulary projection fused with the combine */
+  DELS_KCLASS_HEAD_GEMM = 1,     /* tcgen05 local-head products                          */
+  DELS_KCLASS_HEAD_MISC = 2,     /* head gates / norms / attention / f32 head kernels     */
+  DELS_KCLASS_MERGE = 3,         /* per-position merge + next-input gather                */
+  DELS_KCLASS_POS0 = 4,          /* position-0 row reduction                              */
+  DELS_KCLASS_VERIFY = 5,        /* verification                                          */
+  DELS_KCLASS_COMBINE = 6,       /* dels_combine_argmax                                   */
+  DELS_KCLASS_COUNT = 7
+};
+
+/*
+ * Per-kernel timing for performance analysis. While enabled, every kernel the
+ * library launches is bracketed by CUDA events recorded on the launching
+ * stream (the events are created by the library and reused). dels_profile_read
+ * waits for the recorded events and returns, for one kernel class, the number
+ * of launches and their summed device time in milliseconds since the last
+ * reset. Process-wide; not thread-safe against concurrent library calls.
+ */
+int dels_profile_enable(int on);
+int dels_profile_reset(void);
+int dels_profile_read(int kernel_class, int* out_launches, double* out_total_ms);
+
 /* Human-readable name of a status or error code. */
 const char* dels_status_string(int code);
 

@@ -25,6 +25,7 @@ __all__ = [
     "dels_combine_workspace_bytes", "dels_combine_argmax",
     "dels_verify_workspace_bytes", "dels_verify_block",
     "dels_read_status", "dels_prior_from_counts", "dels_status_string", "dels_version",
+    "dels_profile_enable", "dels_profile_reset", "dels_profile_read", "KCLASS",
     "make_head", "Drafter", "dtype_code",
 ]
 
@@ -65,7 +66,13 @@ _SIGS = {
     "dels_prior_from_counts": (_i, [_vp, _i, _d, _vp]),
     "dels_status_string": (ctypes.c_char_p, [_i]),
     "dels_version": (_i, []),
+    "dels_profile_enable": (_i, [_i]),
+    "dels_profile_reset": (_i, []),
+    "dels_profile_read": (_i, [_i, ctypes.POINTER(ctypes.c_int), ctypes.POINTER(ctypes.c_double)]),
 }
+
+# kernel classes of the optional profiler
+KCLASS = {"vocab_combine": 0, "head_gemm": 1, "head_misc": 2, "merge": 3, "pos0": 4, "verify": 5, "combine": 6}
 
 
 def exported_symbols():
@@ -191,6 +198,22 @@ def dels_prior_from_counts(counts: torch.Tensor, lam: float = 1.0) -> torch.Tens
     _check(lib().dels_prior_from_counts(c.data_ptr(), c.numel(), float(lam), out.data_ptr()),
            "dels_prior_from_counts")
     return out
+
+
+def dels_profile_enable(on: bool) -> None:
+    _check(lib().dels_profile_enable(1 if on else 0), "dels_profile_enable")
+
+
+def dels_profile_reset() -> None:
+    _check(lib().dels_profile_reset(), "dels_profile_reset")
+
+
+def dels_profile_read(kernel_class: int):
+    """(launches, total device ms) of one kernel class since the last reset."""
+    n = ctypes.c_int(0)
+    ms = ctypes.c_double(0.0)
+    _check(lib().dels_profile_read(int(kernel_class), ctypes.byref(n), ctypes.byref(ms)), "dels_profile_read")
+    return n.value, ms.value
 
 
 # ----------------------------------------------------------------------------- conveniences

@@ -81,6 +81,56 @@ bool encode_tmap_3d(CUtensorMap* m, const void* base, CUtensorMapDataType dt, in
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+
+// ------------------------------------------------------- optional profiler
+namespace prof {
+bool on = false;
+struct Rec {
+  int cls;
+  cudaEvent_t a, b;
+};
+std::vector<Rec> recs;
+std::vector<cudaEvent_t> pool;
+
+cudaEvent_t take() {
+  if (!pool.empty()) {
+    cudaEvent_t e = pool.back();
+    pool.pop_back();
+    return e;
+  }
+  cudaEvent_t e = nullptr;
+  return cudaEventCreate(&e) == cudaSuccess ? e : nullptr;
+}
+
+// Brackets one kernel launch with events on its stream while profiling is on.
+struct Scope {
+  int cls;
+  cudaStream_t s;
+  cudaEvent_t a = nullptr;
+  Scope(int c, cudaStream_t st) : cls(c), s(st) {
+    if (on) {
+      a = take();
+      if (a && cudaEventRecord(a, s) != cudaSuccess) {
+        pool.push_back(a);
+        a = nullptr;
+      }
+    }
+  }
+  ~Scope() {
+    if (!a) return;
+    cudaEvent_t b = take();
+    if (b && cudaEventRecord(b, s) == cudaSuccess) {
+      recs.push_back({cls, a, b});
+    } else {
+      pool.push_back(a);
+      if (b) pool.push_back(b);
+    }
+  }
+};
+}  // namespace prof
+
+#define PROF(cls) prof::Scope prof_scope_(cls, s)
+
 namespace {
 
 // ------------------------------------------------------------- tcgen05 plans
@@ -396,11 +446,11 @@ int draft_position0(const void* long_logits, dels_dtype ldt, int B, int n, int V
   a.partials = partials;
   a.partial_ld = partial_ld;
   a.status = status;
-  DELS_CUDA(launch_combine_rows(a, ldt, true, false, s));
+  { PROF(DELS_KCLASS_POS0); DELS_CUDA(launch_combine_rows(a, ldt, true, false, s)); }
   MergeArgs m = merge_base;
   m.count = p.nchunks;
   m.j = 0;
-  DELS_CUDA(launch_draft_merge(m, s));
+  { PROF(DELS_KCLASS_MERGE); DELS_CUDA(launch_draft_merge(m, s)); }
   return DELS_OK;
 }
 
@@ -412,6 +462,40 @@ using namespace dels;
 extern "C" {
 
 int dels_version(void) { return 100; }
+
+int dels_profile_enable(int on) {
+  prof::on = on != 0;
+  return DELS_OK;
+}
+
+int dels_profile_reset(void) {
+  for (auto& r : prof::recs) {
+    cudaEventSynchronize(r.b);
+    prof::pool.push_back(r.a);
+    prof::pool.push_back(r.b);
+  }
+  prof::recs.clear();
+  return DELS_OK;
+}
+
+int dels_profile_read(int kernel_class, int* out_launches, double* out_total_ms) {
+  if (!out_launches || !out_total_ms) return DELS_ERR_NULL_POINTER;
+  if (kernel_class < 0 || kernel_class >= DELS_KCLASS_COUNT) return DELS_ERR_BAD_SHAPE;
+  int nl = 0;
+  double ms = 0.0;
+  for (auto& r : prof::recs) {
+    if (r.cls != kernel_class) continue;
+    if (cudaEventSynchronize(r.b) != cudaSuccess) return DELS_ERR_CUDA;
+    float t = 0.f;
+    if (cudaEventElapsedTime(&t, r.a, r.b) != cudaSuccess) return DELS_ERR_CUDA;
+    ms += t;
+    ++nl;
+  }
+  *out_launches = nl;
+  *out_total_ms = ms;
+  return DELS_OK;
+}
+
 
 const char* dels_status_string(int code) {
   switch (code) {
@@ -511,8 +595,9 @@ int dels_combine_argmax(const void* long_logits, const void* short_logits, dels_
   a.out_lp = out_logprob;
   a.out_gap = out_top2_gap;
   a.status = at<int>(workspace, 0);
-  if (launch_combine_rows(a, dtype, vec, true, reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess)
-    return DELS_ERR_CUDA;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  PROF(DELS_KCLASS_COMBINE);
+  if (launch_combine_rows(a, dtype, vec, true, s) != cudaSuccess) return DELS_ERR_CUDA;
   return DELS_OK;
 }
 
@@ -575,7 +660,9 @@ int dels_verify_block(const int32_t* draft_tokens, const void* target_logits, de
   a.out_accept = out_accept_len;
   a.out_bonus = out_bonus;
   a.status = at<int>(workspace, 0);
-  if (launch_verify_rows(a, dtype, vec, reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess) return DELS_ERR_CUDA;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  PROF(DELS_KCLASS_VERIFY);
+  if (launch_verify_rows(a, dtype, vec, s) != cudaSuccess) return DELS_ERR_CUDA;
   return DELS_OK;
 }
 
@@ -646,16 +733,16 @@ int dels_draft_block(const dels_local_head* head, const void* long_logits, dels_
                           partials, L.partial_ld, status, sms))
           return DELS_ERR_CUDA;
         for (int j = 1; j < n; ++j) {
-          DELS_CUDA(run(gg, s));
-          DELS_CUDA(launch_gru_gates(gpart, gg.a.seg_splits[0], gg.a.seg_splits[1], B, H, h, hb, s));
-          DELS_CUDA(run(gr, s));
+          { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run(gg, s)); }
+          { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_gru_gates(gpart, gg.a.seg_splits[0], gg.a.seg_splits[1], B, H, h, hb, s)); }
+          { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run(gr, s)); }
           gv.a.j = j;
-          DELS_CUDA(run(gv, s));
+          { PROF(DELS_KCLASS_VOCAB_COMBINE); DELS_CUDA(run(gv, s)); }
           MergeArgs m = mb;
           m.count = gv.grid;
           m.j = j;
           if (j == n - 1) m.table = nullptr;
-          DELS_CUDA(launch_draft_merge(m, s));
+          { PROF(DELS_KCLASS_MERGE); DELS_CUDA(launch_draft_merge(m, s)); }
         }
       } else {
         const float* E = static_cast<const float*>(eg);
@@ -665,20 +752,20 @@ int dels_draft_block(const dels_local_head* head, const void* long_logits, dels_
         float* feat = static_cast<float*>(rr);
         const int nch = std::max(1, std::min(L.partial_ld, (V + 255) / 256));
         for (int j = 1; j < n; ++j) {
-          DELS_CUDA(launch_gemv_f32(E, D, Wih, B, 3 * H, D, ACT_NONE, gpart, 3 * H, s));
-          DELS_CUDA(launch_gemv_f32(h, H, Whh, B, 3 * H, H, ACT_NONE, gpart + (size_t)B * 3 * H, 3 * H, s));
-          DELS_CUDA(launch_gru_gates(gpart, 1, 1, B, H, h, hb, s));
-          DELS_CUDA(launch_gemv_f32(h, H, Wr, B, R, H, ACT_SILU, feat, R, s));
-          DELS_CUDA(launch_vocab_combine_f32(feat, R, static_cast<const float*>(head->w_vocab),
+          { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_gemv_f32(E, D, Wih, B, 3 * H, D, ACT_NONE, gpart, 3 * H, s)); }
+          { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_gemv_f32(h, H, Whh, B, 3 * H, H, ACT_NONE, gpart + (size_t)B * 3 * H, 3 * H, s)); }
+          { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_gru_gates(gpart, 1, 1, B, H, h, hb, s)); }
+          { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_gemv_f32(h, H, Wr, B, R, H, ACT_SILU, feat, R, s)); }
+          { PROF(DELS_KCLASS_VOCAB_COMBINE); DELS_CUDA(launch_vocab_combine_f32(feat, R, static_cast<const float*>(head->w_vocab),
                                              static_cast<const uint8_t*>(long_logits) +
                                                  (size_t)j * V * (logit_dtype == DELS_F32 ? 4 : 2),
                                              logit_dtype == DELS_F32, (long long)n * V, log_prior, alpha, beta, B, V,
-                                             partials, L.partial_ld, nch, status, s));
+                                             partials, L.partial_ld, nch, status, s)); }
           MergeArgs m = mb;
           m.count = nch;
           m.j = j;
           if (j == n - 1) m.table = nullptr;
-          DELS_CUDA(launch_draft_merge(m, s));
+          { PROF(DELS_KCLASS_MERGE); DELS_CUDA(launch_draft_merge(m, s)); }
         }
       }
       return DELS_OK;
@@ -708,41 +795,41 @@ int dels_draft_block(const dels_local_head* head, const void* long_logits, dels_
                           partials, L.partial_ld, status, sms))
           return DELS_ERR_CUDA;
         for (int j = 1; j < n; ++j) {
-          DELS_CUDA(run(g1, s));
-          DELS_CUDA(launch_splitk_finish(mpart, g1.a.total_splits, B, Hd, nullptr, ACT_GELU, nullptr, 0,
-                                         static_cast<uint16_t*>(h1), Hd, s));
+          { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run(g1, s)); }
+          { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_splitk_finish(mpart, g1.a.total_splits, B, Hd, nullptr, ACT_GELU, nullptr, 0,
+                                         static_cast<uint16_t*>(h1), Hd, s)); }
           if (head->n_layers == 2) {
-            DELS_CUDA(run(g2, s));
-            DELS_CUDA(launch_splitk_finish(mpart, g2.a.total_splits, B, Hd, nullptr, ACT_GELU, nullptr, 0,
-                                           static_cast<uint16_t*>(h2), Hd, s));
+            { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run(g2, s)); }
+            { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_splitk_finish(mpart, g2.a.total_splits, B, Hd, nullptr, ACT_GELU, nullptr, 0,
+                                           static_cast<uint16_t*>(h2), Hd, s)); }
           }
           gv.a.j = j;
-          DELS_CUDA(run(gv, s));
+          { PROF(DELS_KCLASS_VOCAB_COMBINE); DELS_CUDA(run(gv, s)); }
           MergeArgs m = mb;
           m.count = gv.grid;
           m.j = j;
           if (j == n - 1) m.table = nullptr;
-          DELS_CUDA(launch_draft_merge(m, s));
+          { PROF(DELS_KCLASS_MERGE); DELS_CUDA(launch_draft_merge(m, s)); }
         }
       } else {
         const int nch = std::max(1, std::min(L.partial_ld, (V + 255) / 256));
         for (int j = 1; j < n; ++j) {
-          DELS_CUDA(launch_gemv_f32(static_cast<const float*>(u), K1, static_cast<const float*>(head->w[0]), B, Hd,
-                                    K1, ACT_GELU, static_cast<float*>(h1), Hd, s));
+          { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_gemv_f32(static_cast<const float*>(u), K1, static_cast<const float*>(head->w[0]), B, Hd,
+                                    K1, ACT_GELU, static_cast<float*>(h1), Hd, s)); }
           if (head->n_layers == 2)
-            DELS_CUDA(launch_gemv_f32(static_cast<const float*>(h1), Hd, static_cast<const float*>(head->w[1]), B,
-                                      Hd, Hd, ACT_GELU, static_cast<float*>(h2), Hd, s));
-          DELS_CUDA(launch_vocab_combine_f32(static_cast<const float*>(feat), Hd,
+            { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_gemv_f32(static_cast<const float*>(h1), Hd, static_cast<const float*>(head->w[1]), B,
+                                      Hd, Hd, ACT_GELU, static_cast<float*>(h2), Hd, s)); }
+          { PROF(DELS_KCLASS_VOCAB_COMBINE); DELS_CUDA(launch_vocab_combine_f32(static_cast<const float*>(feat), Hd,
                                              static_cast<const float*>(head->w_vocab),
                                              static_cast<const uint8_t*>(long_logits) +
                                                  (size_t)j * V * (logit_dtype == DELS_F32 ? 4 : 2),
                                              logit_dtype == DELS_F32, (long long)n * V, log_prior, alpha, beta, B, V,
-                                             partials, L.partial_ld, nch, status, s));
+                                             partials, L.partial_ld, nch, status, s)); }
           MergeArgs m = mb;
           m.count = nch;
           m.j = j;
           if (j == n - 1) m.table = nullptr;
-          DELS_CUDA(launch_draft_merge(m, s));
+          { PROF(DELS_KCLASS_MERGE); DELS_CUDA(launch_draft_merge(m, s)); }
         }
       }
       return DELS_OK;
@@ -785,31 +872,31 @@ int dels_draft_block(const dels_local_head* head, const void* long_logits, dels_
       const uint16_t* pos = static_cast<const uint16_t*>(head->w[0]);
       for (int j = 1; j < n; ++j) {
         const int p = j - 1;   // position of the newest drafted token x_{j-1}
-        DELS_CUDA(launch_xfmr_embed(ex, pos, p, B, D, t, ab, s));
-        DELS_CUDA(run(gq, s));
-        DELS_CUDA(launch_splitk_finish(xpart, gq.a.total_splits, B, D, nullptr, ACT_NONE, q, D, nullptr, 0, s));
-        DELS_CUDA(run(gk, s));
-        DELS_CUDA(launch_splitk_finish(xpart, gk.a.total_splits, B, D, nullptr, ACT_NONE, kc + (size_t)p * D, P * D,
-                                       nullptr, 0, s));
-        DELS_CUDA(run(gvv, s));
-        DELS_CUDA(launch_splitk_finish(xpart, gvv.a.total_splits, B, D, nullptr, ACT_NONE, vc + (size_t)p * D, P * D,
-                                       nullptr, 0, s));
-        DELS_CUDA(launch_attention(q, kc, vc, B, D, NH, p + 1, P, ob, s));
-        DELS_CUDA(run(go, s));
-        DELS_CUDA(launch_splitk_finish(xpart, go.a.total_splits, B, D, t, ACT_NONE, uu, D, nullptr, 0, s));
-        DELS_CUDA(launch_rmsnorm_bf16(uu, B, D, D, anb, s));
-        DELS_CUDA(run(g1, s));
-        DELS_CUDA(launch_splitk_finish(xpart, g1.a.total_splits, B, F, nullptr, ACT_GELU, nullptr, 0, fb, F, s));
-        DELS_CUDA(run(g2, s));
-        DELS_CUDA(launch_splitk_finish(xpart, g2.a.total_splits, B, D, uu, ACT_NONE, y, D, nullptr, 0, s));
-        DELS_CUDA(launch_rmsnorm_bf16(y, B, D, D, feat, s));
+        { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_xfmr_embed(ex, pos, p, B, D, t, ab, s)); }
+        { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run(gq, s)); }
+        { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_splitk_finish(xpart, gq.a.total_splits, B, D, nullptr, ACT_NONE, q, D, nullptr, 0, s)); }
+        { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run(gk, s)); }
+        { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_splitk_finish(xpart, gk.a.total_splits, B, D, nullptr, ACT_NONE, kc + (size_t)p * D, P * D,
+                                       nullptr, 0, s)); }
+        { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run(gvv, s)); }
+        { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_splitk_finish(xpart, gvv.a.total_splits, B, D, nullptr, ACT_NONE, vc + (size_t)p * D, P * D,
+                                       nullptr, 0, s)); }
+        { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_attention(q, kc, vc, B, D, NH, p + 1, P, ob, s)); }
+        { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run(go, s)); }
+        { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_splitk_finish(xpart, go.a.total_splits, B, D, t, ACT_NONE, uu, D, nullptr, 0, s)); }
+        { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_rmsnorm_bf16(uu, B, D, D, anb, s)); }
+        { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run(g1, s)); }
+        { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_splitk_finish(xpart, g1.a.total_splits, B, F, nullptr, ACT_GELU, nullptr, 0, fb, F, s)); }
+        { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run(g2, s)); }
+        { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_splitk_finish(xpart, g2.a.total_splits, B, D, uu, ACT_NONE, y, D, nullptr, 0, s)); }
+        { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_rmsnorm_bf16(y, B, D, D, feat, s)); }
         gv.a.j = j;
-        DELS_CUDA(run(gv, s));
+        { PROF(DELS_KCLASS_VOCAB_COMBINE); DELS_CUDA(run(gv, s)); }
         MergeArgs m = mb;
         m.count = gv.grid;
         m.j = j;
         if (j == n - 1) m.table = nullptr;
-        DELS_CUDA(launch_draft_merge(m, s));
+        { PROF(DELS_KCLASS_MERGE); DELS_CUDA(launch_draft_merge(m, s)); }
       }
       return DELS_OK;
     }
@@ -829,22 +916,22 @@ int dels_draft_block(const dels_local_head* head, const void* long_logits, dels_
         int count;
         if (bf) {
           gv.a.j = j;
-          DELS_CUDA(run(gv, s));
+          { PROF(DELS_KCLASS_VOCAB_COMBINE); DELS_CUDA(run(gv, s)); }
           count = gv.grid;
         } else {
-          DELS_CUDA(launch_vocab_combine_f32(static_cast<const float*>(feat), R,
+          { PROF(DELS_KCLASS_VOCAB_COMBINE); DELS_CUDA(launch_vocab_combine_f32(static_cast<const float*>(feat), R,
                                              static_cast<const float*>(head->w_vocab),
                                              static_cast<const uint8_t*>(long_logits) +
                                                  (size_t)j * V * (logit_dtype == DELS_F32 ? 4 : 2),
                                              logit_dtype == DELS_F32, (long long)n * V, log_prior, alpha, beta, B, V,
-                                             partials, L.partial_ld, nch, status, s));
+                                             partials, L.partial_ld, nch, status, s)); }
           count = nch;
         }
         MergeArgs m = mb;
         m.count = count;
         m.j = j;
         if (j == n - 1) m.table = nullptr;
-        DELS_CUDA(launch_draft_merge(m, s));
+        { PROF(DELS_KCLASS_MERGE); DELS_CUDA(launch_draft_merge(m, s)); }
       }
       return DELS_OK;
     }
