@@ -58,6 +58,7 @@ enum {
   DELS_ERR_WORKSPACE = -5,         /* workspace NULL or smaller than required */
   DELS_ERR_UNSUPPORTED = -6,       /* head kind / dims this build does not run */
   DELS_ERR_CUDA = -7,              /* a CUDA runtime or driver call failed */
+  DELS_ERR_TOO_LARGE = -8,         /* problem needs more than the fixed no-allocation scratch */
   /* detected on the device; bits of the workspace status word */
   DELS_STATUS_NONFINITE = 1,       /* NaN or +inf logit, or a row that is all -inf */
   DELS_STATUS_TIMEOUT = 2,         /* a bounded device-side wait expired */
@@ -164,6 +165,37 @@ int dels_combine_argmax(const void* long_logits, const void* short_logits, dels_
                         const float* log_prior, float alpha, float beta, int rows, int V,
                         int32_t* out_token, float* out_logprob, float* out_top2_gap, void* workspace,
                         size_t workspace_bytes, dels_stream_t stream);
+
+/*
+ * dels_combine_argmax for callers that cannot allocate device memory.
+ *
+ * Same operation, arguments and outputs as dels_combine_argmax, minus the
+ * workspace. (The paper has no counterpart; this is a deployment variant.)
+ * It is meant for callers that own only the buffers they pass in and out —
+ * a plugin inside a host framework whose allocator it cannot reach, or a
+ * latency-critical loop where an allocation could stall the device — and so
+ * cannot provide a workspace.
+ *
+ * Scratch: a fixed 4 MiB array compiled into the library; every GPU that
+ * loads the library holds it until the process exits. A call whose scratch
+ * need (dels_combine_workspace_bytes for the same rows, V, dtype) exceeds
+ * 4 MiB returns DELS_ERR_TOO_LARGE and enqueues nothing; at V = 151936 that
+ * is reached only beyond roughly 200,000 rows.
+ * Set-up: the first call on a device, with that device current, looks up
+ * the scratch's device address (cudaGetSymbolAddress); make that first call
+ * before any stream capture.
+ * The call allocates nothing (no cudaMalloc, cudaFree or allocating library
+ * routine). It clears the part of the scratch that must start at zero with
+ * cudaMemsetAsync on `stream`. All calls on a device share the one scratch,
+ * which keeps the last call's contents: calls that overlap on the GPU (on
+ * different streams without ordering) race and give wrong results.
+ * Device-detected errors cannot be read back through a status word here:
+ * a non-finite row shows up as token -1 and logprob NaN in the outputs.
+ */
+int dels_combine_argmax_noalloc(const void* long_logits, const void* short_logits, dels_dtype dtype,
+                                const float* log_prior, float alpha, float beta, int rows, int V,
+                                int32_t* out_token, float* out_logprob, float* out_top2_gap,
+                                dels_stream_t stream);
 
 /* ---- greedy verification (Algorithm 1, last two steps) ------------------ */
 

@@ -22,7 +22,7 @@ __all__ = [
     "DELS_STATUS_NONFINITE", "DELS_STATUS_TIMEOUT", "DELS_STATUS_BAD_TOKEN",
     "DelsError", "LocalHead", "lib", "library_path", "exported_symbols",
     "dels_draft_workspace_bytes", "dels_draft_block",
-    "dels_combine_workspace_bytes", "dels_combine_argmax",
+    "dels_combine_workspace_bytes", "dels_combine_argmax", "dels_combine_argmax_noalloc",
     "dels_verify_workspace_bytes", "dels_verify_block",
     "dels_read_status", "dels_prior_from_counts", "dels_status_string", "dels_version",
     "dels_profile_enable", "dels_profile_reset", "dels_profile_read", "KCLASS",
@@ -33,6 +33,7 @@ DELS_OK = 0
 DELS_F32, DELS_BF16 = 0, 1
 DELS_HEAD_GRU, DELS_HEAD_MLP, DELS_HEAD_XFMR, DELS_HEAD_MARKOV = 0, 1, 2, 3
 DELS_STATUS_NONFINITE, DELS_STATUS_TIMEOUT, DELS_STATUS_BAD_TOKEN = 1, 2, 4
+DELS_ERR_TOO_LARGE = -8
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _LIB_PATH = os.path.join(_HERE, "libdels.so")
@@ -60,6 +61,7 @@ _SIGS = {
                               _vp]),
     "dels_combine_workspace_bytes": (_sz, [_i, _i, _i]),
     "dels_combine_argmax": (_i, [_vp, _vp, _i, _vp, _f, _f, _i, _i, _vp, _vp, _vp, _vp, _sz, _vp]),
+    "dels_combine_argmax_noalloc": (_i, [_vp, _vp, _i, _vp, _f, _f, _i, _i, _vp, _vp, _vp, _vp]),
     "dels_verify_workspace_bytes": (_sz, [_i, _i, _i, _i]),
     "dels_verify_block": (_i, [_vp, _vp, _i, _i, _i, _i, _vp, _vp, _vp, _vp, _sz, _vp]),
     "dels_read_status": (_i, [_vp, _vp, ctypes.POINTER(ctypes.c_int32)]),
@@ -172,6 +174,15 @@ def dels_combine_argmax(long_logits, short_logits, dtype: int, log_prior, alpha:
     return lib().dels_combine_argmax(_ptr(long_logits), _ptr(short_logits), dtype, _ptr(log_prior), alpha, beta,
                                      rows, V, _ptr(out_token), _ptr(out_logprob), _ptr(out_top2_gap),
                                      _ptr(workspace), workspace_bytes, _stream(stream))
+
+
+def dels_combine_argmax_noalloc(long_logits, short_logits, dtype: int, log_prior, alpha: float, beta: float,
+                                rows: int, V: int, out_token, out_logprob, out_top2_gap, stream=None) -> int:
+    """dels_combine_argmax without a workspace: uses the library's fixed 4 MiB
+    device scratch (for callers that cannot allocate device memory)."""
+    return lib().dels_combine_argmax_noalloc(_ptr(long_logits), _ptr(short_logits), dtype, _ptr(log_prior), alpha,
+                                             beta, rows, V, _ptr(out_token), _ptr(out_logprob), _ptr(out_top2_gap),
+                                             _stream(stream))
 
 
 def dels_verify_workspace_bytes(B: int, n: int, V: int, dtype: int) -> int:

@@ -507,6 +507,7 @@ const char* dels_status_string(int code) {
     case DELS_ERR_WORKSPACE: return "workspace missing or too small";
     case DELS_ERR_UNSUPPORTED: return "unsupported head configuration";
     case DELS_ERR_CUDA: return "CUDA call failed";
+    case DELS_ERR_TOO_LARGE: return "problem exceeds the fixed no-allocation scratch";
     case DELS_STATUS_NONFINITE: return "device: non-finite logits";
     case DELS_STATUS_TIMEOUT: return "device: bounded wait expired";
     case DELS_STATUS_BAD_TOKEN: return "device: draft token out of range";
