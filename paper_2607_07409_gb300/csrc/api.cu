@@ -241,7 +241,9 @@ bool plan_combine(Gemm& g, int B, int V, int n, const void* X, int K, const void
   a.partials = partials;
   a.partial_ld = partial_ld;
   a.status = status;
-  const int l_fixed = 2 * a.l_boxes * a.l_box_rows * 128;
+  const int grid = std::min(a.num_o_tiles, std::max(1, sms));
+  a.max_items_per_cta = (a.num_o_tiles + grid - 1) / grid;
+  const int l_fixed = 2 * a.l_boxes * a.l_box_rows * 128 + a.max_items_per_cta * n_tile * 4;
   a.a_resident = (a.seg_chunks[0] <= 4) ? 1 : 0;
   if (a.a_resident) {
     a.stages = pick_stages(a, n_tile * 128, a.seg_chunks[0] * 128 * 128 + l_fixed);
@@ -256,7 +258,7 @@ bool plan_combine(Gemm& g, int B, int V, int n, const void* X, int K, const void
     return false;
   g.mA1 = g.mA0;
   g.mB1 = g.mB0;
-  g.grid = std::min(a.num_o_tiles, std::max(1, sms));
+  g.grid = grid;
   g.smem = tc_gemm_smem_bytes(a);
   return true;
 }
@@ -718,9 +720,14 @@ int dels_draft_block(const dels_local_head* head, const void* long_logits, dels_
       void* rr = at<void>(workspace, L.r);
       mb.D = D;
       mb.dest = eg;
-      DELS_CUDA(cudaMemsetAsync(h, 0, (size_t)B * H * 4, s));
-      DELS_CUDA(cudaMemsetAsync(hb, 0, (size_t)B * H * 2, s));
+      // h_0 = 0: the position-0 merge clears the recurrent state
+      mb.zero_f32 = h;
+      mb.zero_bf16 = hb;
+      mb.zero_len = H;
       r = draft_position0(long_logits, logit_dtype, B, n, V, partials, L.partial_ld, status, mb, sms, s);
+      mb.zero_f32 = nullptr;
+      mb.zero_bf16 = nullptr;
+      mb.zero_len = 0;
       if (r != DELS_OK || n == 1) return r;
       if (bf) {
         Gemm gg, gr, gv;

@@ -83,6 +83,29 @@ __device__ __forceinline__ void lse_chunk(const float (&x)[K], float best, float
   s += acc;
 }
 
+// Hardware base-2 exponential (PTX ex2.approx, flush-to-zero); -inf -> 0.
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+constexpr float kLog2e = 1.4426950408889634f;
+
+// lse_chunk with the exponent pre-scaled to base 2: one FFMA + one ex2 per
+// element (exp(x - best) = 2^(x*log2e - best*log2e)).
+template <int K>
+__device__ __forceinline__ void lse_chunk_ex2(const float (&x)[K], float best, float& m, float& s) {
+  if (best == -INFINITY) return;
+  const float nb = -best * kLog2e;
+  s *= ex2_approx(fmaf(m, kLog2e, nb));
+  m = best;
+  float acc = 0.f;
+#pragma unroll
+  for (int i = 0; i < K; ++i) acc += ex2_approx(fmaf(x[i], kLog2e, nb));
+  s += acc;
+}
+
 // Merge two partial states (any index order). Ties on the value go to the
 // lower index; the runner-up becomes the larger of the loser's top-1 and the
 // winner's runner-up.
@@ -161,6 +184,12 @@ __device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t by
                : "memory");
 }
 
+// Adds `bytes` to the barrier's expected transaction count without arriving.
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.expect_tx.relaxed.cta.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+               : "memory");
+}
+
 __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   uint32_t ok;
   asm volatile(
@@ -190,6 +219,15 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint64
   }
   return true;
 }
+
+// ----------------------------------------------------------------------------
+// programmatic dependent launch: a kernel launched with the programmatic
+// stream-serialization attribute may start before its predecessor finishes;
+// it must call pdl_wait() before touching anything the predecessor writes.
+// Both are no-ops for a normally launched kernel.
+// ----------------------------------------------------------------------------
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 
 // ----------------------------------------------------------------------------
 // TMA (tiled tensor copies global -> shared, completion on an mbarrier)

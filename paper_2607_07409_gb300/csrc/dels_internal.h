@@ -4,6 +4,7 @@
 
 #include <cstddef>
 #include <cstdint>
+#include <utility>
 #include <cuda_runtime.h>
 #include <cuda.h>
 
@@ -17,6 +18,25 @@ constexpr int kMaxBatchTile = 128;         // tcgen05 M: batch rows per tile
 constexpr uint64_t kWaitBudgetNs = 2000000000ull;   // bounded device waits: 2 s
 
 struct RowAcc;
+
+// Launch with programmatic stream serialization: the kernel may begin while
+// its predecessor on the stream is still running; it waits for it with
+// griddepcontrol.wait before touching the predecessor's outputs.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                       Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
 
 // ---- row reductions (combine / verify / draft position 0) -------------------
 struct RowsArgs {
@@ -67,6 +87,10 @@ struct MergeArgs {
   int table_f32;
   int D, window;
   void* dest;                    // [B, window*D] same dtype as table
+  // optional per-row zeroing (recurrent state at the start of a block)
+  float* zero_f32;               // [B, zero_len]
+  uint16_t* zero_bf16;           // [B, zero_len]
+  int zero_len;
 };
 cudaError_t launch_draft_merge(const MergeArgs& a, cudaStream_t s);
 
@@ -85,6 +109,7 @@ struct TcGemmArgs {
   int epi;
   int a_resident;                // A (activations) loaded once per CTA
   int stages;
+  int max_items_per_cta;         // EPI_COMBINE: sizes the per-CTA prior slice in smem
   // EPI_STORE
   int act;
   float* out_f32;                // [split][B][ldo] (or final when total_splits == 1)

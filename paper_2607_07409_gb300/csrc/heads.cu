@@ -26,6 +26,8 @@ __device__ __forceinline__ float bf16_to_f(uint16_t u) { return __uint_as_float(
 //   c = tanh(gi_n + r * gh_n), h' = (1 - z) * c + z * h
 __global__ void k_gru_gates(const float* __restrict__ part, int S0, int S1, int B, int H, float* __restrict__ h,
                             uint16_t* __restrict__ h_bf16) {
+  if (threadIdx.x == 0) pdl_trigger();
+  pdl_wait();
   const long long total = (long long)B * H;
   const long long split_stride = (long long)B * 3 * H;
   for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < total;
@@ -56,6 +58,8 @@ __global__ void k_gru_gates(const float* __restrict__ part, int S0, int S1, int 
 __global__ void k_splitk_finish(const float* __restrict__ part, int S, int B, int O,
                                 const float* __restrict__ residual, int act, float* __restrict__ out_f32, int ld_f32,
                                 uint16_t* __restrict__ out_bf16, int ld_bf16) {
+  if (threadIdx.x == 0) pdl_trigger();
+  pdl_wait();
   const long long total = (long long)B * O;
   for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < total;
        e += (long long)gridDim.x * blockDim.x) {
@@ -90,6 +94,8 @@ __device__ __forceinline__ float block_sum(float v) {
 
 // out = bf16( x / sqrt(mean(x^2) + 1e-6) ), one CTA per row
 __global__ void k_rmsnorm_bf16(const float* __restrict__ x, int D, int ld, uint16_t* __restrict__ out) {
+  if (threadIdx.x == 0) pdl_trigger();
+  pdl_wait();
   const float* row = x + (long long)blockIdx.x * ld;
   float ss = 0.f;
   for (int i = threadIdx.x; i < D; i += blockDim.x) ss += row[i] * row[i];
@@ -101,6 +107,8 @@ __global__ void k_rmsnorm_bf16(const float* __restrict__ x, int D, int ld, uint1
 // t = E[x] + P[pos] (float32), a = bf16(RMSNorm(t)); one CTA per row
 __global__ void k_xfmr_embed(const uint16_t* __restrict__ e_rows, const uint16_t* __restrict__ pos_table, int pos,
                              int D, float* __restrict__ t_out, uint16_t* __restrict__ a_bf16) {
+  if (threadIdx.x == 0) pdl_trigger();
+  pdl_wait();
   const long long off = (long long)blockIdx.x * D;
   float ss = 0.f;
   for (int i = threadIdx.x; i < D; i += blockDim.x) {
@@ -117,6 +125,8 @@ __global__ void k_xfmr_embed(const uint16_t* __restrict__ e_rows, const uint16_t
 // block: one CTA per (row, head); o = softmax(q k^T / sqrt(dh)) v, stored bf16.
 __global__ void k_attention(const float* __restrict__ q, const float* __restrict__ kc, const float* __restrict__ vc,
                             int D, int nh, int npos, int cache_ld_pos, uint16_t* __restrict__ o_bf16) {
+  if (threadIdx.x == 0) pdl_trigger();
+  pdl_wait();
   const int b = blockIdx.x / nh, hd = blockIdx.x % nh;
   const int dh = D / nh;
   __shared__ float w[64];
@@ -150,6 +160,8 @@ __global__ void k_attention(const float* __restrict__ q, const float* __restrict
 template <int BMAX>
 __global__ void k_gemv_f32(const float* __restrict__ X, int ldx, const float* __restrict__ W, int B, int O, int K,
                            int act, float* __restrict__ Y, int ldy) {
+  if (threadIdx.x == 0) pdl_trigger();
+  pdl_wait();
   const int lane = threadIdx.x & 31;
   const int o = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   if (o >= O) return;
@@ -183,6 +195,8 @@ __global__ void __launch_bounds__(256) k_vocab_combine_f32(const float* __restri
                                                            const float* __restrict__ prior, float alpha, float beta,
                                                            int V, void* partials, int partial_ld, int nchunks,
                                                            int* status) {
+  if (threadIdx.x == 0) pdl_trigger();
+  pdl_wait();
   const int chunk = blockIdx.x % nchunks, b = blockIdx.x / nchunks;
   const int per = (V + nchunks - 1) / nchunks;
   const int v0 = chunk * per, v1 = min(V, v0 + per);
@@ -227,47 +241,41 @@ inline int grid_for(long long total, int threads) {
 
 cudaError_t launch_gru_gates(const float* part, int S0, int S1, int B, int H, float* h, uint16_t* h_bf16,
                              cudaStream_t s) {
-  k_gru_gates<<<grid_for((long long)B * H, 256), 256, 0, s>>>(part, S0, S1, B, H, h, h_bf16);
-  return cudaGetLastError();
+  return launch_pdl(k_gru_gates, dim3(grid_for((long long)B * H, 256)), dim3(256), 0, s, part, S0, S1, B, H, h, h_bf16);
 }
 
 cudaError_t launch_splitk_finish(const float* part, int S, int B, int O, const float* residual, int act,
                                  float* out_f32, int ld_f32, uint16_t* out_bf16, int ld_bf16, cudaStream_t s) {
-  k_splitk_finish<<<grid_for((long long)B * O, 256), 256, 0, s>>>(part, S, B, O, residual, act, out_f32, ld_f32,
-                                                                  out_bf16, ld_bf16);
-  return cudaGetLastError();
+  return launch_pdl(k_splitk_finish, dim3(grid_for((long long)B * O, 256)), dim3(256), 0, s, part, S, B, O, residual,
+                    act, out_f32, ld_f32, out_bf16, ld_bf16);
 }
 
 cudaError_t launch_rmsnorm_bf16(const float* x, int B, int D, int ld, uint16_t* out, cudaStream_t s) {
-  k_rmsnorm_bf16<<<B, 256, 0, s>>>(x, D, ld, out);
-  return cudaGetLastError();
+  return launch_pdl(k_rmsnorm_bf16, dim3(B), dim3(256), 0, s, x, D, ld, out);
 }
 
 cudaError_t launch_xfmr_embed(const uint16_t* e_rows, const uint16_t* pos_table, int pos, int B, int D,
                               float* t_out, uint16_t* a_bf16, cudaStream_t s) {
-  k_xfmr_embed<<<B, 256, 0, s>>>(e_rows, pos_table, pos, D, t_out, a_bf16);
-  return cudaGetLastError();
+  return launch_pdl(k_xfmr_embed, dim3(B), dim3(256), 0, s, e_rows, pos_table, pos, D, t_out, a_bf16);
 }
 
 cudaError_t launch_attention(const float* q, const float* kcache, const float* vcache, int B, int D, int nh,
                              int npos, int cache_ld_pos, uint16_t* o_bf16, cudaStream_t s) {
-  k_attention<<<B * nh, 128, 0, s>>>(q, kcache, vcache, D, nh, npos, cache_ld_pos, o_bf16);
-  return cudaGetLastError();
+  return launch_pdl(k_attention, dim3(B * nh), dim3(128), 0, s, q, kcache, vcache, D, nh, npos, cache_ld_pos, o_bf16);
 }
 
 cudaError_t launch_gemv_f32(const float* X, int ldx, const float* W, int B, int O, int K, int act, float* Y, int ldy,
                             cudaStream_t s) {
   const int warps = 8;
-  k_gemv_f32<8><<<(O + warps - 1) / warps, warps * 32, 0, s>>>(X, ldx, W, B, O, K, act, Y, ldy);
-  return cudaGetLastError();
+  return launch_pdl(k_gemv_f32<8>, dim3((O + warps - 1) / warps), dim3(warps * 32), 0, s, X, ldx, W, B, O, K, act, Y,
+                    ldy);
 }
 
 cudaError_t launch_vocab_combine_f32(const float* feat, int K, const float* Wv, const void* longp, int long_f32,
                                      long long ld_long, const float* prior, float alpha, float beta, int B, int V,
                                      void* partials, int partial_ld, int nchunks, int* status, cudaStream_t s) {
-  k_vocab_combine_f32<<<B * nchunks, 256, 0, s>>>(feat, K, Wv, longp, long_f32, ld_long, prior, alpha, beta, V,
-                                                  partials, partial_ld, nchunks, status);
-  return cudaGetLastError();
+  return launch_pdl(k_vocab_combine_f32, dim3(B * nchunks), dim3(256), 0, s, feat, K, Wv, longp, long_f32, ld_long,
+                    prior, alpha, beta, V, partials, partial_ld, nchunks, status);
 }
 
 }  // namespace dels

@@ -92,6 +92,8 @@ __device__ __forceinline__ void block_reduce_rows(const RowAcc (&acc)[R], RowAcc
 // ----------------------------------------------------------------------------
 template <typename T, int R, bool VEC, bool SH, bool PR, bool FINAL>
 __global__ void __launch_bounds__(kRowsThreads) k_combine_rows(RowsArgs a) {
+  if (threadIdx.x == 0) pdl_trigger();
+  pdl_wait();
   const int chunk = blockIdx.x % a.nchunks;
   const int group = blockIdx.x / a.nchunks;
   const int r0 = group * R;
@@ -234,6 +236,8 @@ __device__ __forceinline__ ArgAcc argacc_warp_reduce(ArgAcc a) {
 
 template <typename T, bool VEC>
 __global__ void __launch_bounds__(kRowsThreads) k_verify_rows(RowsArgs a) {
+  if (threadIdx.x == 0) pdl_trigger();
+  pdl_wait();
   const int chunk = blockIdx.x % a.nchunks;
   const int row = blockIdx.x / a.nchunks;        // b * (n + 1) + j
   const int c0 = chunk * a.chunk_cols;
@@ -330,7 +334,15 @@ __global__ void __launch_bounds__(kRowsThreads) k_verify_rows(RowsArgs a) {
 // local head's next input rows
 // ----------------------------------------------------------------------------
 __global__ void __launch_bounds__(256) k_draft_merge(MergeArgs a) {
+  if (threadIdx.x == 0) pdl_trigger();
+  pdl_wait();
   const int b = blockIdx.x;
+  if (a.zero_len > 0) {
+    for (int i = threadIdx.x; i < a.zero_len; i += blockDim.x) {
+      if (a.zero_f32) a.zero_f32[(long long)b * a.zero_len + i] = 0.f;
+      if (a.zero_bf16) a.zero_bf16[(long long)b * a.zero_len + i] = 0;
+    }
+  }
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   __shared__ RowAcc red[8];
   __shared__ int s_tok;
@@ -376,10 +388,8 @@ cudaError_t launch_combine_t(const RowsArgs& a, bool finalize, cudaStream_t s) {
   const long long grid = (long long)groups * a.nchunks;
   if (grid == 0) return cudaSuccess;
   if (finalize)
-    k_combine_rows<T, R, VEC, SH, PR, true><<<(unsigned)grid, kRowsThreads, 0, s>>>(a);
-  else
-    k_combine_rows<T, R, VEC, SH, PR, false><<<(unsigned)grid, kRowsThreads, 0, s>>>(a);
-  return cudaGetLastError();
+    return launch_pdl(k_combine_rows<T, R, VEC, SH, PR, true>, dim3((unsigned)grid), dim3(kRowsThreads), 0, s, a);
+  return launch_pdl(k_combine_rows<T, R, VEC, SH, PR, false>, dim3((unsigned)grid), dim3(kRowsThreads), 0, s, a);
 }
 
 template <typename T, int R, bool VEC>
@@ -428,20 +438,17 @@ cudaError_t launch_combine_rows(const RowsArgs& a, dels_dtype dt, bool vec, bool
 cudaError_t launch_verify_rows(const RowsArgs& a, dels_dtype dt, bool vec, cudaStream_t s) {
   const long long grid = (long long)a.rows * a.nchunks;
   if (grid == 0) return cudaSuccess;
-  if (dt == DELS_BF16) {
-    if (vec) k_verify_rows<uint16_t, true><<<(unsigned)grid, kRowsThreads, 0, s>>>(a);
-    else k_verify_rows<uint16_t, false><<<(unsigned)grid, kRowsThreads, 0, s>>>(a);
-  } else {
-    if (vec) k_verify_rows<float, true><<<(unsigned)grid, kRowsThreads, 0, s>>>(a);
-    else k_verify_rows<float, false><<<(unsigned)grid, kRowsThreads, 0, s>>>(a);
-  }
-  return cudaGetLastError();
+  const dim3 g((unsigned)grid), blk(kRowsThreads);
+  if (dt == DELS_BF16)
+    return vec ? launch_pdl(k_verify_rows<uint16_t, true>, g, blk, 0, s, a)
+               : launch_pdl(k_verify_rows<uint16_t, false>, g, blk, 0, s, a);
+  return vec ? launch_pdl(k_verify_rows<float, true>, g, blk, 0, s, a)
+             : launch_pdl(k_verify_rows<float, false>, g, blk, 0, s, a);
 }
 
 cudaError_t launch_draft_merge(const MergeArgs& a, cudaStream_t s) {
   if (a.B == 0) return cudaSuccess;
-  k_draft_merge<<<a.B, 256, 0, s>>>(a);
-  return cudaGetLastError();
+  return launch_pdl(k_draft_merge, dim3(a.B), dim3(256), 0, s, a);
 }
 
 }  // namespace dels
