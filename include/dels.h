@@ -244,7 +244,8 @@ enum {
   DELS_KCLASS_POS0 = 4,          /* position-0 row reduction                              */
   DELS_KCLASS_VERIFY = 5,        /* verification                                          */
   DELS_KCLASS_COMBINE = 6,       /* dels_combine_argmax                                   */
-  DELS_KCLASS_COUNT = 7
+  DELS_KCLASS_DRAFT_BLOCK = 7,   /* persistent per-block drafting kernel (whole block)    */
+  DELS_KCLASS_COUNT = 8
 };
 
 /*

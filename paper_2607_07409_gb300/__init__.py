@@ -74,7 +74,8 @@ _SIGS = {
 }
 
 # kernel classes of the optional profiler
-KCLASS = {"vocab_combine": 0, "head_gemm": 1, "head_misc": 2, "merge": 3, "pos0": 4, "verify": 5, "combine": 6}
+KCLASS = {"vocab_combine": 0, "head_gemm": 1, "head_misc": 2, "merge": 3, "pos0": 4, "verify": 5, "combine": 6,
+          "draft_block": 7}
 
 
 def exported_symbols():

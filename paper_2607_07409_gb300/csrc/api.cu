@@ -4,6 +4,7 @@
 // projection + fused combine -> merge/feedback for positions 1..n-1).
 #include <algorithm>
 #include <cmath>
+#include <cstdlib>
 #include <cstring>
 #include <mutex>
 #include <vector>
@@ -144,10 +145,10 @@ struct Gemm {
 
 constexpr int kSmemReserve = 512 + 2 * 128 * 16 + 1024 + 256;   // barriers, reduction scratch, alignment slack
 
-// A = X [B, K] bf16 (row pitch K*2); W = [O, K] bf16.
-bool map_x(CUtensorMap* m, const void* X, int B, int K) {
+// A = X [B, K] bf16 (row pitch K*2), boxes of `box_rows` rows; W = [O, K] bf16.
+bool map_x(CUtensorMap* m, const void* X, int B, int K, int box_rows) {
   return encode_tmap_2d(m, X, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (uint64_t)K, (uint64_t)B, (uint64_t)K * 2, 64,
-                        128, CU_TENSOR_MAP_SWIZZLE_128B);
+                        (uint32_t)box_rows, CU_TENSOR_MAP_SWIZZLE_128B);
 }
 bool map_w(CUtensorMap* m, const void* W, int O, int K, int n_tile) {
   return encode_tmap_2d(m, W, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (uint64_t)K, (uint64_t)O, (uint64_t)K * 2, 64,
@@ -192,9 +193,12 @@ bool plan_store(Gemm& g, int B, int O, const void* X0, const void* W0, int K0, c
   a.ldo_bf16 = ldo_bf16;
   a.status = status;
   a.stages = pick_stages(a, 128 * 128 + n_tile * 128, 0);
-  if (!map_x(&g.mA0, X0, B, K0) || !map_w(&g.mB0, W0, O, K0, n_tile)) return false;
+  // only the B real rows are loaded; the tile's other rows feed unused outputs
+  a.a_box_rows = std::min(128, (B + 7) / 8 * 8);
+  a.a_copies = 1;
+  if (!map_x(&g.mA0, X0, B, K0, a.a_box_rows) || !map_w(&g.mB0, W0, O, K0, n_tile)) return false;
   if (K1 > 0) {
-    if (!map_x(&g.mA1, X1, B, K1) || !map_w(&g.mB1, W1, O, K1, n_tile)) return false;
+    if (!map_x(&g.mA1, X1, B, K1, a.a_box_rows) || !map_w(&g.mB1, W1, O, K1, n_tile)) return false;
   } else {
     g.mA1 = g.mA0;
     g.mB1 = g.mB0;
@@ -251,7 +255,13 @@ bool plan_combine(Gemm& g, int B, int V, int n, const void* X, int K, const void
     a.stages = pick_stages(a, 128 * 128 + n_tile * 128, l_fixed);
   }
   const int es = a.long_f32 ? 4 : 2;
-  if (!map_x(&g.mA0, X, B, K) || !map_w(&g.mB0, Wv, V, K, n_tile)) return false;
+  // Rows of the A tile: the B requests rounded up to whole TMEM lane
+  // quadrants; when that is 32 or 64 rows, 4 or 2 copies fill the tile so
+  // every epilogue warp owns live rows (the copies split the columns).
+  const int rpc = (B + 31) / 32 * 32;
+  a.a_box_rows = rpc;
+  a.a_copies = (rpc == 32) ? 4 : (rpc == 64 ? 2 : 1);
+  if (!map_x(&g.mA0, X, B, K, a.a_box_rows) || !map_w(&g.mB0, Wv, V, K, n_tile)) return false;
   if (!encode_tmap_3d(&g.mL, longp, a.long_f32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16,
                       es, (uint64_t)V, (uint64_t)n, (uint64_t)B, (uint64_t)V * es, (uint64_t)n * V * es,
                       (uint32_t)a.l_box_cols, 1, (uint32_t)a.l_box_rows, CU_TENSOR_MAP_SWIZZLE_128B))
@@ -265,6 +275,16 @@ bool plan_combine(Gemm& g, int B, int V, int n, const void* X, int K, const void
 
 cudaError_t run(const Gemm& g, cudaStream_t s) {
   return launch_tc_gemm(g.a, &g.mA0, &g.mB0, &g.mA1, &g.mB1, &g.mL, g.grid, g.smem, s);
+}
+
+// bf16 GRU heads have two drafting paths that compute the same block: the
+// per-position kernel sequence chained by programmatic dependent launch (the
+// default, and the faster one as measured), and one cooperative persistent
+// launch per block with grid-wide barriers between phases, selected by
+// DELS_DRAFT_PERSISTENT=1 in the environment.
+bool persistent_enabled() {
+  const char* e = std::getenv("DELS_DRAFT_PERSISTENT");
+  return e && e[0] == '1';
 }
 
 // ------------------------------------------------------------ draft layout
@@ -720,6 +740,58 @@ int dels_draft_block(const dels_local_head* head, const void* long_logits, dels_
       void* rr = at<void>(workspace, L.r);
       mb.D = D;
       mb.dest = eg;
+      if (bf && persistent_enabled() && B <= sms && R <= 256) {
+        // one cooperative launch for the whole block
+        Gemm gg, gr, gv;
+        if (!plan_store(gg, B, 3 * H, eg, head->w[0], D, hb, head->w[1], H, 128, L.gru_s0, L.gru_s1, ACT_NONE,
+                        gpart, nullptr, 0, status, sms) ||
+            !plan_store(gr, B, R, hb, head->w[2], H, nullptr, nullptr, 0, 32, 1, 0, ACT_SILU, nullptr,
+                        static_cast<uint16_t*>(rr), R, status, sms) ||
+            !plan_combine(gv, B, V, n, rr, R, head->w_vocab, long_logits, logit_dtype, log_prior, alpha, beta,
+                          partials, L.partial_ld, status, sms))
+          return DELS_ERR_CUDA;
+        PersistGruArgs P{};
+        P.B = B; P.n = n; P.V = V; P.D = D; P.H = H; P.R = R;
+        P.stages = 12;
+        P.gru = gg.a;
+        P.gru.out_bmajor = 1;                    // partials as [split][3H][B]
+        P.gru.ldb = B;
+        P.gru.out_split_stride = (long long)3 * H * B;
+        P.rank = gr.a;
+        P.vocab = gv.a;
+        P.gru.stages = P.rank.stages = P.vocab.stages = P.stages;
+        P.vocab.max_items_per_cta = (P.vocab.num_o_tiles + sms - 1) / sms;
+        P.emb = static_cast<const uint16_t*>(head->emb);
+        P.longp = long_logits;
+        P.long_f32 = logit_dtype == DELS_F32;
+        P.eg = static_cast<uint16_t*>(eg);
+        P.h = h;
+        P.hb = hb;
+        P.gpart = gpart;
+        P.r = static_cast<uint16_t*>(rr);
+        P.partials = partials;
+        P.partial_ld = L.partial_ld;
+        P.pos0_chunks = std::max(1, std::min(sms / B, L.partial_ld));
+        P.pos0_chunk_cols = (int)round_up((size_t)((V + P.pos0_chunks - 1) / P.pos0_chunks), 8);
+        P.tokens = out_tokens;
+        P.out_lp = out_logprob;
+        P.out_gap = out_top2_gap;
+        P.status = status;
+        P.grid_bar = at<unsigned>(workspace, 0) + 16;      // counter at byte 64, generation at byte 192
+        P.abort_global = at<int>(workspace, 0) + 4;        // byte 16
+        // as many pipeline stages as shared memory holds (at most 12)
+        size_t smem = draft_gru_smem_bytes(P);
+        while (P.stages > 2 && (int)smem > device_max_smem_optin()) {
+          --P.stages;
+          smem = draft_gru_smem_bytes(P);
+        }
+        P.gru.stages = P.rank.stages = P.vocab.stages = P.stages;
+        if (P.vocab.a_resident && P.vocab.seg_chunks[0] <= P.stages && (int)smem <= device_max_smem_optin()) {
+          const CUtensorMap maps[9] = {gg.mA0, gg.mB0, gg.mA1, gg.mB1, gr.mA0, gr.mB0, gv.mA0, gv.mB0, gv.mL};
+          { PROF(DELS_KCLASS_DRAFT_BLOCK); DELS_CUDA(launch_draft_gru(P, maps, sms, smem, s)); }
+          return DELS_OK;
+        }
+      }
       // h_0 = 0: the position-0 merge clears the recurrent state
       mb.zero_f32 = h;
       mb.zero_bf16 = hb;

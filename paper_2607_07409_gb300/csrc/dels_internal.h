@@ -110,6 +110,8 @@ struct TcGemmArgs {
   int a_resident;                // A (activations) loaded once per CTA
   int stages;
   int max_items_per_cta;         // EPI_COMBINE: sizes the per-CTA prior slice in smem
+  int a_box_rows;                // activation rows per TMA box (the map's box height)
+  int a_copies;                  // copies of the activation rows stacked in the 128-row tile
   // EPI_STORE
   int act;
   float* out_f32;                // [split][B][ldo] (or final when total_splits == 1)
@@ -117,6 +119,8 @@ struct TcGemmArgs {
   int ldo;
   uint16_t* out_bf16;            // [B][ldo_bf16] activation output (total_splits == 1)
   int ldo_bf16;
+  int out_bmajor;                // f32 output as [split][o][ldb] (batch index fastest): each warp
+  int ldb;                       // store instruction then writes one contiguous 128-byte line
   // EPI_COMBINE
   const float* prior;
   float alpha, beta;
@@ -134,6 +138,33 @@ cudaError_t launch_tc_gemm(const TcGemmArgs& a, const CUtensorMap* mA0, const CU
                            const CUtensorMap* mA1, const CUtensorMap* mB1, const CUtensorMap* mL, int grid,
                            size_t smem_bytes, cudaStream_t s);
 size_t tc_gemm_smem_bytes(const TcGemmArgs& a);
+
+// ---- persistent per-block drafting kernel (GRU head, bf16) --------------------
+struct PersistGruArgs {
+  int B, n, V, D, H, R;
+  int stages;                    // pipeline stages shared by the three GEMM phases
+  TcGemmArgs gru, rank, vocab;   // the tensor-core phases of one position
+  const uint16_t* emb;           // E_tgt [V, D]
+  const void* longp;             // [B, n, V]
+  int long_f32;
+  uint16_t* eg;                  // [B, D] gathered embeddings
+  float* h;                      // [H, B] GRU state (batch index fastest)
+  uint16_t* hb;                  // [B, H] its bf16 copy
+  float* gpart;                  // [S0 + S1][3H][B] gate-product partials (batch fastest)
+  uint16_t* r;                   // [B, R] low-rank state
+  void* partials;                // [B][partial_ld] RowAcc
+  int partial_ld;
+  int pos0_chunks, pos0_chunk_cols;
+  int32_t* tokens;
+  float* out_lp;
+  float* out_gap;
+  int* status;
+  unsigned* grid_bar;            // grid-barrier counter (workspace header)
+  int* abort_global;             // set by a CTA whose bounded wait expired
+};
+size_t draft_gru_smem_bytes(const PersistGruArgs& P);
+cudaError_t launch_draft_gru(const PersistGruArgs& P, const CUtensorMap* maps, int grid, size_t smem,
+                             cudaStream_t s);
 
 // ---- small head kernels -------------------------------------------------------
 cudaError_t launch_gru_gates(const float* part, int S0, int S1, int B, int H, float* h, uint16_t* h_bf16,

@@ -215,6 +215,20 @@ def test_draft_small_matches_oracle(name, stress):
     print(name, stress, info)
 
 
+@pytest.mark.parametrize("stress", [False, True])
+@pytest.mark.parametrize("name", ["gru", "gru_b64"])
+def test_draft_persistent_kernel_matches_oracle(name, stress, monkeypatch):
+    # the one-launch-per-block drafting path for bf16 GRU heads
+    monkeypatch.setenv("DELS_DRAFT_PERSISTENT", "1")
+    w = SMALL[name]
+    if stress:
+        w = synth.stress(w)
+    d = synth.make_inputs(w, device=DEV, target=False)
+    tok, lp, gap, W, prior = _draft(w, d)
+    info = check_draft(tok, lp, gap, _oracle_head(w, W), d["long"].cpu(), prior, w.alpha, w.beta, LP_TOL_BF16)
+    print(name, stress, info)
+
+
 def test_draft_zero_weight_is_dflash_argmax():
     w = synth.with_sizes(synth.stress(synth.WORKLOADS["qwen3_8b_batched"]), B=8, n=5, V=2048, weight=0.0,
                          head_d_model=128, head_d_hidden=64, head_d_rank=64)
