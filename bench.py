@@ -57,9 +57,8 @@ def parse_args():
 def dist_setup(n_expected):
     import torch
     import torch.distributed as dist
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
+    from paper_2607_07409_gb300 import replicas
+    world, rank, local = replicas.rank_info()
     if world > 1 and not dist.is_initialized():
         backend = "nccl" if torch.cuda.is_available() else "gloo"
         if backend == "nccl":
@@ -254,10 +253,14 @@ def run_ours(args):
     import synth
     import paper_2607_07409_gb300 as dels
 
+    from paper_2607_07409_gb300 import replicas
+
     world, rank, local = dist_setup(args.gpus)
     dev = torch.device(f"cuda:{local}")
     torch.cuda.set_device(dev)
-    w = synth.WORKLOADS[WORKLOAD]
+    # weak scaling: every replica drafts its own batch of the same shape
+    w0 = synth.WORKLOADS[WORKLOAD]
+    w = synth.with_sizes(w0, seed=replicas.replica_seed(w0.seed, rank))
     d = synth.make_inputs(w, device=dev)
     W = {k[5:]: v for k, v in d.items() if k.startswith("head.")}
     prior = dels.dels_prior_from_counts(d["counts"]).to(dev)
@@ -290,8 +293,7 @@ def run_ours(args):
         gpu_id = "GPU-" + str(torch.cuda.get_device_properties(dev).uuid)
     except Exception:
         pass
-    if world > 1:
-        dist.barrier()
+    replicas.barrier()
     torch.cuda.synchronize()
     with ClockSampler(gpu_id) as clk:
         e0.record(stream)
@@ -299,13 +301,8 @@ def run_ours(args):
             step(long, target)
         e1.record(stream)
         torch.cuda.synchronize()
-    if world > 1:
-        dist.barrier()
-    ms = e0.elapsed_time(e1)
-    t = torch.tensor([ms], dtype=torch.float64, device=dev)
-    if world > 1:
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    ms_max = float(t.item())
+    replicas.barrier()
+    ms_max = replicas.max_over_ranks(e0.elapsed_time(e1), dev)
 
     # ---- second timed region, same steps, with the library's per-kernel CUDA
     # events on (they serialise the kernels, so the value above is taken without)
@@ -330,7 +327,7 @@ def run_ours(args):
     if drafter.status() != 0 or dels.dels_read_status(vws) != 0:
         raise RuntimeError("device status set during the timed region")
     tokens_per_step = w.B * w.n
-    value = tokens_per_step * args.steps * world / (ms_max / 1e3)
+    value = replicas.job_throughput([tokens_per_step * args.steps] * world, ms_max)
 
     # ---- roofline of the dominant kernel (vocabulary projection + combine)
     peak, peak_kind = measured_peaks()
@@ -355,8 +352,7 @@ def run_ours(args):
     acc_h = torch.empty(w.B, dtype=torch.int32).pin_memory()
     bonus_h = torch.empty(w.B, dtype=torch.int32).pin_memory()
     k_e2e = max(1, min(args.e2e_steps, args.steps))
-    if world > 1:
-        dist.barrier()
+    replicas.barrier()
     torch.cuda.synchronize()
     f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     f0.record(stream)
@@ -369,11 +365,8 @@ def run_ours(args):
         bonus_h.copy_(bonus, non_blocking=True)
     f1.record(stream)
     torch.cuda.synchronize()
-    e2e_ms = f0.elapsed_time(f1)
-    te = torch.tensor([e2e_ms], dtype=torch.float64, device=dev)
-    if world > 1:
-        dist.all_reduce(te, op=dist.ReduceOp.MAX)
-    e2e_val = tokens_per_step * k_e2e * world / (float(te.item()) / 1e3)
+    e2e_ms = replicas.max_over_ranks(f0.elapsed_time(f1), dev)
+    e2e_val = replicas.job_throughput([tokens_per_step * k_e2e] * world, e2e_ms)
     h2d = long.numel() * long.element_size() + target.numel() * target.element_size()
     d2h = tok_h.numel() * 4 + acc_h.numel() * 4 + bonus_h.numel() * 4
 
