@@ -86,6 +86,11 @@ typedef enum {
  *     w_vocab = W_vocab [V, d_rank].
  *     h_j = GRU(E_tgt[x_{j-1}], h_{j-1}) bias-free (PyTorch gate form),
  *     h_0 = 0; r_j = SiLU(W_rank h_j); l_S = W_vocab r_j.
+ *     Optional, bf16 heads only: w[3] = G [V, 3*d_hidden] float32, the input
+ *     table G = E_tgt W_ih^T written by dels_gru_build_input_table. When set,
+ *     the input product W_ih E_tgt[x] of every step is read as row x of G
+ *     instead of being recomputed (same value up to float32 summation order);
+ *     w[0] is then not read by dels_draft_block.
  * DELS_HEAD_MLP: emb = E [V, d_model]; w[0] = W_1 [d_hidden, window*d_model];
  *     w[1] = W_2 [d_hidden, d_hidden] when n_layers == 2; w_vocab [V, d_hidden];
  *     d_rank must equal d_hidden. u = [E x_{j-1}; ...; E x_{j-window}] with
@@ -115,6 +120,30 @@ typedef struct {
   const void* w[8];
   const void* w_vocab;
 } dels_local_head;
+
+/* ---- GRU input table (head preparation, once per set of weights) -------- */
+
+/*
+ * The GRU's input product depends on the previous token only:
+ * W_ih E_tgt[x] = (E_tgt W_ih^T)[x] (Appendix A). Precomputing the table
+ * G = E_tgt W_ih^T [V, 3*d_hidden] float32 once per head trades HBM capacity
+ * (V * 3 * d_hidden * 4 bytes, 1.87 GB for V = 151936, d_hidden = 1024) for
+ * the W_ih stream of every drafted position (3*d_hidden*d_model*2 bytes).
+ * (The paper computes the product directly; this is an implementation
+ * choice with the same result up to float32 summation order.)
+ *
+ * dels_gru_input_table_bytes: bytes of G for this head and V; 0 if the head
+ * is not a bf16 GRU head.
+ * dels_gru_build_input_table: writes G into `table` [device], caller-owned,
+ * >= dels_gru_input_table_bytes bytes, 16-byte aligned. Reads head->emb and
+ * head->w[0] (bf16). `workspace` [device] >= 256 bytes, zero-filled, holds
+ * the device status word (read with dels_read_status). Asynchronous on
+ * `stream`; bf16 products with float32 accumulation on tensor cores.
+ * Returns DELS_OK or a negative host-detected error (nothing enqueued).
+ */
+size_t dels_gru_input_table_bytes(const dels_local_head* head, int V);
+int dels_gru_build_input_table(const dels_local_head* head, int V, float* table, size_t table_bytes,
+                               void* workspace, size_t workspace_bytes, dels_stream_t stream);
 
 /* ---- per-block drafting (Algorithm 1, temperature 0) --------------------- */
 

@@ -26,6 +26,7 @@ __all__ = [
     "dels_verify_workspace_bytes", "dels_verify_block",
     "dels_read_status", "dels_prior_from_counts", "dels_status_string", "dels_version",
     "dels_profile_enable", "dels_profile_reset", "dels_profile_read", "KCLASS",
+    "dels_gru_input_table_bytes", "dels_gru_build_input_table", "gru_input_table",
     "make_head", "Drafter", "dtype_code",
 ]
 
@@ -56,6 +57,8 @@ class LocalHead(ctypes.Structure):
 
 
 _SIGS = {
+    "dels_gru_input_table_bytes": (_sz, [ctypes.POINTER(LocalHead), _i]),
+    "dels_gru_build_input_table": (_i, [ctypes.POINTER(LocalHead), _i, _vp, _sz, _vp, _sz, _vp]),
     "dels_draft_workspace_bytes": (_sz, [ctypes.POINTER(LocalHead), _i, _i, _i]),
     "dels_draft_block": (_i, [ctypes.POINTER(LocalHead), _vp, _i, _vp, _f, _f, _i, _i, _i, _vp, _vp, _vp, _vp, _sz,
                               _vp]),
@@ -152,6 +155,34 @@ def dels_status_string(code: int) -> str:
     return lib().dels_status_string(int(code)).decode()
 
 
+def dels_gru_input_table_bytes(head: LocalHead, V: int) -> int:
+    return lib().dels_gru_input_table_bytes(ctypes.byref(head), V)
+
+
+def dels_gru_build_input_table(head: LocalHead, V: int, table, table_bytes: int, workspace, workspace_bytes: int,
+                               stream=None) -> int:
+    return lib().dels_gru_build_input_table(ctypes.byref(head), V, _ptr(table), table_bytes, _ptr(workspace),
+                                            workspace_bytes, _stream(stream))
+
+
+def gru_input_table(spec, weights: Dict[str, torch.Tensor], V: int, stream=None) -> torch.Tensor:
+    """The GRU input table G = E W_ih^T [V, 3*d_hidden] float32 of a bf16 GRU
+    head, built on the weights' device. Put it in the weights dict as
+    ``input_table`` to have dels_draft_block read it."""
+    head = make_head(spec, {k: v for k, v in weights.items() if k != "input_table"})
+    nbytes = dels_gru_input_table_bytes(head, V)
+    if nbytes == 0:
+        raise DelsError(-6, "dels_gru_input_table_bytes")
+    dev = weights["emb"].device
+    table = torch.empty(nbytes // 4, dtype=torch.float32, device=dev).view(V, -1)
+    ws = torch.zeros(256, dtype=torch.uint8, device=dev)
+    _check(dels_gru_build_input_table(head, V, table, nbytes, ws, 256, stream), "dels_gru_build_input_table")
+    st = dels_read_status(ws, stream)
+    if st != 0:
+        raise DelsError(st, "dels_gru_build_input_table (device status)")
+    return table
+
+
 def dels_draft_workspace_bytes(head: LocalHead, B: int, n: int, V: int) -> int:
     return lib().dels_draft_workspace_bytes(ctypes.byref(head), B, n, V)
 
@@ -232,7 +263,7 @@ def dels_profile_read(kernel_class: int):
 
 _KIND = {"gru": DELS_HEAD_GRU, "mlp": DELS_HEAD_MLP, "xfmr": DELS_HEAD_XFMR, "markov": DELS_HEAD_MARKOV}
 _SLOTS = {
-    "gru": ["w_ih", "w_hh", "w_rank"],
+    "gru": ["w_ih", "w_hh", "w_rank", "input_table"],
     "mlp": ["w1", "w2"],
     "xfmr": ["pos", "wq", "wk", "wv", "wo", "w1", "w2"],
     "markov": [],

@@ -289,6 +289,11 @@ bool persistent_enabled() {
 
 // ------------------------------------------------------------ draft layout
 
+// Input-table GRU path: output tile widths of the rank product (full K per
+// tile, SiLU epilogue) and of the recurrent product (split over K).
+constexpr int kRankTile = 32;
+constexpr int kHhTile = 64;
+
 struct Carve {
   size_t off = kHeaderBytes;
   size_t take(size_t bytes) {
@@ -306,6 +311,7 @@ struct DraftLayout {
   // GRU
   size_t eg = 0, h = 0, hb = 0, gpart = 0, r = 0;
   int gru_s0 = 0, gru_s1 = 0;
+  int rank_grid = 0, hh_splits = 0;          // input-table path: grouped rank + recurrent product
   // MLP
   size_t u = 0, mpart = 0, h1 = 0, h2 = 0;
   int mlp_s1 = 0, mlp_s2 = 0;
@@ -338,11 +344,13 @@ DraftLayout draft_layout(const dels_local_head* hd, int B, int n, int V) {
       if (bf) {
         L.gru_s0 = std::max(1, std::min((D + 63) / 64, sms / std::max(1, (3 * H + 127) / 128) - 1));
         L.gru_s1 = 1;
+        L.rank_grid = (R + kRankTile - 1) / kRankTile;
+        L.hh_splits = splits_for(3 * H, kHhTile, H, std::max(1, sms - L.rank_grid));
       } else {
         L.gru_s0 = 1;
         L.gru_s1 = 1;
       }
-      L.gpart = c.take((size_t)(L.gru_s0 + L.gru_s1) * B * 3 * H * 4);
+      L.gpart = c.take((size_t)std::max(L.gru_s0 + L.gru_s1, L.hh_splits) * B * 3 * H * 4);
       L.r = c.take((size_t)B * R * es);
       break;
     }
@@ -452,9 +460,10 @@ T* at(void* ws, size_t off) {
   return reinterpret_cast<T*>(static_cast<uint8_t*>(ws) + off);
 }
 
-// Position 0: x_0 = argmax l_L[b, 0, :], partials then merge (+ gather).
-int draft_position0(const void* long_logits, dels_dtype ldt, int B, int n, int V, void* partials, int partial_ld,
-                    int* status, const MergeArgs& merge_base, int sms, cudaStream_t s) {
+// Position 0: x_0 = argmax l_L[b, 0, :] as per-chunk records (no merge);
+// returns the number of records per request.
+int position0_rows(const void* long_logits, dels_dtype ldt, int B, int n, int V, void* partials, int partial_ld,
+                   int* status, int sms, cudaStream_t s, int* count) {
   RowsArgs a{};
   const int es = ldt == DELS_F32 ? 4 : 2;
   RowsPlan p = plan_rows(B, V, es, sms, true, partial_ld);
@@ -468,9 +477,19 @@ int draft_position0(const void* long_logits, dels_dtype ldt, int B, int n, int V
   a.partials = partials;
   a.partial_ld = partial_ld;
   a.status = status;
+  *count = p.nchunks;
   { PROF(DELS_KCLASS_POS0); DELS_CUDA(launch_combine_rows(a, ldt, true, false, s)); }
+  return DELS_OK;
+}
+
+// Position 0 merged (+ the gather of the next input).
+int draft_position0(const void* long_logits, dels_dtype ldt, int B, int n, int V, void* partials, int partial_ld,
+                    int* status, const MergeArgs& merge_base, int sms, cudaStream_t s) {
+  int count = 0;
+  const int r = position0_rows(long_logits, ldt, B, n, V, partials, partial_ld, status, sms, s, &count);
+  if (r != DELS_OK) return r;
   MergeArgs m = merge_base;
-  m.count = p.nchunks;
+  m.count = count;
   m.j = 0;
   { PROF(DELS_KCLASS_MERGE); DELS_CUDA(launch_draft_merge(m, s)); }
   return DELS_OK;
@@ -689,6 +708,44 @@ int dels_verify_block(const int32_t* draft_tokens, const void* target_logits, de
   return DELS_OK;
 }
 
+// ------------------------------------------------------- GRU input table
+
+size_t dels_gru_input_table_bytes(const dels_local_head* head, int V) {
+  if (!head || head->kind != DELS_HEAD_GRU || head->wdtype != DELS_BF16 || V < 1) return 0;
+  if (!head->emb || !head->w[0] || head->d_model <= 0 || head->d_hidden <= 0) return 0;
+  return (size_t)V * 3 * (size_t)head->d_hidden * 4;
+}
+
+int dels_gru_build_input_table(const dels_local_head* head, int V, float* table, size_t table_bytes,
+                               void* workspace, size_t workspace_bytes, dels_stream_t stream) {
+  if (!head || !table) return DELS_ERR_NULL_POINTER;
+  if (head->kind != DELS_HEAD_GRU || head->wdtype != DELS_BF16) return DELS_ERR_UNSUPPORTED;
+  if (!head->emb || !head->w[0]) return DELS_ERR_NULL_POINTER;
+  if (!workspace || workspace_bytes < kHeaderBytes) return DELS_ERR_WORKSPACE;
+  const int D = head->d_model, H = head->d_hidden;
+  if (V < 1 || D < 16 || D % 16 || D > 65536 || H < 16 || H % 16 || H > 65536) return DELS_ERR_BAD_SHAPE;
+  if (!aligned16(head->emb) || !aligned16(head->w[0]) || !aligned16(table) || !aligned16(workspace))
+    return DELS_ERR_ALIGNMENT;
+  if (table_bytes < dels_gru_input_table_bytes(head, V)) return DELS_ERR_WORKSPACE;
+  const int sms = device_sm_count();
+  if (sms <= 0) return DELS_ERR_CUDA;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  int* status = at<int>(workspace, 0);
+  const uint16_t* E = static_cast<const uint16_t*>(head->emb);
+  // G[v0 : v0 + 128] = E[v0 : v0 + 128] W_ih^T, one 128-row block of the
+  // vocabulary per launch (the rows sit on the MMA's M like a batch).
+  for (int v0 = 0; v0 < V; v0 += kMaxBatchTile) {
+    const int rows = std::min(kMaxBatchTile, V - v0);
+    Gemm g;
+    if (!plan_store(g, rows, 3 * H, E + (size_t)v0 * D, head->w[0], D, nullptr, nullptr, 0, 128, 1, 0, ACT_NONE,
+                    table + (size_t)v0 * 3 * H, nullptr, 0, status, sms))
+      return DELS_ERR_CUDA;
+    PROF(DELS_KCLASS_HEAD_GEMM);
+    DELS_CUDA(run(g, s));
+  }
+  return DELS_OK;
+}
+
 // ------------------------------------------------------------------- draft
 
 size_t dels_draft_workspace_bytes(const dels_local_head* head, int B, int n, int V) {
@@ -791,6 +848,65 @@ int dels_draft_block(const dels_local_head* head, const void* long_logits, dels_
           { PROF(DELS_KCLASS_DRAFT_BLOCK); DELS_CUDA(launch_draft_gru(P, maps, sms, smem, s)); }
           return DELS_OK;
         }
+      }
+      const float* G = static_cast<const float*>(head->w[3]);
+      if (bf && G) {
+        // Input-table path (gi = G[x] with G = E W_ih^T precomputed): three
+        // launches per position —
+        //   gates(j)  merge x_{j-1} from the previous position's records, then
+        //             h_j from G[x_{j-1}], the partials of W_hh h_{j-1} and h_{j-1};
+        //   products  r_j = SiLU(W_rank h_j) side by side with the partials of
+        //             W_hh h_j (consumed by gates(j+1));
+        //   vocab(j)  l_S = W_vocab r_j fused with the combine -> per-CTA records.
+        // A last merge kernel decodes x_{n-1}. h_0 = 0 needs no clearing:
+        // gates(1) runs with no recurrent partials and h = 0.
+        mb.table = nullptr;
+        if (n == 1) return draft_position0(long_logits, logit_dtype, B, n, V, partials, L.partial_ld, status, mb, sms, s);
+        int count = 0;
+        r = position0_rows(long_logits, logit_dtype, B, n, V, partials, L.partial_ld, status, sms, s, &count);
+        if (r != DELS_OK) return r;
+        Gemm gr, gh, gv;
+        if (!plan_store(gr, B, R, hb, head->w[2], H, nullptr, nullptr, 0, kRankTile, 1, 0, ACT_SILU, nullptr,
+                        static_cast<uint16_t*>(rr), R, status, sms) ||
+            !plan_store(gh, B, 3 * H, hb, head->w[1], H, nullptr, nullptr, 0, kHhTile, L.hh_splits, 0, ACT_NONE,
+                        gpart, nullptr, 0, status, sms) ||
+            !plan_combine(gv, B, V, n, rr, R, head->w_vocab, long_logits, logit_dtype, log_prior, alpha, beta,
+                          partials, L.partial_ld, status, sms))
+          return DELS_ERR_CUDA;
+        // both products fit one wave next to each other
+        gh.grid = std::min(gh.grid, std::max(1, sms - gr.grid));
+        const TcGemmGroup hh{&gh.a, &gh.mA0, &gh.mB0, gh.grid};
+        GatesTableArgs ga{};
+        ga.partials = partials;
+        ga.partial_ld = L.partial_ld;
+        ga.tokens = out_tokens;
+        ga.out_lp = out_logprob;
+        ga.out_gap = out_top2_gap;
+        ga.n = n;
+        ga.G = G;
+        ga.V = V;
+        ga.part = gpart;
+        ga.B = B;
+        ga.H = H;
+        ga.h = h;
+        ga.h_bf16 = hb;
+        ga.status = status;
+        for (int j = 1; j < n; ++j) {
+          ga.count = j == 1 ? count : gv.grid;
+          ga.jprev = j - 1;
+          ga.S = j == 1 ? 0 : gh.a.total_splits;
+          { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_gru_gates_table(ga, s)); }
+          { PROF(DELS_KCLASS_HEAD_GEMM);
+            DELS_CUDA(launch_tc_gemm(gr.a, &gr.mA0, &gr.mB0, &gr.mA1, &gr.mB1, &gr.mL, gr.grid, gr.smem, s,
+                                     j + 1 < n ? &hh : nullptr)); }
+          gv.a.j = j;
+          { PROF(DELS_KCLASS_VOCAB_COMBINE); DELS_CUDA(run(gv, s)); }
+        }
+        MergeArgs m = mb;
+        m.count = gv.grid;
+        m.j = n - 1;
+        { PROF(DELS_KCLASS_MERGE); DELS_CUDA(launch_draft_merge(m, s)); }
+        return DELS_OK;
       }
       // h_0 = 0: the position-0 merge clears the recurrent state
       mb.zero_f32 = h;

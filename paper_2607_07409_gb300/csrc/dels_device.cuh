@@ -149,6 +149,27 @@ __device__ __forceinline__ bool rowacc_valid(const RowAcc& a) {
   return a.m > -INFINITY && a.m < INFINITY && a.s == a.s && a.s > 0.5f && a.s < INFINITY;
 }
 
+// A published RowAcc record (16 bytes), read past L1: records are written by
+// other CTAs of the same or an earlier grid.
+__device__ __forceinline__ RowAcc ld_rowacc_cg(const void* base, long long i) {
+  const float4 v = __ldcg(reinterpret_cast<const float4*>(base) + i);
+  RowAcc r;
+  r.m = v.x; r.s = v.y; r.second = v.z; r.idx = __float_as_int(v.w);
+  return r;
+}
+
+// Greedy decode of one fully merged row: token = argmax, logprob of the token
+// = -log(sum exp(l - max)), top-2 gap. A row with no finite value flags the
+// status word and yields token -1.
+__device__ __forceinline__ void write_decode(const RowAcc& r, long long out_i, int32_t* tok, float* lp, float* gap,
+                                             int* status) {
+  const bool ok = rowacc_valid(r);
+  if (!ok) raise_status(status, DELS_STATUS_NONFINITE);
+  tok[out_i] = ok ? r.idx : -1;
+  if (lp) lp[out_i] = ok ? -logf(r.s) : NAN;
+  if (gap) gap[out_i] = ok ? (r.m - r.second) : NAN;
+}
+
 // Argmax-only update (verification): value and lowest index.
 __device__ __forceinline__ void argmax_push(float x, int v, float& best, int& idx, bool& nan_seen) {
   const bool gt = x > best;

@@ -134,9 +134,18 @@ struct TcGemmArgs {
   int debug_skip_producer;       // test hook: producer never fills (exercises the bounded waits)
 };
 
+// One launch of k_tc_gemm runs one GEMM on `grid` CTAs, or two independent
+// GEMMs side by side ("grouped"): CTAs [0, grid) run the first, CTAs
+// [grid, grid + grid2) the second (single K segment, its own A/B maps).
+struct TcGemmGroup {
+  const TcGemmArgs* a;           // null: no second GEMM
+  const CUtensorMap* mA;
+  const CUtensorMap* mB;
+  int grid;
+};
 cudaError_t launch_tc_gemm(const TcGemmArgs& a, const CUtensorMap* mA0, const CUtensorMap* mB0,
                            const CUtensorMap* mA1, const CUtensorMap* mB1, const CUtensorMap* mL, int grid,
-                           size_t smem_bytes, cudaStream_t s);
+                           size_t smem_bytes, cudaStream_t s, const TcGemmGroup* second = nullptr);
 size_t tc_gemm_smem_bytes(const TcGemmArgs& a);
 
 // ---- persistent per-block drafting kernel (GRU head, bf16) --------------------
@@ -169,6 +178,27 @@ cudaError_t launch_draft_gru(const PersistGruArgs& P, const CUtensorMap* maps, i
 // ---- small head kernels -------------------------------------------------------
 cudaError_t launch_gru_gates(const float* part, int S0, int S1, int B, int H, float* h, uint16_t* h_bf16,
                              cudaStream_t s);
+// GRU step with a precomputed input table G = E W_ih^T [V, 3H] (f32), fused
+// with the merge of the previous position: x = the merged argmax of request
+// b's `count` records [B][partial_ld] (written to tokens/lp/gap at column
+// jprev), gi = G[x], gh = sum of S recurrent partials [S][B][3H] (S = 0:
+// gh = 0, the step from h = 0).
+struct GatesTableArgs {
+  const void* partials;
+  int partial_ld, count;
+  int32_t* tokens;               // [B, n]
+  float* out_lp;                 // [B, n]
+  float* out_gap;                // [B, n] or null
+  int n, jprev;
+  const float* G;                // [V, 3H]
+  int V;
+  const float* part;             // [S][B][3H]
+  int S, B, H;
+  float* h;                      // [B, H]
+  uint16_t* h_bf16;              // [B, H]
+  int* status;
+};
+cudaError_t launch_gru_gates_table(const GatesTableArgs& a, cudaStream_t s);
 cudaError_t launch_splitk_finish(const float* part, int S, int B, int O, const float* residual, int act,
                                  float* out_f32, int ld_f32, uint16_t* out_bf16, int ld_bf16, cudaStream_t s);
 cudaError_t launch_rmsnorm_bf16(const float* x, int B, int D, int ld, uint16_t* out, cudaStream_t s);

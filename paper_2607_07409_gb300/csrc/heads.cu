@@ -53,6 +53,75 @@ __global__ void k_gru_gates(const float* __restrict__ part, int S0, int S1, int 
   }
 }
 
+// The same GRU step with the input product read from a precomputed table:
+// gi = W_ih E[x] = G[x] with G = E W_ih^T [V, 3H] (row x holds the r, z, n
+// gate inputs of token x). The CTA first merges request b's per-CTA records
+// of the previous position into x (every CTA of the row does this; the
+// first also writes the decoded token, logprob and gap), so the merge costs
+// no launch of its own. gh is the sum of S recurrent partials [S][B][3H];
+// S = 0 means gh = 0 (the step from h = 0). A row that decoded to no token
+// (non-finite logits, already flagged) takes gi = 0.
+constexpr int kGatesThreads = 256;
+
+__global__ void __launch_bounds__(kGatesThreads) k_gru_gates_table(GatesTableArgs a) {
+  if (threadIdx.x == 0) pdl_trigger();
+  pdl_wait();
+  const int b = blockIdx.x;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int H = a.H;
+  // This thread's hidden unit (one per thread: the launch covers H with
+  // gridDim.y CTAs of kGatesThreads).
+  const int i = blockIdx.y * kGatesThreads + threadIdx.x;
+  const bool live = i < H;
+  // Loads that do not depend on the token go out before the merge.
+  float ghr = 0.f, ghz = 0.f, ghn = 0.f, hp = 0.f;
+  if (live) {
+    const long long split_stride = (long long)a.B * 3 * H;
+    const long long base = (long long)b * 3 * H + i;
+#pragma unroll 4
+    for (int sp = 0; sp < a.S; ++sp) {
+      const float* q = a.part + sp * split_stride + base;
+      ghr += __ldcg(q);
+      ghz += __ldcg(q + H);
+      ghn += __ldcg(q + 2 * H);
+    }
+    if (a.S > 0) hp = a.h[(long long)b * H + i];
+  }
+  __shared__ RowAcc red[kGatesThreads / 32];
+  __shared__ int s_tok;
+  RowAcc x = rowacc_init();
+  for (int k = threadIdx.x; k < a.count; k += kGatesThreads)
+    x = rowacc_merge(x, ld_rowacc_cg(a.partials, (long long)b * a.partial_ld + k));
+  x = rowacc_warp_reduce(x);
+  if (lane == 0) red[warp] = x;
+  __syncthreads();
+  if (warp == 0) {
+    x = lane < kGatesThreads / 32 ? red[lane] : rowacc_init();
+    x = rowacc_warp_reduce(x);
+    if (lane == 0) {
+      if (blockIdx.y == 0) write_decode(x, (long long)b * a.n + a.jprev, a.tokens, a.out_lp, a.out_gap, a.status);
+      s_tok = rowacc_valid(x) ? x.idx : -1;
+    }
+  }
+  __syncthreads();
+  if (!live) return;
+  const int tok = s_tok;
+  float gir = 0.f, giz = 0.f, gin = 0.f;
+  if (tok >= 0 && tok < a.V) {
+    const float* g = a.G + (long long)tok * 3 * H + i;
+    gir = __ldg(g);
+    giz = __ldg(g + H);
+    gin = __ldg(g + 2 * H);
+  }
+  const float r = sigmoidf_(gir + ghr);
+  const float z = sigmoidf_(giz + ghz);
+  const float c = tanhf(gin + r * ghn);
+  const float hn = (1.f - z) * c + z * hp;
+  const long long e = (long long)b * H + i;
+  a.h[e] = hn;
+  a.h_bf16[e] = f32_to_bf16_rne(hn);
+}
+
 // out[b, o] = act(sum_s part[s, b, o] (+ residual[b, o])); partials and the
 // residual are dense [.., B, O]; outputs have their own row pitch.
 __global__ void k_splitk_finish(const float* __restrict__ part, int S, int B, int O,
@@ -242,6 +311,12 @@ inline int grid_for(long long total, int threads) {
 cudaError_t launch_gru_gates(const float* part, int S0, int S1, int B, int H, float* h, uint16_t* h_bf16,
                              cudaStream_t s) {
   return launch_pdl(k_gru_gates, dim3(grid_for((long long)B * H, 256)), dim3(256), 0, s, part, S0, S1, B, H, h, h_bf16);
+}
+
+cudaError_t launch_gru_gates_table(const GatesTableArgs& a, cudaStream_t s) {
+  const int chunks = (a.H + kGatesThreads - 1) / kGatesThreads;   // one hidden unit per thread
+  if (chunks > 65535) return cudaErrorInvalidValue;
+  return launch_pdl(k_gru_gates_table, dim3(a.B, chunks), dim3(kGatesThreads), 0, s, a);
 }
 
 cudaError_t launch_splitk_finish(const float* part, int S, int B, int O, const float* residual, int act,

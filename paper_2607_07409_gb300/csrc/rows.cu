@@ -28,24 +28,10 @@ __device__ __forceinline__ void load8(const float* p, float (&x)[8]) {
 __device__ __forceinline__ float load1(const uint16_t* p) { return __uint_as_float((uint32_t)__ldcs(p) << 16); }
 __device__ __forceinline__ float load1(const float* p) { return __ldcs(p); }
 
-__device__ __forceinline__ RowAcc ld_rowacc_cg(const void* base, long long i) {
-  const float4 v = __ldcg(reinterpret_cast<const float4*>(base) + i);
-  RowAcc r;
-  r.m = v.x; r.s = v.y; r.second = v.z; r.idx = __float_as_int(v.w);
-  return r;
-}
 __device__ __forceinline__ void st_rowacc(void* base, long long i, const RowAcc& r) {
   reinterpret_cast<float4*>(base)[i] = make_float4(r.m, r.s, r.second, __int_as_float(r.idx));
 }
 
-__device__ __forceinline__ void write_decode(const RowAcc& r, long long out_i, int32_t* tok, float* lp, float* gap,
-                                             int* status) {
-  const bool ok = rowacc_valid(r);
-  if (!ok) raise_status(status, DELS_STATUS_NONFINITE);
-  tok[out_i] = ok ? r.idx : -1;
-  if (lp) lp[out_i] = ok ? -logf(r.s) : NAN;
-  if (gap) gap[out_i] = ok ? (r.m - r.second) : NAN;
-}
 
 // Per-thread running state of one row.
 struct RowState {

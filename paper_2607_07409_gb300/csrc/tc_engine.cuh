@@ -118,10 +118,17 @@ __device__ __forceinline__ void item_range(const TcGemmArgs& a, int cta, int nct
   }
 }
 
-__device__ __forceinline__ float act_apply(int act, float x) {
-  if (act == ACT_SILU) return x / (1.f + __expf(-x));
-  if (act == ACT_GELU) return 0.5f * x * (1.f + erff(x * 0.70710678118654752f));
-  return x;
+// Activation of a 32-value accumulator chunk. The branch sits outside the
+// unrolled loops: inside them the compiler predicates every activation's
+// arithmetic for every value, which costs microseconds per tile.
+__device__ __forceinline__ void act_apply32(int act, float (&x)[32]) {
+  if (act == ACT_SILU) {
+#pragma unroll
+    for (int i = 0; i < 32; ++i) x[i] = __fdividef(x[i], 1.f + __expf(-x[i]));
+  } else if (act == ACT_GELU) {
+#pragma unroll
+    for (int i = 0; i < 32; ++i) x[i] = 0.5f * x[i] * (1.f + erff(x[i] * 0.70710678118654752f));
+  }
 }
 
 // ------------------------------------------------------------------ producer
@@ -431,8 +438,7 @@ __device__ __forceinline__ bool epi_run(const Ctx& c, const Phase& p, EpiState& 
         tmem_ld_wait();
         const int cbase = it.o0 + cc * 32;
         if (b < a.B) {
-#pragma unroll
-          for (int i = 0; i < 32; ++i) acc[i] = act_apply(a.act, acc[i]);
+          if (a.act != ACT_NONE) act_apply32(a.act, acc);
           if (a.out_f32 && a.out_bmajor) {
             // column-by-column: the warp's 32 rows are 32 consecutive floats
             float* dst = a.out_f32 + (long long)it.split * a.out_split_stride + (long long)cbase * a.ldb + b;

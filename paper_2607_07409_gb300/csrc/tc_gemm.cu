@@ -62,10 +62,17 @@ __host__ __device__ inline Smem smem_layout(const TcGemmArgs& a) {
 __global__ void __launch_bounds__(kThreads, 1)
     k_tc_gemm(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ CUtensorMap mB0,
               const __grid_constant__ CUtensorMap mA1, const __grid_constant__ CUtensorMap mB1,
-              const __grid_constant__ CUtensorMap mL, const TcGemmArgs a, uint64_t budget_ns) {
+              const __grid_constant__ CUtensorMap mL, const __grid_constant__ TcGemmArgs a0,
+              const __grid_constant__ CUtensorMap gA, const __grid_constant__ CUtensorMap gB,
+              const __grid_constant__ TcGemmArgs a1, int grid0, uint64_t budget_ns) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   uint8_t* smem = smem_raw + (((raw + 1023u) & ~1023u) - raw);
+  // CTAs past grid0 run the second GEMM of a grouped launch
+  const bool second = (int)blockIdx.x >= grid0;
+  const TcGemmArgs& a = second ? a1 : a0;
+  const int cta = second ? (int)blockIdx.x - grid0 : (int)blockIdx.x;
+  const int ncta = second ? (int)gridDim.x - grid0 : grid0;
   const Smem lay = smem_layout(a);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const bool comb = a.epi == EPI_COMBINE;
@@ -112,10 +119,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     *c.abort_flag = 0;
     fence_mbarrier_init();
   }
+  const CUtensorMap* pA0 = second ? &gA : &mA0;
+  const CUtensorMap* pB0 = second ? &gB : &mB0;
   if (warp == 0 && lane == 0) {
-    tma_prefetch_desc(&mA0);
-    tma_prefetch_desc(&mB0);
-    if (a.seg_splits[1] > 0) {
+    tma_prefetch_desc(pA0);
+    tma_prefetch_desc(pB0);
+    if (!second && a.seg_splits[1] > 0) {
       tma_prefetch_desc(&mA1);
       tma_prefetch_desc(&mB1);
     }
@@ -132,13 +141,13 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   Phase p;
   p.a = &a;
-  p.mA0 = &mA0;
-  p.mB0 = &mB0;
-  p.mA1 = &mA1;
-  p.mB1 = &mB1;
+  p.mA0 = pA0;
+  p.mB0 = pB0;
+  p.mA1 = second ? &gA : &mA1;
+  p.mB1 = second ? &gB : &mB1;
   p.mL = &mL;
   p.j = a.j;
-  item_range(a, blockIdx.x, gridDim.x, p.first, p.count, p.stride);
+  item_range(a, cta, ncta, p.first, p.count, p.stride);
 
   if (warp == 0) {
     if (lane == 0) {
@@ -185,7 +194,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (comb) epi_stage_prior(c, p, threadIdx.x - 64);   // an input: no wait needed
     pdl_wait();
     EpiState st;
-    epi_run(c, p, st, warp, lane, blockIdx.x);
+    epi_run(c, p, st, warp, lane, cta);
   }
 
   tc_fence_before();
@@ -195,6 +204,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     tmem_dealloc(c.tmem_base, tmem_cols);
   }
+
 }
 
 }  // namespace
@@ -203,8 +213,10 @@ size_t tc_gemm_smem_bytes(const TcGemmArgs& a) { return smem_layout(a).total; }
 
 cudaError_t launch_tc_gemm(const TcGemmArgs& a, const CUtensorMap* mA0, const CUtensorMap* mB0,
                            const CUtensorMap* mA1, const CUtensorMap* mB1, const CUtensorMap* mL, int grid,
-                           size_t smem_bytes, cudaStream_t s) {
-  if (grid <= 0) return cudaSuccess;
+                           size_t smem_bytes, cudaStream_t s, const TcGemmGroup* second) {
+  const bool two = second && second->a && second->grid > 0;
+  if (grid <= 0 && !two) return cudaSuccess;
+  if (two) smem_bytes = std::max(smem_bytes, tc_gemm_smem_bytes(*second->a));
   // The opt-in shared-memory limit is a per-device function attribute; raise
   // it once per device to the largest request seen.
   static int configured_bytes[64] = {0};
@@ -218,7 +230,12 @@ cudaError_t launch_tc_gemm(const TcGemmArgs& a, const CUtensorMap* mA0, const CU
     configured_bytes[dev] = (int)smem_bytes;
   }
   const uint64_t budget = a.debug_skip_producer ? 100000000ull : kWaitBudgetNs;
-  return launch_pdl(k_tc_gemm, dim3(grid), dim3(kThreads), smem_bytes, s, *mA0, *mB0, *mA1, *mB1, *mL, a, budget);
+  const int g0 = std::max(grid, 0);
+  if (two)
+    return launch_pdl(k_tc_gemm, dim3(g0 + second->grid), dim3(kThreads), smem_bytes, s, *mA0, *mB0, *mA1, *mB1,
+                      *mL, a, *second->mA, *second->mB, *second->a, g0, budget);
+  return launch_pdl(k_tc_gemm, dim3(g0), dim3(kThreads), smem_bytes, s, *mA0, *mB0, *mA1, *mB1, *mL, a, *mA0, *mB0,
+                    a, g0, budget);
 }
 
 }  // namespace dels

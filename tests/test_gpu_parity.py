@@ -229,6 +229,48 @@ def test_draft_persistent_kernel_matches_oracle(name, stress, monkeypatch):
     print(name, stress, info)
 
 
+def _with_table(w, d):
+    W = {k[5:]: v for k, v in d.items() if k.startswith("head.")}
+    d = dict(d)
+    d["head.input_table"] = dels.gru_input_table(w.head, W, w.V)
+    return d
+
+
+@pytest.mark.parametrize("V", [3000, 4096])
+def test_gru_input_table_is_the_input_product(V):
+    w = synth.with_sizes(synth.stress(synth.WORKLOADS["qwen3_8b_batched"]), B=2, n=2, V=V,
+                         head_d_model=256, head_d_hidden=128, head_d_rank=64)
+    d = synth.make_inputs(w, device=DEV, target=False)
+    G = _with_table(w, d)["head.input_table"]
+    torch.cuda.synchronize()
+    E = d["head.emb"].double().cpu()
+    Wih = d["head.w_ih"].double().cpu()
+    ref = E @ Wih.T
+    got = G.double().cpu()
+    assert got.shape == ref.shape
+    # bf16 x bf16 products are exact in f32; only the f32 summation of d_model
+    # terms rounds: |error| <= d_model * 2^-23 * sum |E_k W_k| (standard bound)
+    bound = w.head.d_model * 2.0 ** -23 * (E.abs() @ Wih.abs().T) + 1e-30
+    assert torch.all((got - ref).abs() <= bound), float(((got - ref).abs() / bound).max())
+
+
+@pytest.mark.parametrize("stress", [False, True])
+@pytest.mark.parametrize("name", ["gru", "gru_b64"])
+def test_draft_with_input_table_matches_oracle(name, stress):
+    w = SMALL[name]
+    if stress:
+        w = synth.stress(w)
+    d = _with_table(w, synth.make_inputs(w, device=DEV, target=False))
+    tok, lp, gap, W, prior = _draft(w, d)
+    W = {k: v for k, v in W.items() if k != "input_table"}
+    info = check_draft(tok, lp, gap, _oracle_head(w, W), d["long"].cpu(), prior, w.alpha, w.beta, LP_TOL_BF16)
+    # the fused merge's ticket resets itself: a second call gives the same block
+    tok2, lp2, gap2, _, _ = _draft(w, d)
+    np.testing.assert_array_equal(tok2, tok)
+    np.testing.assert_array_equal(lp2, lp)
+    print(name, stress, info)
+
+
 def test_draft_zero_weight_is_dflash_argmax():
     w = synth.with_sizes(synth.stress(synth.WORKLOADS["qwen3_8b_batched"]), B=8, n=5, V=2048, weight=0.0,
                          head_d_model=128, head_d_hidden=64, head_d_rank=64)
