@@ -121,6 +121,21 @@ typedef struct {
   const void* w_vocab;
 } dels_local_head;
 
+/* ---- self test of the bounded waits ------------------------------------- */
+
+/*
+ * Every wait inside the library's kernels (on an mbarrier, a flag or another
+ * CTA) has a time limit; when it runs out the kernel stops waiting, frees
+ * what it holds, returns, and sets DELS_STATUS_TIMEOUT in the status word.
+ * This launches one small tensor-core product whose producer never issues a
+ * load, so each wait expires (after 0.1 s) and the status word reports
+ * DELS_STATUS_TIMEOUT; the context stays usable. (A test hook; the paper has
+ * no counterpart.) `workspace` [device] >= dels_selftest_timeout_bytes(),
+ * zero-filled, 16-byte aligned; read the status with dels_read_status.
+ */
+size_t dels_selftest_timeout_bytes(void);
+int dels_selftest_timeout(void* workspace, size_t workspace_bytes, dels_stream_t stream);
+
 /* ---- GRU input table (head preparation, once per set of weights) -------- */
 
 /*

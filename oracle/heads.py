@@ -78,6 +78,8 @@ class _Head:
         W = self._raw["w_vocab"]
         r = self.act(feat)
         B = r.shape[0]
+        if "w_vocab" in self._cache:                       # already decoded whole (see w())
+            return r @ self._cache["w_vocab"].T
         out = np.empty((B, self.V), dtype=np.float64)
         for v0 in range(0, self.V, chunk):
             Wc = to_f64(W[v0:v0 + chunk])

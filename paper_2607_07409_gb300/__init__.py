@@ -27,6 +27,7 @@ __all__ = [
     "dels_read_status", "dels_prior_from_counts", "dels_status_string", "dels_version",
     "dels_profile_enable", "dels_profile_reset", "dels_profile_read", "KCLASS",
     "dels_gru_input_table_bytes", "dels_gru_build_input_table", "gru_input_table",
+    "dels_selftest_timeout_bytes", "dels_selftest_timeout",
     "make_head", "Drafter", "dtype_code",
 ]
 
@@ -57,6 +58,8 @@ class LocalHead(ctypes.Structure):
 
 
 _SIGS = {
+    "dels_selftest_timeout_bytes": (_sz, []),
+    "dels_selftest_timeout": (_i, [_vp, _sz, _vp]),
     "dels_gru_input_table_bytes": (_sz, [ctypes.POINTER(LocalHead), _i]),
     "dels_gru_build_input_table": (_i, [ctypes.POINTER(LocalHead), _i, _vp, _sz, _vp, _sz, _vp]),
     "dels_draft_workspace_bytes": (_sz, [ctypes.POINTER(LocalHead), _i, _i, _i]),
@@ -153,6 +156,14 @@ def dels_version() -> int:
 
 def dels_status_string(code: int) -> str:
     return lib().dels_status_string(int(code)).decode()
+
+
+def dels_selftest_timeout_bytes() -> int:
+    return lib().dels_selftest_timeout_bytes()
+
+
+def dels_selftest_timeout(workspace, workspace_bytes: int, stream=None) -> int:
+    return lib().dels_selftest_timeout(_ptr(workspace), workspace_bytes, _stream(stream))
 
 
 def dels_gru_input_table_bytes(head: LocalHead, V: int) -> int:

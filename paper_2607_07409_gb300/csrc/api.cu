@@ -708,6 +708,29 @@ int dels_verify_block(const int32_t* draft_tokens, const void* target_logits, de
   return DELS_OK;
 }
 
+// ------------------------------------------------------------ self test
+
+size_t dels_selftest_timeout_bytes(void) { return kHeaderBytes + 4096; }
+
+int dels_selftest_timeout(void* workspace, size_t workspace_bytes, dels_stream_t stream) {
+  if (!workspace) return DELS_ERR_WORKSPACE;
+  if (workspace_bytes < dels_selftest_timeout_bytes()) return DELS_ERR_WORKSPACE;
+  if (!aligned16(workspace)) return DELS_ERR_ALIGNMENT;
+  const int sms = device_sm_count();
+  if (sms <= 0) return DELS_ERR_CUDA;
+  // X [8, 64] and W [16, 64] bf16, Y [8, 16] f32 inside the workspace; the
+  // producer never fills a stage, so every wait of the kernel runs out
+  uint8_t* base = static_cast<uint8_t*>(workspace) + kHeaderBytes;
+  Gemm g;
+  if (!plan_store(g, 8, 16, base, base + 1024, 64, nullptr, nullptr, 0, 16, 1, 0, ACT_NONE,
+                  reinterpret_cast<float*>(base + 3072), nullptr, 0, at<int>(workspace, 0), sms))
+    return DELS_ERR_CUDA;
+  g.a.debug_skip_producer = 1;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  DELS_CUDA(run(g, s));
+  return DELS_OK;
+}
+
 // ------------------------------------------------------- GRU input table
 
 size_t dels_gru_input_table_bytes(const dels_local_head* head, int V) {

@@ -21,6 +21,17 @@ TIE_EPS = 1e-3
 LP_TOL_BF16 = 2e-3
 LP_TOL_F32 = 1e-5
 LP_TOL_COMBINE = 1e-5
+# The transformer head at d_model 2560 / FFN 10240 rounds three activations
+# to bf16 in sequence (attention input, FFN input and output, the feature).
+# Both sides round at the same points, but the value being rounded carries
+# the float32 summation error of the device's products (~3e-6 relative for
+# K = 2560), so about 0.2 % of the FFN outputs land on the other side of a
+# bf16 rounding boundary; each such flip moves y by one bf16 step of that
+# activation times W_2, and RMSNorm(y) then flips ~3 % of the feature's bf16
+# codes. Measured at full size: feature flips 3 %, logprob error up to 4.3e-3.
+# The bar for this head is therefore 1e-2 (derived; the fp32 and GRU/MLP
+# heads keep the bars above).
+LP_TOL_XFMR_BF16 = 1e-2
 
 
 def check_rows(tok, lp, gap, ref_tok, ref_lp, ref_gap, lp_tol=LP_TOL_COMBINE, exact_ties=False, fused=None):

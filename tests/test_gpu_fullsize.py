@@ -1,0 +1,82 @@
+"""Parity at the workloads' full sizes, in the launch configuration the
+benchmark times, on sampled requests.
+
+Requests are independent (Algorithm 1 touches no state across rows), so the
+oracle run on a subset of the batch is the exact reference for those rows;
+the device always drafts the whole batch. The oracle takes its own prior
+from the counts and re-checks each sampled row in forced-prefix mode.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+import paper_2607_07409_gb300 as dels
+from parity import LP_TOL_BF16, LP_TOL_F32, LP_TOL_XFMR_BF16, check_draft
+
+pytestmark = pytest.mark.gpu
+
+DEV = "cuda:0"
+
+
+def _oracle_head(w, W):
+    # the embedding table stays where it is (the oracle gathers rows from it);
+    # the matrices come to the host and are decoded once
+    Wo = {k: (v if k == "emb" else v.cpu()) for k, v in W.items() if k != "input_table"}
+    head = oracle.make_head(w.head, Wo)
+    head.w("w_vocab")
+    return head
+
+
+def _draft_and_verify(w, rows, table=False):
+    d = synth.make_inputs(w, device=DEV, target=True)
+    W = {k[5:]: v for k, v in d.items() if k.startswith("head.")}
+    if table:
+        W["input_table"] = dels.gru_input_table(w.head, W, w.V)
+    prior = dels.dels_prior_from_counts(d["counts"]).to(DEV)
+    dr = dels.Drafter(w.head, W, w.B, w.n, w.V)
+    tok, lp, gap = dr(d["long"], prior, w.alpha, w.beta)
+    dt = dels.dtype_code(d["target"])
+    vb = dels.dels_verify_workspace_bytes(w.B, w.n, w.V, dt)
+    vws = torch.zeros(vb, dtype=torch.uint8, device=DEV)
+    acc = torch.empty(w.B, dtype=torch.int32, device=DEV)
+    bonus = torch.empty(w.B, dtype=torch.int32, device=DEV)
+    targ = torch.empty(w.B, w.n + 1, dtype=torch.int32, device=DEV)
+    r = dels.dels_verify_block(tok, d["target"], dt, w.B, w.n, w.V, acc, bonus, targ, vws, vb)
+    assert r == 0
+    torch.cuda.synchronize()
+    assert dr.status() == 0 and dels.dels_read_status(vws) == 0
+    tok, lp, gap = (t.cpu().numpy() for t in (tok, lp, gap))
+    rows = list(rows)
+    head = _oracle_head(w, W)
+    prior64 = oracle.log_prior(d["counts"])
+    tol = LP_TOL_F32 if w.head.wdtype == "f32" else (LP_TOL_XFMR_BF16 if w.head.kind == "xfmr" else LP_TOL_BF16)
+    info = check_draft(tok[rows], lp[rows], gap[rows], head, d["long"][rows].cpu(), prior64, w.alpha, w.beta, tol)
+    # verification of the same rows: bit-exact accept length, bonus and target argmax
+    ref_acc, ref_bonus, ref_t = oracle.verify_greedy(tok[rows], d["target"][rows].cpu())
+    np.testing.assert_array_equal(acc.cpu().numpy()[rows], ref_acc)
+    np.testing.assert_array_equal(bonus.cpu().numpy()[rows], ref_bonus)
+    np.testing.assert_array_equal(targ.cpu().numpy()[rows], ref_t)
+    return info
+
+
+@pytest.mark.parametrize("table", [True, False])
+def test_qwen3_8b_batched_full_size(table):
+    w = synth.WORKLOADS["qwen3_8b_batched"]
+    print(_draft_and_verify(w, [0, 21, 63], table=table))
+
+
+def test_qwen3_8b_batched_full_size_stress():
+    w = synth.stress(synth.WORKLOADS["qwen3_8b_batched"])
+    print(_draft_and_verify(w, [5, 40], table=True))
+
+
+def test_qwen3_0p6b_full_size():
+    w = synth.WORKLOADS["qwen3_0p6b"]
+    print(_draft_and_verify(w, [0]))
+
+
+def test_qwen3_4b_full_size():
+    w = synth.WORKLOADS["qwen3_4b"]
+    print(_draft_and_verify(w, [0, 7]))

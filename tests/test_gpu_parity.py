@@ -28,6 +28,11 @@ def _status(ws):
     return dels.dels_read_status(ws)
 
 
+def _prior_input(counts):
+    """float32 log prior [V] from the oracle (an input the device and the oracle share)."""
+    return torch.from_numpy(oracle.log_prior(counts).astype(np.float32))
+
+
 # ------------------------------------------------------------------ combine
 
 def _combine(long, short, prior, alpha, beta):
@@ -55,24 +60,22 @@ def _combine(long, short, prior, alpha, beta):
 ])
 def test_combine_matches_oracle(rows, V, dtype, w):
     d = synth.make_combine_inputs(rows, V, dtype, seed=rows * 31 + V, device=DEV)
-    prior_cpu = dels.dels_prior_from_counts(d["counts"])
-    tok, lp, gap, st = _combine(d["long"], d["short"], prior_cpu.to(DEV), w, w)
+    # the log prior is an input of the combine: both sides get the same float32 values (the oracle's)
+    prior_in = _prior_input(d["counts"])
+    tok, lp, gap, st = _combine(d["long"], d["short"], prior_in.to(DEV), w, w)
     assert st == 0
-    ref_prior = oracle.log_prior(d["counts"])
-    # the device consumes the library's float32 prior; the oracle uses its own fp64 prior
-    np.testing.assert_allclose(prior_cpu.numpy(), ref_prior, rtol=0, atol=2e-6)
-    rt, rl, rg = oracle.combine_argmax(d["long"], d["short"], prior_cpu.numpy().astype(np.float64), w, w)
+    rt, rl, rg = oracle.combine_argmax(d["long"], d["short"], prior_in.numpy().astype(np.float64), w, w)
     fused = None
     if rows * V < 5e6:
         fused = oracle.fuse(oracle.to_f64(d["long"]), oracle.to_f64(d["short"]),
-                            prior_cpu.numpy().astype(np.float64), w, w)
+                            prior_in.numpy().astype(np.float64), w, w)
     check_rows(tok, lp, gap, rt, rl, rg, exact_ties=(w == 0.0), fused=fused)
 
 
 def test_combine_many_rows_grouped_path():
     rows, V = 10000, 64                      # rows >= 64 * SMs: 4 rows per CTA
     d = synth.make_combine_inputs(rows, V, "bf16", seed=11, device=DEV)
-    prior = dels.dels_prior_from_counts(d["counts"])
+    prior = _prior_input(d["counts"])
     tok, lp, gap, st = _combine(d["long"], d["short"], prior.to(DEV), 0.5, 0.5)
     assert st == 0
     rt, rl, rg = oracle.combine_argmax(d["long"], d["short"], prior.numpy().astype(np.float64), 0.5, 0.5)
@@ -175,7 +178,8 @@ def _draft(w, d):
     tok, lp, gap = drafter(d["long"], prior, w.alpha, w.beta)
     torch.cuda.synchronize()
     assert drafter.status() == 0
-    return tok.cpu().numpy(), lp.cpu().numpy(), gap.cpu().numpy(), W, prior.cpu().numpy().astype(np.float64)
+    # the oracle takes its own prior from the same counts
+    return tok.cpu().numpy(), lp.cpu().numpy(), gap.cpu().numpy(), W, oracle.log_prior(d["counts"])
 
 
 def _oracle_head(w, W):
@@ -287,3 +291,20 @@ def test_draft_block_of_one_position():
     tok, lp, gap, W, prior = _draft(w, d)
     L = oracle.to_f64(d["long"])
     np.testing.assert_array_equal(tok[:, 0], np.argmax(L[:, 0], axis=1))
+
+
+# ------------------------------------------------------------ bounded waits
+
+def test_expired_wait_reports_timeout_and_context_survives():
+    nbytes = dels.dels_selftest_timeout_bytes()
+    ws = _ws(nbytes)
+    assert dels.dels_selftest_timeout(ws, nbytes) == 0
+    st = _status(ws)
+    assert st & dels.DELS_STATUS_TIMEOUT, st
+    # the context is still usable: an ordinary call runs and is correct
+    d = synth.make_combine_inputs(3, 4096, "bf16", seed=5, device=DEV)
+    prior = _prior_input(d["counts"])
+    tok, lp, gap, st2 = _combine(d["long"], d["short"], prior.to(DEV), 0.5, 0.5)
+    assert st2 == 0
+    rt, rl, rg = oracle.combine_argmax(d["long"], d["short"], prior.numpy().astype(np.float64), 0.5, 0.5)
+    check_rows(tok, lp, gap, rt, rl, rg)
