@@ -49,6 +49,9 @@ def parse_args():
     p.add_argument("--e2e-steps", type=int, default=20)
     p.add_argument("--cpu-rows", type=int, default=4, help="requests in the CPU-oracle baseline sample")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--sweep", action="store_true",
+                   help="instead of the drafting step: HBM GB/s of dels_combine_argmax and dels_verify_block over "
+                        "the combine/verify sweep grid (one JSON line per point)")
     p.add_argument("--no-input-table", action="store_true",
                    help="recompute the GRU input product W_ih E[x] at every position instead of reading the "
                         "precomputed table G = E W_ih^T")
@@ -82,7 +85,7 @@ def measured_peaks():
 
 def kernel_source_digest():
     h = hashlib.sha256()
-    for name in ("tc_gemm.cu", "dels_device.cuh"):
+    for name in ("tc_gemm.cu", "tc_engine.cuh", "dels_device.cuh"):
         with open(os.path.join(ROOT, "paper_2607_07409_gb300", "csrc", name), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]
@@ -445,10 +448,99 @@ def run_ours(args):
     return 0
 
 
+def run_sweep(args):
+    """dels_combine_argmax over rows = B*n independent rows [rows, V] (long and
+    short logits plus the prior) and dels_verify_block over [B, n+1, V] target
+    logits, for every (V, dtype, B, n) of the sweep grid. The combination
+    weight does not change the bytes a call moves, so the timing runs at
+    w = 0.5 (parity over the weights is in the tests). Each launch is timed
+    alone with CUDA events after an L2 flush (a 256 MB write)."""
+    import torch
+    import synth
+    import paper_2607_07409_gb300 as dels
+    from paper_2607_07409_gb300 import replicas
+    world, rank, local = dist_setup(args.gpus)
+    dev = torch.device(f"cuda:{local}")
+    torch.cuda.set_device(dev)
+    peak, peak_kind = measured_peaks()
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    reps = max(3, min(args.steps, 10))
+    seen = set()
+
+    def timed(fn):
+        ts = []
+        for i in range(reps + 2):
+            flush.fill_(i & 0xFF)
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            fn()
+            b.record()
+            b.synchronize()
+            if i >= 2:
+                ts.append(a.elapsed_time(b) * 1e-3)
+        return statistics.median(ts)
+
+    for pt in synth.sweep_points():
+        key = (pt["V"], pt["dtype"], pt["B"], pt["n"])
+        if key in seen:
+            continue
+        seen.add(key)
+        V, dt, B, n = key
+        es = 4 if dt == "f32" else 2
+        rows = B * n
+        d = synth.make_combine_inputs(rows, V, dt, seed=B * 131 + n * 7 + V % 97, device=dev)
+        prior = dels.dels_prior_from_counts(d["counts"]).to(dev)
+        code = dels.dtype_code(d["long"])
+        cb = dels.dels_combine_workspace_bytes(rows, V, code)
+        cws = torch.zeros(cb, dtype=torch.uint8, device=dev)
+        tok = torch.empty(rows, dtype=torch.int32, device=dev)
+        lp = torch.empty(rows, dtype=torch.float32, device=dev)
+        gap = torch.empty(rows, dtype=torch.float32, device=dev)
+
+        def comb():
+            r = dels.dels_combine_argmax(d["long"], d["short"], code, prior, 0.5, 0.5, rows, V, tok, lp, gap, cws, cb)
+            if r != 0:
+                raise dels.DelsError(r, "dels_combine_argmax")
+
+        t_c = timed(comb)
+        c_bytes = 2 * rows * V * es + 4 * V + 12 * rows
+        del d
+        target = torch.empty(B, n + 1, V, dtype=torch.float32 if dt == "f32" else torch.bfloat16, device=dev)
+        target.normal_(0.0, 3.0, generator=torch.Generator(device=dev).manual_seed(B * 17 + n))
+        draft = torch.randint(0, V, (B, n), dtype=torch.int32, device=dev)
+        vb = dels.dels_verify_workspace_bytes(B, n, V, code)
+        vws = torch.zeros(vb, dtype=torch.uint8, device=dev)
+        acc = torch.empty(B, dtype=torch.int32, device=dev)
+        bonus = torch.empty(B, dtype=torch.int32, device=dev)
+
+        def ver():
+            r = dels.dels_verify_block(draft, target, code, B, n, V, acc, bonus, None, vws, vb)
+            if r != 0:
+                raise dels.DelsError(r, "dels_verify_block")
+
+        t_v = timed(ver)
+        v_bytes = B * (n + 1) * V * es
+        del target
+        if rank == 0:
+            print(json.dumps({"sweep": "combine_verify", "V": V, "dtype": dt, "B": B, "n": n,
+                              "combine": {"bytes": c_bytes, "us": round(t_c * 1e6, 2),
+                                          "gbs": round(c_bytes / t_c / 1e9, 1),
+                                          "frac": round(c_bytes / t_c / 1e9 / peak, 4)},
+                              "verify": {"bytes": v_bytes, "us": round(t_v * 1e6, 2),
+                                         "gbs": round(v_bytes / t_v / 1e9, 1),
+                                         "frac": round(v_bytes / t_v / 1e9 / peak, 4)},
+                              "peak_gbs": peak, "peak_source": peak_kind, "l2": "flushed before each launch"}),
+                  flush=True)
+    replicas.barrier()
+    return 0
+
+
 def main():
     args = parse_args()
     if args.impl == "reference":
         return run_reference(args)
+    if args.sweep:
+        return run_sweep(args)
     return run_ours(args)
 
 
