@@ -292,6 +292,7 @@ bool persistent_enabled() {
 // Input-table GRU path: output tile widths of the rank product (full K per
 // tile, SiLU epilogue) and of the recurrent product (split over K).
 constexpr int kRankTile = 32;
+constexpr int kRankSplits = 4;     // K splits of the rank product, reduced inside a 4-CTA cluster
 constexpr int kHhTile = 64;
 
 struct Carve {
@@ -344,7 +345,7 @@ DraftLayout draft_layout(const dels_local_head* hd, int B, int n, int V) {
       if (bf) {
         L.gru_s0 = std::max(1, std::min((D + 63) / 64, sms / std::max(1, (3 * H + 127) / 128) - 1));
         L.gru_s1 = 1;
-        L.rank_grid = (R + kRankTile - 1) / kRankTile;
+        L.rank_grid = (R + kRankTile - 1) / kRankTile * kRankSplits;
         L.hh_splits = splits_for(3 * H, kHhTile, H, std::max(1, sms - L.rank_grid));
       } else {
         L.gru_s0 = 1;
@@ -889,15 +890,26 @@ int dels_draft_block(const dels_local_head* head, const void* long_logits, dels_
         r = position0_rows(long_logits, logit_dtype, B, n, V, partials, L.partial_ld, status, sms, s, &count);
         if (r != DELS_OK) return r;
         Gemm gr, gh, gv;
-        if (!plan_store(gr, B, R, hb, head->w[2], H, nullptr, nullptr, 0, kRankTile, 1, 0, ACT_SILU, nullptr,
-                        static_cast<uint16_t*>(rr), R, status, sms) ||
+        if (!plan_store(gr, B, R, hb, head->w[2], H, nullptr, nullptr, 0, kRankTile, kRankSplits, 0, ACT_SILU,
+                        nullptr, static_cast<uint16_t*>(rr), R, status, sms) ||
             !plan_store(gh, B, 3 * H, hb, head->w[1], H, nullptr, nullptr, 0, kHhTile, L.hh_splits, 0, ACT_NONE,
                         gpart, nullptr, 0, status, sms) ||
             !plan_combine(gv, B, V, n, rr, R, head->w_vocab, long_logits, logit_dtype, log_prior, alpha, beta,
                           partials, L.partial_ld, status, sms))
           return DELS_ERR_CUDA;
-        // both products fit one wave next to each other
-        gh.grid = std::min(gh.grid, std::max(1, sms - gr.grid));
+        // The rank product's K splits reduce inside a cluster (one cluster per
+        // output tile, no partials in HBM); its SiLU needs the whole sum.
+        const int ck = gr.a.total_splits;
+        if (ck > 1) {
+          gr.a.cluster_k = ck;
+          gr.grid = gr.a.num_o_tiles * ck;
+          const int per = (gr.a.seg_chunks[0] + ck - 1) / ck;
+          gr.a.stages = std::max(2, std::min(gr.a.stages, per));
+          gr.smem = tc_gemm_smem_bytes(gr.a);
+        }
+        // both products fit one wave next to each other; whole clusters only
+        gh.grid = std::min(gh.grid, std::max(ck, sms - gr.grid));
+        gh.grid = std::max(ck, gh.grid / ck * ck);
         const TcGemmGroup hh{&gh.a, &gh.mA0, &gh.mB0, gh.grid};
         GatesTableArgs ga{};
         ga.partials = partials;

@@ -22,20 +22,36 @@ struct RowAcc;
 // Launch with programmatic stream serialization: the kernel may begin while
 // its predecessor on the stream is still running; it waits for it with
 // griddepcontrol.wait before touching the predecessor's outputs.
+// As launch_pdl, with thread-block clusters of `cluster_x` CTAs along x
+// (1: no cluster attribute).
 template <typename... KArgs, typename... Args>
-cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
-                       Args&&... args) {
+cudaError_t launch_pdl_cluster(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                               int cluster_x, Args&&... args) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = grid;
   cfg.blockDim = block;
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
+  int na = 1;
+  if (cluster_x > 1) {
+    attr[1].id = cudaLaunchAttributeClusterDimension;
+    attr[1].val.clusterDim.x = (unsigned)cluster_x;
+    attr[1].val.clusterDim.y = 1;
+    attr[1].val.clusterDim.z = 1;
+    na = 2;
+  }
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = na;
   return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                       Args&&... args) {
+  return launch_pdl_cluster(kernel, grid, block, smem, s, 1, std::forward<Args>(args)...);
 }
 
 // ---- row reductions (combine / verify / draft position 0) -------------------
@@ -132,6 +148,11 @@ struct TcGemmArgs {
   int partial_ld;
   int* status;
   int debug_skip_producer;       // test hook: producer never fills (exercises the bounded waits)
+  // EPI_STORE, optional: the K splits of one output tile run on the CTAs of
+  // one thread-block cluster (cluster_k CTAs, split = rank in the cluster);
+  // the others send their accumulators to rank 0 through distributed shared
+  // memory, and rank 0 sums, applies the activation and stores. 1: off.
+  int cluster_k;
 };
 
 // One launch of k_tc_gemm runs one GEMM on `grid` CTAs, or two independent

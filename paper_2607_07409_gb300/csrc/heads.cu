@@ -63,6 +63,12 @@ __global__ void k_gru_gates(const float* __restrict__ part, int S0, int S1, int 
 // (non-finite logits, already flagged) takes gi = 0.
 constexpr int kGatesThreads = 256;
 
+__device__ __forceinline__ float ld_cg_f32(const float* p) {
+  float v;
+  asm volatile("ld.global.cg.f32 %0, [%1];" : "=f"(v) : "l"(p));
+  return v;
+}
+
 __global__ void __launch_bounds__(kGatesThreads) k_gru_gates_table(GatesTableArgs a) {
   if (threadIdx.x == 0) pdl_trigger();
   pdl_wait();
@@ -73,34 +79,48 @@ __global__ void __launch_bounds__(kGatesThreads) k_gru_gates_table(GatesTableArg
   // gridDim.y CTAs of kGatesThreads).
   const int i = blockIdx.y * kGatesThreads + threadIdx.x;
   const bool live = i < H;
-  // Loads that do not depend on the token go out before the merge.
-  float ghr = 0.f, ghz = 0.f, ghn = 0.f, hp = 0.f;
+  // Loads that do not depend on the token are issued first (volatile, so
+  // they stay ahead of the merge); their sums come after it.
+  constexpr int kMaxS = 8;
+  float q[kMaxS][3];
+  float hp = 0.f;
+  const int S = min(a.S, kMaxS);
   if (live) {
     const long long split_stride = (long long)a.B * 3 * H;
-    const long long base = (long long)b * 3 * H + i;
-#pragma unroll 4
-    for (int sp = 0; sp < a.S; ++sp) {
-      const float* q = a.part + sp * split_stride + base;
-      ghr += __ldcg(q);
-      ghz += __ldcg(q + H);
-      ghn += __ldcg(q + 2 * H);
+    const float* base = a.part + (long long)b * 3 * H + i;
+#pragma unroll
+    for (int sp = 0; sp < kMaxS; ++sp) {
+      if (sp < S) {
+        q[sp][0] = ld_cg_f32(base + sp * split_stride);
+        q[sp][1] = ld_cg_f32(base + sp * split_stride + H);
+        q[sp][2] = ld_cg_f32(base + sp * split_stride + 2 * H);
+      }
     }
-    if (a.S > 0) hp = a.h[(long long)b * H + i];
+    if (S > 0) hp = ld_cg_f32(a.h + (long long)b * H + i);
   }
-  __shared__ RowAcc red[kGatesThreads / 32];
+  // merge of request b's records: warp 0 alone, every record load in flight at once
   __shared__ int s_tok;
-  RowAcc x = rowacc_init();
-  for (int k = threadIdx.x; k < a.count; k += kGatesThreads)
-    x = rowacc_merge(x, ld_rowacc_cg(a.partials, (long long)b * a.partial_ld + k));
-  x = rowacc_warp_reduce(x);
-  if (lane == 0) red[warp] = x;
-  __syncthreads();
   if (warp == 0) {
-    x = lane < kGatesThreads / 32 ? red[lane] : rowacc_init();
+    RowAcc x = rowacc_init();
+    const float4* rec = reinterpret_cast<const float4*>(a.partials) + (long long)b * a.partial_ld;
+    for (int k0 = 0; k0 < a.count; k0 += 8 * 32) {
+      float4 v[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int k = k0 + u * 32 + lane;
+        v[u] = k < a.count ? __ldcg(rec + k) : make_float4(-INFINITY, 0.f, -INFINITY, __int_as_float(INT_MAX));
+      }
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        RowAcc y;
+        y.m = v[u].x; y.s = v[u].y; y.second = v[u].z; y.idx = __float_as_int(v[u].w);
+        x = rowacc_merge(x, y);
+      }
+    }
     x = rowacc_warp_reduce(x);
     if (lane == 0) {
-      if (blockIdx.y == 0) write_decode(x, (long long)b * a.n + a.jprev, a.tokens, a.out_lp, a.out_gap, a.status);
       s_tok = rowacc_valid(x) ? x.idx : -1;
+      if (blockIdx.y == 0) write_decode(x, (long long)b * a.n + a.jprev, a.tokens, a.out_lp, a.out_gap, a.status);
     }
   }
   __syncthreads();
@@ -112,6 +132,15 @@ __global__ void __launch_bounds__(kGatesThreads) k_gru_gates_table(GatesTableArg
     gir = __ldg(g);
     giz = __ldg(g + H);
     gin = __ldg(g + 2 * H);
+  }
+  float ghr = 0.f, ghz = 0.f, ghn = 0.f;
+#pragma unroll
+  for (int sp = 0; sp < kMaxS; ++sp) {
+    if (sp < S) {
+      ghr += q[sp][0];
+      ghz += q[sp][1];
+      ghn += q[sp][2];
+    }
   }
   const float r = sigmoidf_(gir + ghr);
   const float z = sigmoidf_(giz + ghz);
@@ -315,7 +344,7 @@ cudaError_t launch_gru_gates(const float* part, int S0, int S1, int B, int H, fl
 
 cudaError_t launch_gru_gates_table(const GatesTableArgs& a, cudaStream_t s) {
   const int chunks = (a.H + kGatesThreads - 1) / kGatesThreads;   // one hidden unit per thread
-  if (chunks > 65535) return cudaErrorInvalidValue;
+  if (chunks > 65535 || a.S > 8) return cudaErrorInvalidValue;
   return launch_pdl(k_gru_gates_table, dim3(a.B, chunks), dim3(kGatesThreads), 0, s, a);
 }
 

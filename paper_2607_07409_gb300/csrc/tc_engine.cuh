@@ -105,6 +105,14 @@ __device__ __forceinline__ Item get_item(const TcGemmArgs& a, int i) {
 __device__ __forceinline__ void item_range(const TcGemmArgs& a, int cta, int ncta, int& first, int& count,
                                            int& stride) {
   const int total = a.num_o_tiles * a.total_splits;
+  if (a.cluster_k > 1) {
+    // one item per CTA: the tile is the cluster's index, the K split its rank
+    const int ck = a.cluster_k;
+    first = (cta % ck) * a.num_o_tiles + cta / ck;
+    count = (cta / ck < a.num_o_tiles && cta % ck < a.total_splits) ? 1 : 0;
+    stride = ncta;
+    return;
+  }
   if (a.epi == EPI_COMBINE) {
     const long long lo = (long long)cta * total / ncta;
     const long long hi = (long long)(cta + 1) * total / ncta;

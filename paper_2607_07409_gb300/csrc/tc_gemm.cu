@@ -32,7 +32,7 @@ constexpr int kThreads = kWarps * 32;
 constexpr int kLWarp = 10;
 
 struct Smem {
-  uint32_t a_off, b_off, l_off, p_off, bar_off, red_off, total;
+  uint32_t a_off, b_off, l_off, p_off, bar_off, red_off, clus_off, total;
 };
 
 __host__ __device__ inline Smem smem_layout(const TcGemmArgs& a) {
@@ -55,8 +55,81 @@ __host__ __device__ inline Smem smem_layout(const TcGemmArgs& a) {
   off += 64 * 8;                                  // mbarriers + tmem slot + flags
   s.red_off = off;
   off += comb ? 2 * 128 * 16 : 0;
+  s.clus_off = off;                               // cluster split-K: the other ranks' accumulators
+  off += a.cluster_k > 1 ? (uint32_t)(a.cluster_k - 1) * 128u * (uint32_t)a.n_tile * 4u : 0u;
   s.total = off + 1024;                           // slack for 1024-byte alignment
   return s;
+}
+
+// Cluster split-K, ranks >= 1: wait for the accumulator, then write it into
+// rank 0's buffer slot (rank - 1) through distributed shared memory
+// ([slot][128 rows][n_tile] f32). Rank 0 only waits for its accumulator here.
+__device__ __forceinline__ void epi_cluster_send(const Ctx& c, const TcGemmArgs& a, uint32_t clus_local, int warp,
+                                                 int lane, uint32_t rank) {
+  if (!mbar_wait(&c.accf[0], 0, c.deadline, c.abort_flag)) return;
+  tc_fence_after();
+  if (rank == 0) return;
+  const int q = warp & 3, g = (warp - 2) >> 2;
+  if (q * 32 >= a.B) return;
+  const int row = q * 32 + lane;
+  const uint32_t tbase = c.tmem_base + ((uint32_t)(q * 32) << 16);
+  for (int cc = g; cc < a.n_tile / 32; cc += 2) {
+    float acc[32];
+    tmem_ld_32x32b_x32(tbase + (uint32_t)(cc * 32), acc);
+    tmem_ld_wait();
+    const uint32_t dst = cluster_map(
+        clus_local + ((((rank - 1) * 128u + (uint32_t)row) * (uint32_t)a.n_tile) + (uint32_t)cc * 32u) * 4u, 0);
+#pragma unroll
+    for (int k = 0; k < 8; ++k) st_cluster_v4(dst + k * 16, acc[4 * k], acc[4 * k + 1], acc[4 * k + 2], acc[4 * k + 3]);
+  }
+  tc_fence_before();
+}
+
+// Cluster split-K, rank 0, after the cluster barrier: own accumulator plus
+// the other ranks' slots, activation, final store.
+__device__ __forceinline__ void epi_cluster_finish(const Ctx& c, const TcGemmArgs& a, const float* clus, int o0,
+                                                   int warp, int lane) {
+  const int q = warp & 3, g = (warp - 2) >> 2;
+  if (q * 32 >= a.B) return;
+  const int b = q * 32 + lane;
+  tc_fence_after();
+  const uint32_t tbase = c.tmem_base + ((uint32_t)(q * 32) << 16);
+  for (int cc = g; cc < a.n_tile / 32; cc += 2) {
+    float acc[32];
+    tmem_ld_32x32b_x32(tbase + (uint32_t)(cc * 32), acc);
+    tmem_ld_wait();
+    for (int r = 1; r < a.cluster_k; ++r) {
+      const float4* src = reinterpret_cast<const float4*>(clus + (((r - 1) * 128 + b) * a.n_tile + cc * 32));
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        const float4 v = src[k];
+        acc[4 * k] += v.x; acc[4 * k + 1] += v.y; acc[4 * k + 2] += v.z; acc[4 * k + 3] += v.w;
+      }
+    }
+    if (b >= a.B) continue;
+    if (a.act != ACT_NONE) act_apply32(a.act, acc);
+    const int cbase = o0 + cc * 32;
+    if (a.out_f32)
+      for (int i = 0; i < 32; ++i)
+        if (cbase + i < a.O) a.out_f32[(long long)b * a.ldo + cbase + i] = acc[i];
+    if (a.out_bf16) {
+      uint16_t* dst = a.out_bf16 + (long long)b * a.ldo_bf16 + cbase;
+      if (cbase + 32 <= a.O && (a.ldo_bf16 & 7) == 0) {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          uint4 w;
+          w.x = (uint32_t)f32_to_bf16_rne(acc[k * 8 + 0]) | ((uint32_t)f32_to_bf16_rne(acc[k * 8 + 1]) << 16);
+          w.y = (uint32_t)f32_to_bf16_rne(acc[k * 8 + 2]) | ((uint32_t)f32_to_bf16_rne(acc[k * 8 + 3]) << 16);
+          w.z = (uint32_t)f32_to_bf16_rne(acc[k * 8 + 4]) | ((uint32_t)f32_to_bf16_rne(acc[k * 8 + 5]) << 16);
+          w.w = (uint32_t)f32_to_bf16_rne(acc[k * 8 + 6]) | ((uint32_t)f32_to_bf16_rne(acc[k * 8 + 7]) << 16);
+          reinterpret_cast<uint4*>(dst)[k] = w;
+        }
+      } else {
+        for (int i = 0; i < 32; ++i)
+          if (cbase + i < a.O) dst[i] = f32_to_bf16_rne(acc[i]);
+      }
+    }
+  }
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
@@ -138,6 +211,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   c.tmem_base = *tmem_slot;
+  // cluster split-K: every CTA of the cluster is running before any remote write
+  const bool clus = a.cluster_k > 1;
+  if (clus) cluster_sync_all();
 
   Phase p;
   p.a = &a;
@@ -193,12 +269,25 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else {
     if (comb) epi_stage_prior(c, p, threadIdx.x - 64);   // an input: no wait needed
     pdl_wait();
-    EpiState st;
-    epi_run(c, p, st, warp, lane, cta);
+    if (clus) {
+      if (p.count > 0) epi_cluster_send(c, a, smem_u32(smem + lay.clus_off), warp, lane, cluster_ctarank());
+    } else {
+      EpiState st;
+      epi_run(c, p, st, warp, lane, cta);
+    }
   }
 
   tc_fence_before();
   __syncthreads();
+  if (clus) {
+    // the other ranks' accumulators have landed in rank 0's buffer
+    cluster_sync_all();
+    if (warp >= 2 && warp < 2 + kEpiWarps && cluster_ctarank() == 0 && p.count > 0 && !*c.abort_flag)
+      epi_cluster_finish(c, a, reinterpret_cast<const float*>(smem + lay.clus_off), get_item(a, p.first).o0, warp,
+                         lane);
+    tc_fence_before();
+    __syncthreads();
+  }
   if (threadIdx.x == 0 && *c.abort_flag) raise_status(a.status, DELS_STATUS_TIMEOUT);
   if (warp == 1) {
     tc_fence_after();
@@ -231,11 +320,15 @@ cudaError_t launch_tc_gemm(const TcGemmArgs& a, const CUtensorMap* mA0, const CU
   }
   const uint64_t budget = a.debug_skip_producer ? 100000000ull : kWaitBudgetNs;
   const int g0 = std::max(grid, 0);
+  // clusters (split-K through distributed shared memory) cover the whole grid:
+  // both groups' grids must be whole clusters
+  const int ck = std::max(a.cluster_k, two ? second->a->cluster_k : 1);
+  if (ck > 1 && (g0 % ck != 0 || (two && second->grid % ck != 0))) return cudaErrorInvalidValue;
   if (two)
-    return launch_pdl(k_tc_gemm, dim3(g0 + second->grid), dim3(kThreads), smem_bytes, s, *mA0, *mB0, *mA1, *mB1,
-                      *mL, a, *second->mA, *second->mB, *second->a, g0, budget);
-  return launch_pdl(k_tc_gemm, dim3(g0), dim3(kThreads), smem_bytes, s, *mA0, *mB0, *mA1, *mB1, *mL, a, *mA0, *mB0,
-                    a, g0, budget);
+    return launch_pdl_cluster(k_tc_gemm, dim3(g0 + second->grid), dim3(kThreads), smem_bytes, s, ck, *mA0, *mB0,
+                              *mA1, *mB1, *mL, a, *second->mA, *second->mB, *second->a, g0, budget);
+  return launch_pdl_cluster(k_tc_gemm, dim3(g0), dim3(kThreads), smem_bytes, s, ck, *mA0, *mB0, *mA1, *mB1, *mL, a,
+                            *mA0, *mB0, a, g0, budget);
 }
 
 }  // namespace dels
