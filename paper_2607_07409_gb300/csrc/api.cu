@@ -192,7 +192,7 @@ bool plan_store(Gemm& g, int B, int O, const void* X0, const void* W0, int K0, c
   a.out_bf16 = out_bf16;
   a.ldo_bf16 = ldo_bf16;
   a.status = status;
-  a.stages = pick_stages(a, 128 * 128 + n_tile * 128, 0);
+  a.stages = pick_stages(a, 128 * 128 + n_tile * 128, (out_f32 && !out_bf16) ? kStoreTransposeBytes : 0);
   // only the B real rows are loaded; the tile's other rows feed unused outputs
   a.a_box_rows = std::min(128, (B + 7) / 8 * 8);
   a.a_copies = 1;

@@ -164,6 +164,8 @@ struct TcGemmGroup {
   const CUtensorMap* mB;
   int grid;
 };
+// Shared memory of the f32-row store transpose (8 epilogue warps x 32 x 33 floats).
+constexpr int kStoreTransposeBytes = 8 * 32 * 33 * 4;
 cudaError_t launch_tc_gemm(const TcGemmArgs& a, const CUtensorMap* mA0, const CUtensorMap* mB0,
                            const CUtensorMap* mA1, const CUtensorMap* mB1, const CUtensorMap* mL, int grid,
                            size_t smem_bytes, cudaStream_t s, const TcGemmGroup* second = nullptr);

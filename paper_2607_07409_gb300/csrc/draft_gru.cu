@@ -275,6 +275,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   c.sL = smem + lay.l_off;
   c.sP = reinterpret_cast<float*>(smem + lay.p_off);
   c.red = reinterpret_cast<RowAcc*>(smem + lay.red_off);
+  c.tr = nullptr;
   c.full = bars;
   c.empty = bars + kMaxStages;
   c.accf = bars + 2 * kMaxStages;

@@ -41,6 +41,7 @@ struct Ctx {
   uint8_t* sL;              // 2 DFlash-logit tiles
   float* sP;                // prior slice of this CTA's vocabulary range
   RowAcc* red;              // [256] epilogue merge scratch
+  float* tr;                // [8 warps][32][33] store transpose scratch (EPI_STORE), or null
   uint64_t* full;           // [S]
   uint64_t* empty;          // [S]
   uint64_t* accf;           // [2]
@@ -445,8 +446,22 @@ __device__ __forceinline__ bool epi_run(const Ctx& c, const Phase& p, EpiState& 
         tmem_ld_32x32b_x32(tbase + (uint32_t)(cc * 32), acc);
         tmem_ld_wait();
         const int cbase = it.o0 + cc * 32;
-        if (b < a.B) {
-          if (a.act != ACT_NONE) act_apply32(a.act, acc);
+        if (a.act != ACT_NONE) act_apply32(a.act, acc);
+        if (a.out_f32 && !a.out_bmajor && c.tr && !a.out_bf16) {
+          // f32 rows through a shared-memory transpose (all lanes of the
+          // warp take part): each store instruction then writes 32
+          // consecutive outputs of one row, one 128-byte line
+          float* tr = c.tr + (warp - 2) * 32 * 33;
+#pragma unroll
+          for (int i = 0; i < 32; ++i) tr[lane * 33 + i] = acc[i];
+          __syncwarp();
+          const int r0 = b - lane;
+          const int rows = min(32, a.B - r0);
+          float* dst = a.out_f32 + (long long)it.split * a.out_split_stride + cbase + lane;
+          if (cbase + lane < a.O)
+            for (int r = 0; r < rows; ++r) dst[(long long)(r0 + r) * a.ldo] = tr[r * 33 + lane];
+          __syncwarp();
+        } else if (b < a.B) {
           if (a.out_f32 && a.out_bmajor) {
             // column-by-column: the warp's 32 rows are 32 consecutive floats
             float* dst = a.out_f32 + (long long)it.split * a.out_split_stride + (long long)cbase * a.ldb + b;

@@ -32,8 +32,14 @@ constexpr int kThreads = kWarps * 32;
 constexpr int kLWarp = 10;
 
 struct Smem {
-  uint32_t a_off, b_off, l_off, p_off, bar_off, red_off, clus_off, total;
+  uint32_t a_off, b_off, l_off, p_off, bar_off, red_off, clus_off, tr_off, total;
 };
+
+// EPI_STORE with f32 rows only: the epilogue stores through a per-warp
+// 32 x 33 transpose scratch (kStoreTransposeBytes).
+__host__ __device__ inline bool store_transposes(const TcGemmArgs& a) {
+  return a.epi == EPI_STORE && a.out_f32 && !a.out_bmajor && !a.out_bf16;
+}
 
 __host__ __device__ inline Smem smem_layout(const TcGemmArgs& a) {
   Smem s{};
@@ -57,6 +63,8 @@ __host__ __device__ inline Smem smem_layout(const TcGemmArgs& a) {
   off += comb ? 2 * 128 * 16 : 0;
   s.clus_off = off;                               // cluster split-K: the other ranks' accumulators
   off += a.cluster_k > 1 ? (uint32_t)(a.cluster_k - 1) * 128u * (uint32_t)a.n_tile * 4u : 0u;
+  s.tr_off = off;
+  off += store_transposes(a) ? (uint32_t)kStoreTransposeBytes : 0u;
   s.total = off + 1024;                           // slack for 1024-byte alignment
   return s;
 }
@@ -157,6 +165,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   c.sL = smem + lay.l_off;
   c.sP = reinterpret_cast<float*>(smem + lay.p_off);
   c.red = reinterpret_cast<RowAcc*>(smem + lay.red_off);
+  c.tr = store_transposes(a) ? reinterpret_cast<float*>(smem + lay.tr_off) : nullptr;
   c.full = bars;
   c.empty = bars + kMaxStages;
   c.accf = bars + 2 * kMaxStages;
