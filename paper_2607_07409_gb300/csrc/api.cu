@@ -144,6 +144,7 @@ struct Gemm {
 };
 
 constexpr int kSmemReserve = 512 + 2 * 128 * 16 + 1024 + 256;   // barriers, reduction scratch, alignment slack
+constexpr int kMaxStagesHost = 12;                                 // the engine's ring limit
 
 // A = X [B, K] bf16 (row pitch K*2), boxes of `box_rows` rows; W = [O, K] bf16.
 bool map_x(CUtensorMap* m, const void* X, int B, int K, int box_rows) {
@@ -282,6 +283,14 @@ cudaError_t run(const Gemm& g, cudaStream_t s) {
 // default, and the faster one as measured), and one cooperative persistent
 // launch per block with grid-wide barriers between phases, selected by
 // DELS_DRAFT_PERSISTENT=1 in the environment.
+// The input-table path's products of h_j and the vocabulary projection run
+// as two launches (default, faster as measured) or as one cooperative launch
+// (DELS_DRAFT_FUSED=1 in the environment); both compute the same block.
+bool fused_products_enabled() {
+  const char* e = std::getenv("DELS_DRAFT_FUSED");
+  return e && e[0] == '1';
+}
+
 bool persistent_enabled() {
   const char* e = std::getenv("DELS_DRAFT_PERSISTENT");
   return e && e[0] == '1';
@@ -289,10 +298,12 @@ bool persistent_enabled() {
 
 // ------------------------------------------------------------ draft layout
 
-// Input-table GRU path: output tile widths of the rank product (full K per
-// tile, SiLU epilogue) and of the recurrent product (split over K).
+// Input-table GRU path: output tile widths of the rank product and of the
+// recurrent product (both split over K).
 constexpr int kRankTile = 32;
-constexpr int kRankSplits = 4;     // K splits of the rank product, reduced inside a 4-CTA cluster
+constexpr int kRankSplits = 4;     // K splits of the rank product (grouped launch)
+constexpr int kRankClusterSplits = 2;   // ... in the cooperative products+vocabulary launch (2-CTA clusters)
+constexpr size_t kRReadyOff = 128; // workspace header: rank tiles finished in the current block
 constexpr int kHhTile = 64;
 
 struct Carve {
@@ -352,6 +363,7 @@ DraftLayout draft_layout(const dels_local_head* hd, int B, int n, int V) {
         L.gru_s1 = 1;
       }
       L.gpart = c.take((size_t)std::max(L.gru_s0 + L.gru_s1, L.hh_splits) * B * 3 * H * 4);
+
       L.r = c.take((size_t)B * R * es);
       break;
     }
@@ -874,6 +886,87 @@ int dels_draft_block(const dels_local_head* head, const void* long_logits, dels_
         }
       }
       const float* G = static_cast<const float*>(head->w[3]);
+      if (bf && G && fused_products_enabled() && B <= 64) {
+        // Input-table path, fused variant (DELS_DRAFT_FUSED=1): two launches
+        // per position —
+        //   gates(j)        merge x_{j-1} from the previous position's records,
+        //                   then h_j from G[x_{j-1}], the partials of W_hh h_{j-1}
+        //                   and h_{j-1};
+        //   prod_vocab(j)   (cooperative) r_j = SiLU(W_rank h_j) and the partials
+        //                   of W_hh h_j, then l_S = W_vocab r_j fused with the
+        //                   combine -> per-CTA records.
+        // A last merge kernel decodes x_{n-1}. h_0 = 0 needs no clearing:
+        // gates(1) runs with no recurrent partials and h = 0.
+        mb.table = nullptr;
+        if (n == 1) return draft_position0(long_logits, logit_dtype, B, n, V, partials, L.partial_ld, status, mb, sms, s);
+        unsigned* r_ready = at<unsigned>(workspace, kRReadyOff);
+        DELS_CUDA(cudaMemsetAsync(r_ready, 0, sizeof(unsigned), s));
+        int count = 0;
+        r = position0_rows(long_logits, logit_dtype, B, n, V, partials, L.partial_ld, status, sms, s, &count);
+        if (r != DELS_OK) return r;
+        Gemm gr, gh, gv;
+        if (!plan_store(gr, B, R, hb, head->w[2], H, nullptr, nullptr, 0, kRankTile, kRankClusterSplits, 0,
+                        ACT_SILU, nullptr, static_cast<uint16_t*>(rr), R, status, sms) ||
+            !plan_store(gh, B, 3 * H, hb, head->w[1], H, nullptr, nullptr, 0, kHhTile, L.hh_splits, 0, ACT_NONE,
+                        gpart, nullptr, 0, status, sms) ||
+            !plan_combine(gv, B, V, n, rr, R, head->w_vocab, long_logits, logit_dtype, log_prior, alpha, beta,
+                          partials, L.partial_ld, status, sms))
+          return DELS_ERR_CUDA;
+        // the rank product's K splits form one cluster per output tile
+        gr.a.cluster_k = gr.a.total_splits;
+        ProdVocabArgs P{};
+        P.rank = gr.a;
+        P.hh = gh.a;
+        P.vocab = gv.a;
+        P.rank_ctas = gr.a.num_o_tiles * gr.a.total_splits;
+        const int hh_items = gh.a.num_o_tiles * gh.a.total_splits;
+        // one CTA per SM (cooperative); CTAs past the vocabulary tiles only
+        // take part in the products (and publish neutral records)
+        const int ck = gr.a.cluster_k;
+        const int grid = std::min(sms, std::max(gv.grid, P.rank_ctas + std::min(hh_items, sms))) / ck * ck;
+        if (P.rank_ctas >= grid || grid > L.partial_ld) return DELS_ERR_UNSUPPORTED;
+        P.r_ready = r_ready;
+        P.r = static_cast<uint16_t*>(rr);
+        P.R = R;
+        P.stages = kMaxStagesHost;
+        size_t smem = prod_vocab_smem_bytes(P);
+        while (P.stages > 2 && (int)smem > device_max_smem_optin()) {
+          --P.stages;
+          smem = prod_vocab_smem_bytes(P);
+        }
+        if ((int)smem > device_max_smem_optin()) return DELS_ERR_UNSUPPORTED;
+        const CUtensorMap maps[6] = {gr.mA0, gr.mB0, gh.mB0, gv.mA0, gv.mB0, gv.mL};
+        GatesTableArgs ga{};
+        ga.partials = partials;
+        ga.partial_ld = L.partial_ld;
+        ga.tokens = out_tokens;
+        ga.out_lp = out_logprob;
+        ga.out_gap = out_top2_gap;
+        ga.n = n;
+        ga.G = G;
+        ga.V = V;
+        ga.part = gpart;
+        ga.B = B;
+        ga.H = H;
+        ga.h = h;
+        ga.h_bf16 = hb;
+        ga.status = status;
+        for (int j = 1; j < n; ++j) {
+          ga.count = j == 1 ? count : grid;
+          ga.jprev = j - 1;
+          ga.S = j == 1 ? 0 : gh.a.total_splits;
+          { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_gru_gates_table(ga, s)); }
+          P.vocab.j = j;
+          P.hh_ctas = j + 1 < n ? std::min(hh_items, grid - P.rank_ctas) : 0;
+          P.r_target = (unsigned)(j * gr.a.num_o_tiles);
+          { PROF(DELS_KCLASS_VOCAB_COMBINE); DELS_CUDA(launch_prod_vocab(P, maps, grid, smem, s)); }
+        }
+        MergeArgs m = mb;
+        m.count = grid;
+        m.j = n - 1;
+        { PROF(DELS_KCLASS_MERGE); DELS_CUDA(launch_draft_merge(m, s)); }
+        return DELS_OK;
+      }
       if (bf && G) {
         // Input-table path (gi = G[x] with G = E W_ih^T precomputed): three
         // launches per position —

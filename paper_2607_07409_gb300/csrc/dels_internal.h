@@ -198,6 +198,22 @@ size_t draft_gru_smem_bytes(const PersistGruArgs& P);
 cudaError_t launch_draft_gru(const PersistGruArgs& P, const CUtensorMap* maps, int grid, size_t smem,
                              cudaStream_t s);
 
+// ---- products of h_j + vocabulary projection, one cooperative launch ----------
+struct ProdVocabArgs {
+  TcGemmArgs rank;               // W_rank h, K split over the CTAs of a cluster (cluster_k)
+  TcGemmArgs hh;                 // split-K partials of W_hh h (for the next gates launch)
+  TcGemmArgs vocab;              // EPI_COMBINE, activations r (resident)
+  int rank_ctas, hh_ctas;        // CTAs [0, rank_ctas) rank splits, then hh_ctas recurrent CTAs
+  int stages;                    // ring stages shared by the two phases
+  unsigned* r_ready;             // rank tiles finished since the start of the block
+  unsigned r_target;             // the vocabulary phase waits until *r_ready >= r_target
+  uint16_t* r;                   // [B, R] bf16 = SiLU(sum of the rank partials)
+  int R;
+};
+size_t prod_vocab_smem_bytes(const ProdVocabArgs& P);
+cudaError_t launch_prod_vocab(const ProdVocabArgs& P, const CUtensorMap* maps, int grid, size_t smem,
+                              cudaStream_t s);
+
 // ---- small head kernels -------------------------------------------------------
 cudaError_t launch_gru_gates(const float* part, int S0, int S1, int B, int H, float* h, uint16_t* h_bf16,
                              cudaStream_t s);

@@ -275,6 +275,23 @@ def test_draft_with_input_table_matches_oracle(name, stress):
     print(name, stress, info)
 
 
+@pytest.mark.parametrize("stress", [False, True])
+@pytest.mark.parametrize("name", ["gru", "gru_b64"])
+def test_draft_fused_products_vocab_kernel_matches_oracle(name, stress, monkeypatch):
+    # the input-table path with the products and the vocabulary projection in one cooperative launch
+    monkeypatch.setenv("DELS_DRAFT_FUSED", "1")
+    w = SMALL[name]
+    if stress:
+        w = synth.stress(w)
+    d = _with_table(w, synth.make_inputs(w, device=DEV, target=False))
+    tok, lp, gap, W, prior = _draft(w, d)
+    W = {k: v for k, v in W.items() if k != "input_table"}
+    info = check_draft(tok, lp, gap, _oracle_head(w, W), d["long"].cpu(), prior, w.alpha, w.beta, LP_TOL_BF16)
+    tok2, _, _, _, _ = _draft(w, d)
+    np.testing.assert_array_equal(tok2, tok)
+    print(name, stress, info)
+
+
 def test_draft_zero_weight_is_dflash_argmax():
     w = synth.with_sizes(synth.stress(synth.WORKLOADS["qwen3_8b_batched"]), B=8, n=5, V=2048, weight=0.0,
                          head_d_model=128, head_d_hidden=64, head_d_rank=64)
