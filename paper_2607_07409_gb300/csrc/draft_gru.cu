@@ -391,7 +391,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     } else if (is_mma) {
       mma_run(c, pg, ms);
     } else if (is_epi) {
-      epi_run(c, pg, es, warp, lane, blockIdx.x);
+      epi_run<false>(c, pg, es, warp, lane, blockIdx.x);
     }
     if (!(ok = grid_sync(P.grid_bar, bar_gen, P.abort_global, c.abort_flag, c.deadline))) break;
     if (is_epi) gates_phase(P, P.gru.seg_splits[0], P.gru.seg_splits[1], ep);
@@ -403,7 +403,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     } else if (is_mma) {
       mma_run(c, pr, ms);
     } else if (is_epi) {
-      epi_run(c, pr, es, warp, lane, blockIdx.x);
+      epi_run<false>(c, pr, es, warp, lane, blockIdx.x);
     }
     if (!(ok = grid_sync(P.grid_bar, bar_gen, P.abort_global, c.abort_flag, c.deadline))) break;
     // vocabulary projection fused with the combine
@@ -413,7 +413,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     } else if (is_mma) {
       mma_run(c, pv, ms);
     } else if (is_epi) {
-      epi_run(c, pv, es, warp, lane, blockIdx.x);
+      epi_run<true>(c, pv, es, warp, lane, blockIdx.x);
     } else if (is_lprod) {
       lprod_issue(c, pv, ls, INT_MAX, pol_stream);
       if (j + 1 < n) {

@@ -325,9 +325,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         st.tiles = 1;
       }
     } else if (has_prod) {
-      epi_run(c, pp, st, warp, lane, cta);
+      epi_run<false>(c, pp, st, warp, lane, cta);
     }
-    if (!*c.abort_flag) epi_run(c, pv, st, warp, lane, cta);
+    if (!*c.abort_flag) epi_run<true>(c, pv, st, warp, lane, cta);
   }
 
   tc_fence_before();

@@ -377,9 +377,12 @@ __device__ __forceinline__ void epi_stage_prior(const Ctx& c, const Phase& p, in
 
 // Epilogue of one phase; `warp` is the CTA warp index (2..9), `cta` the
 // index under which combine partials are published.
+// COMB: the phase is a combine phase (EPI_COMBINE); a compile-time flag so
+// that a store-only kernel carries none of the combine's registers.
+template <bool COMB>
 __device__ __forceinline__ bool epi_run(const Ctx& c, const Phase& p, EpiState& st, int warp, int lane, int cta) {
   const TcGemmArgs& a = *p.a;
-  const bool comb = a.epi == EPI_COMBINE;
+  constexpr bool comb = COMB;
   const int q = warp & 3;                      // TMEM lane quadrant
   const int g = (warp - 2) >> 2;               // column-chunk parity
   const int nchunk = a.n_tile / 32;

@@ -140,7 +140,12 @@ __device__ __forceinline__ void epi_cluster_finish(const Ctx& c, const TcGemmArg
   }
 }
 
-__global__ void __launch_bounds__(kThreads, 1)
+// COMB: combine launches (one CTA per SM, the combine epilogue's registers);
+// store launches are compiled separately with at most 2 x 352 threads' worth
+// of registers per SM, so that a store launch's CTAs can share an SM with the
+// small kernels around them.
+template <bool COMB>
+__global__ void __launch_bounds__(kThreads, COMB ? 1 : 2)
     k_tc_gemm(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ CUtensorMap mB0,
               const __grid_constant__ CUtensorMap mA1, const __grid_constant__ CUtensorMap mB1,
               const __grid_constant__ CUtensorMap mL, const __grid_constant__ TcGemmArgs a0,
@@ -156,7 +161,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int ncta = second ? (int)gridDim.x - grid0 : grid0;
   const Smem lay = smem_layout(a);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const bool comb = a.epi == EPI_COMBINE;
+  constexpr bool comb = COMB;
 
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + lay.bar_off);
   Ctx c;
@@ -282,7 +287,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (p.count > 0) epi_cluster_send(c, a, smem_u32(smem + lay.clus_off), warp, lane, cluster_ctarank());
     } else {
       EpiState st;
-      epi_run(c, p, st, warp, lane, cta);
+      epi_run<COMB>(c, p, st, warp, lane, cta);
     }
   }
 
@@ -317,15 +322,18 @@ cudaError_t launch_tc_gemm(const TcGemmArgs& a, const CUtensorMap* mA0, const CU
   if (two) smem_bytes = std::max(smem_bytes, tc_gemm_smem_bytes(*second->a));
   // The opt-in shared-memory limit is a per-device function attribute; raise
   // it once per device to the largest request seen.
-  static int configured_bytes[64] = {0};
+  const bool comb = a.epi == EPI_COMBINE;
+  if (two && (second->a->epi == EPI_COMBINE) != comb) return cudaErrorInvalidValue;
+  auto kern = comb ? k_tc_gemm<true> : k_tc_gemm<false>;
+  static int configured_bytes[2][64] = {{0}};
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
-  if ((int)smem_bytes > configured_bytes[dev]) {
-    e = cudaFuncSetAttribute(k_tc_gemm, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_bytes);
+  if ((int)smem_bytes > configured_bytes[comb][dev]) {
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_bytes);
     if (e != cudaSuccess) return e;
-    configured_bytes[dev] = (int)smem_bytes;
+    configured_bytes[comb][dev] = (int)smem_bytes;
   }
   const uint64_t budget = a.debug_skip_producer ? 100000000ull : kWaitBudgetNs;
   const int g0 = std::max(grid, 0);
@@ -334,9 +342,9 @@ cudaError_t launch_tc_gemm(const TcGemmArgs& a, const CUtensorMap* mA0, const CU
   const int ck = std::max(a.cluster_k, two ? second->a->cluster_k : 1);
   if (ck > 1 && (g0 % ck != 0 || (two && second->grid % ck != 0))) return cudaErrorInvalidValue;
   if (two)
-    return launch_pdl_cluster(k_tc_gemm, dim3(g0 + second->grid), dim3(kThreads), smem_bytes, s, ck, *mA0, *mB0,
+    return launch_pdl_cluster(kern, dim3(g0 + second->grid), dim3(kThreads), smem_bytes, s, ck, *mA0, *mB0,
                               *mA1, *mB1, *mL, a, *second->mA, *second->mB, *second->a, g0, budget);
-  return launch_pdl_cluster(k_tc_gemm, dim3(g0), dim3(kThreads), smem_bytes, s, ck, *mA0, *mB0, *mA1, *mB1, *mL, a,
+  return launch_pdl_cluster(kern, dim3(g0), dim3(kThreads), smem_bytes, s, ck, *mA0, *mB0, *mA1, *mB1, *mL, a,
                             *mA0, *mB0, a, g0, budget);
 }
 
