@@ -9,6 +9,8 @@
 // ticket, reset by that CTA), so no [rows, V] intermediate is ever written.
 #include <climits>
 
+#include <cuda_bf16.h>
+
 #include "dels_device.cuh"
 
 namespace dels {
@@ -26,6 +28,27 @@ __device__ __forceinline__ void load8(const float* p, float (&x)[8]) {
   x[0] = a.x; x[1] = a.y; x[2] = a.z; x[3] = a.w; x[4] = b.x; x[5] = b.y; x[6] = b.z; x[7] = b.w;
 }
 __device__ __forceinline__ float load1(const uint16_t* p) { return __uint_as_float((uint32_t)__ldcs(p) << 16); }
+
+// Maximum of the 8 bf16 values of a 16-byte vector, NaN ignored
+// (flagged in `nan`): packed bf16 maxima, then the two halves.
+__device__ __forceinline__ float vec_max_bf16(const uint4& w, bool& nan) {
+  const __nv_bfloat162 a = *reinterpret_cast<const __nv_bfloat162*>(&w.x);
+  const __nv_bfloat162 b = *reinterpret_cast<const __nv_bfloat162*>(&w.y);
+  const __nv_bfloat162 c = *reinterpret_cast<const __nv_bfloat162*>(&w.z);
+  const __nv_bfloat162 d = *reinterpret_cast<const __nv_bfloat162*>(&w.w);
+  const __nv_bfloat162 m = __hmax2(__hmax2(a, b), __hmax2(c, d));
+  const __nv_bfloat162 mn = __hmax2_nan(__hmax2_nan(a, b), __hmax2_nan(c, d));
+  const float lo = __low2float(m), hi = __high2float(m);
+  const float nlo = __low2float(mn), nhi = __high2float(mn);
+  nan = (nlo != nlo) | (nhi != nhi);
+  return fmaxf(lo, hi);
+}
+template <typename T>
+__device__ __forceinline__ float vec_max(const uint4& w, bool& nan);
+template <>
+__device__ __forceinline__ float vec_max<uint16_t>(const uint4& w, bool& nan) { return vec_max_bf16(w, nan); }
+__device__ __forceinline__ void load_vec(const uint16_t* p, float (&x)[8]) { load8(p, x); }
+
 __device__ __forceinline__ float load1(const float* p) { return __ldcs(p); }
 
 __device__ __forceinline__ void st_rowacc(void* base, long long i, const RowAcc& r) {
@@ -234,7 +257,44 @@ __global__ void __launch_bounds__(kRowsThreads) k_verify_rows(RowsArgs a) {
   float best = -INFINITY;
   int idx = INT_MAX;
   bool nan_seen = false;
-  if constexpr (VEC) {
+  if constexpr (VEC && sizeof(T) == 2) {
+    // bf16, vector by vector: the maximum of each 16-byte vector (packed max
+    // instructions), a strict '>' against the running best (the first vector
+    // holding the thread's maximum wins), and at the end the first element of
+    // that vector equal to the maximum: the same lowest-index argmax as an
+    // element-by-element scan, at a fraction of the instructions.
+    constexpr int U = 4;
+    constexpr int E = 16 / sizeof(T);
+    const int step = kRowsThreads * E;
+    int bvec = -1;
+    for (int cb = c0 + threadIdx.x * E; cb < c1; cb += step * U) {
+      uint4 w[U];
+#pragma unroll
+      for (int u = 0; u < U; ++u)
+        if (cb + u * step < c1) w[u] = __ldcs(reinterpret_cast<const uint4*>(L + cb + u * step));
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const int c = cb + u * step;
+        if (c < c1) {
+          bool nan_v;
+          const float mv = vec_max<T>(w[u], nan_v);
+          nan_seen |= nan_v;
+          if (mv > best) {
+            best = mv;
+            bvec = c;
+          }
+        }
+      }
+    }
+    if (bvec >= 0) {
+      float x[E];
+      load_vec(L + bvec, x);
+#pragma unroll
+      for (int i = E - 1; i >= 0; --i)
+        if (x[i] == best) idx = bvec + i;
+    }
+  } else if constexpr (VEC) {
+    // f32: element by element (measured faster than the vector form here)
     constexpr int U = 4;
     const int step = kRowsThreads * 8;
     for (int cb = c0 + threadIdx.x * 8; cb < c1; cb += step * U) {
