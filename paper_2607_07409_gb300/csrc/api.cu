@@ -603,7 +603,7 @@ size_t dels_combine_workspace_bytes(int rows, int V, dels_dtype dtype) {
   if (sms <= 0) return 0;
   const int es = dtype == DELS_F32 ? 4 : 2;
   const bool vec = (V % (16 / es)) == 0;
-  RowsPlan p = plan_rows(rows, V, 2 * es, sms, vec, 1 << 20);
+  RowsPlan p = plan_rows(rows, V, 2 * es, sms, vec, 1 << 20, true);
   const size_t groups = ((size_t)rows + p.rows_per_cta - 1) / p.rows_per_cta;
   size_t off = kHeaderBytes;
   off = round_up(off + groups * 4, 256);
@@ -628,7 +628,7 @@ int dels_combine_argmax(const void* long_logits, const void* short_logits, dels_
   const int sms = device_sm_count();
   const int es = dtype == DELS_F32 ? 4 : 2;
   const bool vec = (V % (16 / es)) == 0;
-  RowsPlan p = plan_rows(rows, V, 2 * es, sms, vec, 1 << 20);
+  RowsPlan p = plan_rows(rows, V, 2 * es, sms, vec, 1 << 20, true);
   const size_t groups = ((size_t)rows + p.rows_per_cta - 1) / p.rows_per_cta;
   RowsArgs a{};
   a.longp = long_logits;

@@ -85,7 +85,8 @@ struct RowsPlan {
   int nchunks, chunk_cols, rows_per_cta, grid;
 };
 
-RowsPlan plan_rows(int rows, int V, int bytes_per_col, int num_sms, bool vec, int max_chunks);
+RowsPlan plan_rows(int rows, int V, int bytes_per_col, int num_sms, bool vec, int max_chunks,
+                  bool multi_row = false);
 cudaError_t launch_combine_rows(const RowsArgs& a, dels_dtype dt, bool vec, bool finalize, cudaStream_t s);
 cudaError_t launch_verify_rows(const RowsArgs& a, dels_dtype dt, bool vec, cudaStream_t s);
 

@@ -65,7 +65,7 @@ extern "C" int dels_combine_argmax_noalloc(const void* long_logits, const void* 
   const int sms = device_sm_count();
   const int es = dtype == DELS_F32 ? 4 : 2;
   const bool vec = (V % (16 / es)) == 0;
-  const RowsPlan p = plan_rows(rows, V, 2 * es, sms, vec, 1 << 20);
+  const RowsPlan p = plan_rows(rows, V, 2 * es, sms, vec, 1 << 20, true);
   const size_t groups = ((size_t)rows + p.rows_per_cta - 1) / p.rows_per_cta;
   const size_t zero_bytes = kHeaderBytes + (groups * 4 + 255) / 256 * 256;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);

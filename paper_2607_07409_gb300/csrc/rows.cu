@@ -29,6 +29,21 @@ __device__ __forceinline__ void load8(const float* p, float (&x)[8]) {
 }
 __device__ __forceinline__ float load1(const uint16_t* p) { return __uint_as_float((uint32_t)__ldcs(p) << 16); }
 
+// 8 values from raw 16-byte words: one word of 8 bf16, or two words of 4 f32.
+template <typename T, int W>
+__device__ __forceinline__ void unpack8(const uint4 (&w)[W], float (&x)[8]);
+template <>
+__device__ __forceinline__ void unpack8<uint16_t, 1>(const uint4 (&w)[1], float (&x)[8]) {
+  x[0] = bf16lo(w[0].x); x[1] = bf16hi(w[0].x); x[2] = bf16lo(w[0].y); x[3] = bf16hi(w[0].y);
+  x[4] = bf16lo(w[0].z); x[5] = bf16hi(w[0].z); x[6] = bf16lo(w[0].w); x[7] = bf16hi(w[0].w);
+}
+template <>
+__device__ __forceinline__ void unpack8<float, 2>(const uint4 (&w)[2], float (&x)[8]) {
+  x[0] = __uint_as_float(w[0].x); x[1] = __uint_as_float(w[0].y); x[2] = __uint_as_float(w[0].z);
+  x[3] = __uint_as_float(w[0].w); x[4] = __uint_as_float(w[1].x); x[5] = __uint_as_float(w[1].y);
+  x[6] = __uint_as_float(w[1].z); x[7] = __uint_as_float(w[1].w);
+}
+
 // Maximum of the 8 bf16 values of a 16-byte vector, NaN ignored
 // (flagged in `nan`): packed bf16 maxima, then the two halves.
 __device__ __forceinline__ float vec_max_bf16(const uint4& w, bool& nan) {
@@ -118,27 +133,35 @@ __global__ void __launch_bounds__(kRowsThreads) k_combine_rows(RowsArgs a) {
   for (int r = 0; r < R; ++r) st[r].init();
 
   if constexpr (VEC) {
-    constexpr int U = (R == 1) ? 4 : 1;        // 128-bit loads in flight per row
+    // Raw 16-byte words stay in registers until used, so bf16 rows keep as
+    // many bytes in flight per thread as f32 rows (8 loads per row for
+    // bf16, 4 for f32, when one row per CTA).
+    constexpr int WPV = sizeof(T) == 2 ? 1 : 2;            // 16-byte words per 8 values
+    constexpr int U = (R == 1) ? (sizeof(T) == 2 ? 8 : 4) : 1;
     const int step = kRowsThreads * 8;
     for (int cb = c0 + threadIdx.x * 8; cb < c1; cb += step * U) {
-      float lv[U][R][8];
-      float sv[U][R][8];
-      float pv[U][8];
+      uint4 lw[U][R][WPV];
+      uint4 sw[U][R][WPV];
+      // f32: the prior goes out with the logits; bf16: it is read where it
+      // is used (keeps the bf16 kernel at two CTAs per SM)
+      constexpr bool kPriorEarly = sizeof(T) == 4;
+      float4 pw[kPriorEarly ? U : 1][2];
 #pragma unroll
       for (int u = 0; u < U; ++u) {
         const int c = cb + u * step;
         if (c < c1) {
-          if constexpr (PR) {
-            const float4 p0 = __ldg(reinterpret_cast<const float4*>(a.prior + c));
-            const float4 p1 = __ldg(reinterpret_cast<const float4*>(a.prior + c) + 1);
-            pv[u][0] = p0.x; pv[u][1] = p0.y; pv[u][2] = p0.z; pv[u][3] = p0.w;
-            pv[u][4] = p1.x; pv[u][5] = p1.y; pv[u][6] = p1.z; pv[u][7] = p1.w;
+          if constexpr (PR && kPriorEarly) {
+            pw[u][0] = __ldg(reinterpret_cast<const float4*>(a.prior + c));
+            pw[u][1] = __ldg(reinterpret_cast<const float4*>(a.prior + c) + 1);
           }
 #pragma unroll
           for (int r = 0; r < R; ++r) {
             if (r < nr) {
-              load8(L + (long long)r * a.ld_long + c, lv[u][r]);
-              if constexpr (SH) load8(S + (long long)r * a.ld_short + c, sv[u][r]);
+#pragma unroll
+              for (int k = 0; k < WPV; ++k) {
+                lw[u][r][k] = __ldcs(reinterpret_cast<const uint4*>(L + (long long)r * a.ld_long + c) + k);
+                if constexpr (SH) sw[u][r][k] = __ldcs(reinterpret_cast<const uint4*>(S + (long long)r * a.ld_short + c) + k);
+              }
             }
           }
         }
@@ -147,15 +170,31 @@ __global__ void __launch_bounds__(kRowsThreads) k_combine_rows(RowsArgs a) {
       for (int u = 0; u < U; ++u) {
         const int c = cb + u * step;
         if (c < c1) {
+          float pv[8];
+          if constexpr (PR) {
+            float4 p0, p1;
+            if constexpr (kPriorEarly) {
+              p0 = pw[u][0];
+              p1 = pw[u][1];
+            } else {
+              p0 = __ldg(reinterpret_cast<const float4*>(a.prior + c));
+              p1 = __ldg(reinterpret_cast<const float4*>(a.prior + c) + 1);
+            }
+            pv[0] = p0.x; pv[1] = p0.y; pv[2] = p0.z; pv[3] = p0.w;
+            pv[4] = p1.x; pv[5] = p1.y; pv[6] = p1.z; pv[7] = p1.w;
+          }
 #pragma unroll
           for (int r = 0; r < R; ++r) {
             if (r < nr) {
+              float lv[8], sv[8];
+              unpack8<T, WPV>(lw[u][r], lv);
+              if constexpr (SH) unpack8<T, WPV>(sw[u][r], sv);
               float f[8];
 #pragma unroll
               for (int i = 0; i < 8; ++i) {
-                float x = lv[u][r][i];
-                if constexpr (SH) x = fmaf(alpha, sv[u][r][i], x);
-                if constexpr (PR) x = fmaf(nbeta, pv[u][i], x);
+                float x = lv[i];
+                if constexpr (SH) x = fmaf(alpha, sv[i], x);
+                if constexpr (PR) x = fmaf(nbeta, pv[i], x);
                 f[i] = x;
               }
               st[r].push<8>(f, c);
@@ -263,7 +302,7 @@ __global__ void __launch_bounds__(kRowsThreads) k_verify_rows(RowsArgs a) {
     // holding the thread's maximum wins), and at the end the first element of
     // that vector equal to the maximum: the same lowest-index argmax as an
     // element-by-element scan, at a fraction of the instructions.
-    constexpr int U = 4;
+    constexpr int U = 8;
     constexpr int E = 16 / sizeof(T);
     const int step = kRowsThreads * E;
     int bvec = -1;
@@ -457,11 +496,15 @@ cudaError_t dispatch_rv(const RowsArgs& a, bool vec, bool finalize, cudaStream_t
 
 }  // namespace
 
-RowsPlan plan_rows(int rows, int V, int bytes_per_col, int num_sms, bool vec, int max_chunks) {
+RowsPlan plan_rows(int rows, int V, int bytes_per_col, int num_sms, bool vec, int max_chunks, bool multi_row) {
   RowsPlan p{};
   const long long target_items = 16LL * num_sms;
+  // Four rows per CTA (the prior read once per four rows) only for very many
+  // short rows; measured slower than one row per CTA otherwise.
+  p.rows_per_cta = (multi_row && vec && rows >= 64LL * num_sms) ? 4 : 1;
+  const long long groups0 = ((long long)rows + p.rows_per_cta - 1) / p.rows_per_cta;
   int nchunks = 1;
-  if (rows > 0 && rows < target_items) nchunks = (int)((target_items + rows - 1) / rows);
+  if (groups0 > 0 && groups0 < target_items) nchunks = (int)((target_items + groups0 - 1) / groups0);
   const int min_cols = std::max(2048, 32768 / std::max(1, bytes_per_col));
   nchunks = std::min(nchunks, std::max(1, V / min_cols));
   nchunks = std::max(1, std::min(nchunks, max_chunks));
@@ -470,8 +513,7 @@ RowsPlan plan_rows(int rows, int V, int bytes_per_col, int num_sms, bool vec, in
   nchunks = (V + chunk_cols - 1) / chunk_cols;
   p.nchunks = std::max(1, nchunks);
   p.chunk_cols = std::max(8, chunk_cols);
-  p.rows_per_cta = (vec && rows >= 64LL * num_sms && p.nchunks == 1) ? 4 : 1;
-  const long long groups = (rows + p.rows_per_cta - 1) / p.rows_per_cta;
+  const long long groups = groups0;
   p.grid = (int)std::min<long long>(groups * p.nchunks, INT_MAX);
   return p;
 }
