@@ -233,6 +233,9 @@ def draft_block(head, long, prior, alpha, beta, forced=None, keep_short=()):
     Position 0: x_0 = argmax l_L^(0) (no local head, no prior term).
     Position j >= 1: l_S^(j) = head(x_{0:j-1}); l^(j) = l_L^(j) + alpha l_S^(j)
     - beta l_P; x_j = argmax l^(j).
+    ``alpha`` / ``beta``: one weight for every position, or a sequence of n
+    per-position weights (alpha_j, beta_j; entry 0 is unused) — the
+    position-dependent weights whose learned values Appendix C reports.
 
     ``forced`` [B, n]: use these tokens as the drafted prefix instead of the
     oracle's own choices (to re-check a device run position by position after
@@ -242,6 +245,8 @@ def draft_block(head, long, prior, alpha, beta, forced=None, keep_short=()):
     L = long
     B, n, V = L.shape
     P = np.asarray(prior, dtype=np.float64)
+    a_j = np.broadcast_to(np.asarray(alpha, dtype=np.float64), (n,)) if np.ndim(alpha) else np.full(n, float(alpha))
+    b_j = np.broadcast_to(np.asarray(beta, dtype=np.float64), (n,)) if np.ndim(beta) else np.full(n, float(beta))
     tokens = np.zeros((B, n), np.int64)
     amax = np.zeros((B, n), np.int64)
     logp = np.zeros((B, n))
@@ -275,7 +280,7 @@ def draft_block(head, long, prior, alpha, beta, forced=None, keep_short=()):
         state, feat = head.step(state, prev)
         S = head.short_logits(feat)
         for b in range(B):
-            f = fuse(row_long(b, j), S[b], P, alpha, beta)
+            f = fuse(row_long(b, j), S[b], P, a_j[j], b_j[j])
             if (b, j) in keep_short:
                 kept[(b, j)] = S[b].copy()
             record(b, j, f)

@@ -377,3 +377,80 @@ def test_forced_prefix_mode_agrees_with_free_run():
                                 forced=free.tokens)
     np.testing.assert_array_equal(forced.argmax, free.tokens)
     np.testing.assert_allclose(forced.logp_at, free.logp, atol=1e-12)
+
+
+# ------------------------------------------------- per-position weights (Appendix C)
+
+def _learned_weights(n):
+    """alpha_j, beta_j for j = 0..n-1 from the Appendix C table (positions 2..15
+    are j = 1..14; later positions keep the last printed value; j = 0 unused)."""
+    path = os.path.join(os.path.dirname(__file__), "golden", "appendix_c_learned_weights.txt")
+    rows = [l.split() for l in open(path) if l.strip() and not l.startswith("#")]
+    tab = {int(p): (float(a), float(b)) for p, a, b in rows}
+    a = np.zeros(n)
+    b = np.zeros(n)
+    for j in range(1, n):
+        a[j], b[j] = tab[min(j + 1, max(tab))]
+    return a, b
+
+
+def test_appendix_c_table_is_read_as_printed():
+    a, b = _learned_weights(16)
+    assert a[1] == 0.547 and b[1] == 0.512 and a[14] == 0.762 and b[12] == 0.617
+    assert np.all(np.diff(a[1:]) >= 0)          # alpha grows with the position (Appendix C)
+
+
+def test_constant_per_position_weights_equal_the_scalar_weight():
+    base = synth.with_sizes(synth.stress(synth.WORKLOADS["tiny"]), V=64, B=3, n=6)
+    d = synth.make_inputs(base, target=False)
+    W = {k[5:]: v for k, v in d.items() if k.startswith("head.")}
+    prior = oracle.log_prior(d["counts"])
+    r0 = oracle.draft_block(oracle.make_head(base.head, W), d["long"], prior, 0.7, 0.4)
+    r1 = oracle.draft_block(oracle.make_head(base.head, W), d["long"], prior, np.full(6, 0.7), np.full(6, 0.4))
+    np.testing.assert_array_equal(r0.tokens, r1.tokens)
+    np.testing.assert_array_equal(r0.logp, r1.logp)
+
+
+def test_zero_weight_at_one_position_reproduces_dflash_there():
+    base = synth.with_sizes(synth.stress(synth.WORKLOADS["tiny"]), V=64, B=3, n=6)
+    d = synth.make_inputs(base, target=False)
+    W = {k[5:]: v for k, v in d.items() if k.startswith("head.")}
+    prior = oracle.log_prior(d["counts"])
+    a, b = _learned_weights(6)
+    a[3] = b[3] = 0.0
+    r = oracle.draft_block(oracle.make_head(base.head, W), d["long"], prior, a, b)
+    L = oracle.to_f64(d["long"])
+    np.testing.assert_array_equal(r.tokens[:, 3], np.argmax(L[:, 3], axis=1))
+    np.testing.assert_allclose(r.logp[:, 3], sps.log_softmax(L[:, 3], axis=1)[np.arange(3), r.tokens[:, 3]],
+                               atol=1e-12)
+
+
+def test_per_position_weights_brute_force_enumeration():
+    """As the brute-force pin above, with a different (alpha_j, beta_j) at every
+    position: exactly one block is greedy-consistent and the oracle returns it."""
+    V, n, B = 6, 4, 2
+    base = synth.with_sizes(synth.stress(synth.WORKLOADS["tiny"]), V=V, B=B, n=n,
+                            head_d_model=5, head_d_hidden=7, head_d_rank=7)
+    d = synth.make_inputs(base, target=False)
+    W = {k[5:]: v for k, v in d.items() if k.startswith("head.")}
+    prior = oracle.log_prior(d["counts"])
+    a = np.array([0.0, 2.1, 0.4, 1.6])
+    b = np.array([0.0, 0.3, 2.5, 1.1])
+    L = oracle.to_f64(d["long"])
+    res = oracle.draft_block(oracle.make_head(base.head, W), d["long"], prior, a, b)
+    for bb in range(B):
+        consistent = []
+        for blk in itertools.product(range(V), repeat=n):
+            ok = int(np.argmax(L[bb, 0])) == blk[0]
+            if ok:
+                head = oracle.make_head(base.head, W)
+                st = head.init(1)
+                for j in range(1, n):
+                    st, feat = head.step(st, np.array([blk[j - 1]]))
+                    score = L[bb, j] + a[j] * head.short_logits(feat)[0] - b[j] * prior
+                    if int(np.argmax(score)) != blk[j]:
+                        ok = False
+                        break
+            if ok:
+                consistent.append(blk)
+        assert consistent == [tuple(res.tokens[bb])]
