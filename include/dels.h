@@ -187,6 +187,18 @@ int dels_draft_block(const dels_local_head* head, const void* long_logits, dels_
                      int32_t* out_tokens, float* out_logprob, float* out_top2_gap, void* workspace,
                      size_t workspace_bytes, dels_stream_t stream);
 
+/*
+ * dels_draft_block with position-dependent fusion weights: position j >= 1
+ * uses l = l_L + alpha[j] l_S - beta[j] l_P (the learned per-position weights
+ * reported in Appendix C). alpha, beta: [host] float arrays of n entries
+ * (entry 0 is not used: position 0 has no head and no prior term), finite;
+ * read during the call. Everything else as dels_draft_block (same workspace).
+ */
+int dels_draft_block_weighted(const dels_local_head* head, const void* long_logits, dels_dtype logit_dtype,
+                              const float* log_prior, const float* alpha, const float* beta, int B, int n, int V,
+                              int32_t* out_tokens, float* out_logprob, float* out_top2_gap, void* workspace,
+                              size_t workspace_bytes, dels_stream_t stream);
+
 /* ---- fused combine + argmax over independent rows ---------------------- */
 
 size_t dels_combine_workspace_bytes(int rows, int V, dels_dtype dtype);

@@ -21,7 +21,7 @@ __all__ = [
     "DELS_HEAD_GRU", "DELS_HEAD_MLP", "DELS_HEAD_XFMR", "DELS_HEAD_MARKOV",
     "DELS_STATUS_NONFINITE", "DELS_STATUS_TIMEOUT", "DELS_STATUS_BAD_TOKEN",
     "DelsError", "LocalHead", "lib", "library_path", "exported_symbols",
-    "dels_draft_workspace_bytes", "dels_draft_block",
+    "dels_draft_workspace_bytes", "dels_draft_block", "dels_draft_block_weighted",
     "dels_combine_workspace_bytes", "dels_combine_argmax", "dels_combine_argmax_noalloc",
     "dels_verify_workspace_bytes", "dels_verify_block",
     "dels_read_status", "dels_prior_from_counts", "dels_status_string", "dels_version",
@@ -65,6 +65,8 @@ _SIGS = {
     "dels_draft_workspace_bytes": (_sz, [ctypes.POINTER(LocalHead), _i, _i, _i]),
     "dels_draft_block": (_i, [ctypes.POINTER(LocalHead), _vp, _i, _vp, _f, _f, _i, _i, _i, _vp, _vp, _vp, _vp, _sz,
                               _vp]),
+    "dels_draft_block_weighted": (_i, [ctypes.POINTER(LocalHead), _vp, _i, _vp, _vp, _vp, _i, _i, _i, _vp, _vp, _vp,
+                                       _vp, _sz, _vp]),
     "dels_combine_workspace_bytes": (_sz, [_i, _i, _i]),
     "dels_combine_argmax": (_i, [_vp, _vp, _i, _vp, _f, _f, _i, _i, _vp, _vp, _vp, _vp, _sz, _vp]),
     "dels_combine_argmax_noalloc": (_i, [_vp, _vp, _i, _vp, _f, _f, _i, _i, _vp, _vp, _vp, _vp]),
@@ -207,6 +209,19 @@ def dels_draft_block(head: LocalHead, long_logits, logit_dtype: int, log_prior, 
     return r
 
 
+def dels_draft_block_weighted(head: LocalHead, long_logits, logit_dtype: int, log_prior, alpha, beta, B: int,
+                              n: int, V: int, out_tokens, out_logprob, out_top2_gap, workspace,
+                              workspace_bytes: int, stream=None) -> int:
+    """Per-position fusion weights: ``alpha``/``beta`` are sequences of n floats
+    (host; entry 0 unused)."""
+    a = (ctypes.c_float * n)(*[float(x) for x in alpha])
+    b = (ctypes.c_float * n)(*[float(x) for x in beta])
+    return lib().dels_draft_block_weighted(ctypes.byref(head), _ptr(long_logits), logit_dtype, _ptr(log_prior),
+                                           ctypes.cast(a, ctypes.c_void_p), ctypes.cast(b, ctypes.c_void_p), B, n, V,
+                                           _ptr(out_tokens), _ptr(out_logprob), _ptr(out_top2_gap),
+                                           _ptr(workspace), workspace_bytes, _stream(stream))
+
+
 def dels_combine_workspace_bytes(rows: int, V: int, dtype: int) -> int:
     return lib().dels_combine_workspace_bytes(rows, V, dtype)
 
@@ -314,10 +329,18 @@ class Drafter:
         self.logprob = torch.empty(B, n, dtype=torch.float32, device=self.device)
         self.gap = torch.empty(B, n, dtype=torch.float32, device=self.device)
 
-    def __call__(self, long_logits: torch.Tensor, log_prior: torch.Tensor, alpha: float, beta: float, stream=None):
-        _check(dels_draft_block(self.head, long_logits, dtype_code(long_logits), log_prior, alpha, beta, self.B,
-                                self.n, self.V, self.tokens, self.logprob, self.gap, self.workspace, self.ws_bytes,
-                                stream), "dels_draft_block")
+    def __call__(self, long_logits: torch.Tensor, log_prior: torch.Tensor, alpha, beta, stream=None):
+        """``alpha``/``beta``: one weight for the block, or n per-position weights."""
+        if hasattr(alpha, "__len__") or hasattr(beta, "__len__"):
+            a = list(alpha) if hasattr(alpha, "__len__") else [alpha] * self.n
+            b = list(beta) if hasattr(beta, "__len__") else [beta] * self.n
+            _check(dels_draft_block_weighted(self.head, long_logits, dtype_code(long_logits), log_prior, a, b,
+                                             self.B, self.n, self.V, self.tokens, self.logprob, self.gap,
+                                             self.workspace, self.ws_bytes, stream), "dels_draft_block_weighted")
+        else:
+            _check(dels_draft_block(self.head, long_logits, dtype_code(long_logits), log_prior, alpha, beta, self.B,
+                                    self.n, self.V, self.tokens, self.logprob, self.gap, self.workspace,
+                                    self.ws_bytes, stream), "dels_draft_block")
         return self.tokens, self.logprob, self.gap
 
     def status(self, stream=None) -> int:

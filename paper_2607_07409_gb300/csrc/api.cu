@@ -791,10 +791,19 @@ size_t dels_draft_workspace_bytes(const dels_local_head* head, int B, int n, int
   return L.ok ? L.total : 0;
 }
 
-int dels_draft_block(const dels_local_head* head, const void* long_logits, dels_dtype logit_dtype,
-                     const float* log_prior, float alpha, float beta, int B, int n, int V, int32_t* out_tokens,
-                     float* out_logprob, float* out_top2_gap, void* workspace, size_t workspace_bytes,
-                     dels_stream_t stream) {
+}  // extern "C"
+
+namespace dels {
+namespace {
+
+// dels_draft_block with the fusion weights of position j given by aw(j),
+// bw(j): one pair for the block, or per-position arrays.
+int draft_block_impl(const dels_local_head* head, const void* long_logits, dels_dtype logit_dtype,
+                     const float* log_prior, float alpha, float beta, const float* alpha_j, const float* beta_j,
+                     int B, int n, int V, int32_t* out_tokens, float* out_logprob, float* out_top2_gap,
+                     void* workspace, size_t workspace_bytes, dels_stream_t stream) {
+  auto aw = [&](int j) { return alpha_j ? alpha_j[j] : alpha; };
+  auto bw = [&](int j) { return beta_j ? beta_j[j] : beta; };
   int r = validate_draft(head, long_logits, logit_dtype, log_prior, B, n, V, out_tokens, out_logprob, out_top2_gap);
   if (r != DELS_OK) return r;
   if (!workspace) return DELS_ERR_WORKSPACE;
@@ -833,7 +842,7 @@ int dels_draft_block(const dels_local_head* head, const void* long_logits, dels_
       void* rr = at<void>(workspace, L.r);
       mb.D = D;
       mb.dest = eg;
-      if (bf && persistent_enabled() && B <= sms && R <= 256) {
+      if (bf && persistent_enabled() && !alpha_j && !beta_j && B <= sms && R <= 256) {
         // one cooperative launch for the whole block
         Gemm gg, gr, gv;
         if (!plan_store(gg, B, 3 * H, eg, head->w[0], D, hb, head->w[1], H, 128, L.gru_s0, L.gru_s1, ACT_NONE,
@@ -957,6 +966,8 @@ int dels_draft_block(const dels_local_head* head, const void* long_logits, dels_
           ga.S = j == 1 ? 0 : gh.a.total_splits;
           { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_gru_gates_table(ga, s)); }
           P.vocab.j = j;
+          P.vocab.alpha = aw(j);
+          P.vocab.beta = bw(j);
           P.hh_ctas = j + 1 < n ? std::min(hh_items, grid - P.rank_ctas) : 0;
           P.r_target = (unsigned)(j * gr.a.num_o_tiles);
           { PROF(DELS_KCLASS_VOCAB_COMBINE); DELS_CUDA(launch_prod_vocab(P, maps, grid, smem, s)); }
@@ -1028,6 +1039,10 @@ int dels_draft_block(const dels_local_head* head, const void* long_logits, dels_
             DELS_CUDA(launch_tc_gemm(gr.a, &gr.mA0, &gr.mB0, &gr.mA1, &gr.mB1, &gr.mL, gr.grid, gr.smem, s,
                                      j + 1 < n ? &hh : nullptr)); }
           gv.a.j = j;
+        gv.a.alpha = aw(j);
+        gv.a.beta = bw(j);
+          gv.a.alpha = aw(j);
+          gv.a.beta = bw(j);
           { PROF(DELS_KCLASS_VOCAB_COMBINE); DELS_CUDA(run(gv, s)); }
         }
         MergeArgs m = mb;
@@ -1061,6 +1076,10 @@ int dels_draft_block(const dels_local_head* head, const void* long_logits, dels_
           { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_gru_gates(gpart, gg.a.seg_splits[0], gg.a.seg_splits[1], B, H, h, hb, s)); }
           { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run(gr, s)); }
           gv.a.j = j;
+        gv.a.alpha = aw(j);
+        gv.a.beta = bw(j);
+          gv.a.alpha = aw(j);
+          gv.a.beta = bw(j);
           { PROF(DELS_KCLASS_VOCAB_COMBINE); DELS_CUDA(run(gv, s)); }
           MergeArgs m = mb;
           m.count = gv.grid;
@@ -1083,7 +1102,7 @@ int dels_draft_block(const dels_local_head* head, const void* long_logits, dels_
           { PROF(DELS_KCLASS_VOCAB_COMBINE); DELS_CUDA(launch_vocab_combine_f32(feat, R, static_cast<const float*>(head->w_vocab),
                                              static_cast<const uint8_t*>(long_logits) +
                                                  (size_t)j * V * (logit_dtype == DELS_F32 ? 4 : 2),
-                                             logit_dtype == DELS_F32, (long long)n * V, log_prior, alpha, beta, B, V,
+                                             logit_dtype == DELS_F32, (long long)n * V, log_prior, aw(j), bw(j), B, V,
                                              partials, L.partial_ld, nch, status, s)); }
           MergeArgs m = mb;
           m.count = nch;
@@ -1128,6 +1147,10 @@ int dels_draft_block(const dels_local_head* head, const void* long_logits, dels_
                                            static_cast<uint16_t*>(h2), Hd, s)); }
           }
           gv.a.j = j;
+        gv.a.alpha = aw(j);
+        gv.a.beta = bw(j);
+          gv.a.alpha = aw(j);
+          gv.a.beta = bw(j);
           { PROF(DELS_KCLASS_VOCAB_COMBINE); DELS_CUDA(run(gv, s)); }
           MergeArgs m = mb;
           m.count = gv.grid;
@@ -1147,7 +1170,7 @@ int dels_draft_block(const dels_local_head* head, const void* long_logits, dels_
                                              static_cast<const float*>(head->w_vocab),
                                              static_cast<const uint8_t*>(long_logits) +
                                                  (size_t)j * V * (logit_dtype == DELS_F32 ? 4 : 2),
-                                             logit_dtype == DELS_F32, (long long)n * V, log_prior, alpha, beta, B, V,
+                                             logit_dtype == DELS_F32, (long long)n * V, log_prior, aw(j), bw(j), B, V,
                                              partials, L.partial_ld, nch, status, s)); }
           MergeArgs m = mb;
           m.count = nch;
@@ -1215,6 +1238,8 @@ int dels_draft_block(const dels_local_head* head, const void* long_logits, dels_
         { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_splitk_finish(xpart, g2.a.total_splits, B, D, uu, ACT_NONE, y, D, nullptr, 0, s)); }
         { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_rmsnorm_bf16(y, B, D, D, feat, s)); }
         gv.a.j = j;
+        gv.a.alpha = aw(j);
+        gv.a.beta = bw(j);
         { PROF(DELS_KCLASS_VOCAB_COMBINE); DELS_CUDA(run(gv, s)); }
         MergeArgs m = mb;
         m.count = gv.grid;
@@ -1240,6 +1265,10 @@ int dels_draft_block(const dels_local_head* head, const void* long_logits, dels_
         int count;
         if (bf) {
           gv.a.j = j;
+        gv.a.alpha = aw(j);
+        gv.a.beta = bw(j);
+          gv.a.alpha = aw(j);
+          gv.a.beta = bw(j);
           { PROF(DELS_KCLASS_VOCAB_COMBINE); DELS_CUDA(run(gv, s)); }
           count = gv.grid;
         } else {
@@ -1247,7 +1276,7 @@ int dels_draft_block(const dels_local_head* head, const void* long_logits, dels_
                                              static_cast<const float*>(head->w_vocab),
                                              static_cast<const uint8_t*>(long_logits) +
                                                  (size_t)j * V * (logit_dtype == DELS_F32 ? 4 : 2),
-                                             logit_dtype == DELS_F32, (long long)n * V, log_prior, alpha, beta, B, V,
+                                             logit_dtype == DELS_F32, (long long)n * V, log_prior, aw(j), bw(j), B, V,
                                              partials, L.partial_ld, nch, status, s)); }
           count = nch;
         }
@@ -1262,6 +1291,31 @@ int dels_draft_block(const dels_local_head* head, const void* long_logits, dels_
     default:
       return DELS_ERR_UNSUPPORTED;
   }
+}
+
+}  // namespace
+}  // namespace dels
+
+extern "C" {
+
+int dels_draft_block(const dels_local_head* head, const void* long_logits, dels_dtype logit_dtype,
+                     const float* log_prior, float alpha, float beta, int B, int n, int V, int32_t* out_tokens,
+                     float* out_logprob, float* out_top2_gap, void* workspace, size_t workspace_bytes,
+                     dels_stream_t stream) {
+  return draft_block_impl(head, long_logits, logit_dtype, log_prior, alpha, beta, nullptr, nullptr, B, n, V,
+                          out_tokens, out_logprob, out_top2_gap, workspace, workspace_bytes, stream);
+}
+
+int dels_draft_block_weighted(const dels_local_head* head, const void* long_logits, dels_dtype logit_dtype,
+                              const float* log_prior, const float* alpha, const float* beta, int B, int n, int V,
+                              int32_t* out_tokens, float* out_logprob, float* out_top2_gap, void* workspace,
+                              size_t workspace_bytes, dels_stream_t stream) {
+  if (!alpha || !beta) return DELS_ERR_NULL_POINTER;
+  if (n < 1 || n > 32) return DELS_ERR_BAD_SHAPE;
+  for (int j = 0; j < n; ++j)
+    if (!std::isfinite(alpha[j]) || !std::isfinite(beta[j])) return DELS_ERR_BAD_SHAPE;
+  return draft_block_impl(head, long_logits, logit_dtype, log_prior, 0.f, 0.f, alpha, beta, B, n, V, out_tokens,
+                          out_logprob, out_top2_gap, workspace, workspace_bytes, stream);
 }
 
 }  // extern "C"

@@ -117,3 +117,17 @@ def test_draft_validation(dels):
     h.wdtype = 0
     assert L.dels_draft_block(*args(4, 16, 151936)) == -6            # f32 transformer head unsupported
     assert L.dels_draft_workspace_bytes(ctypes.byref(h), 4, 16, 151936) == 0
+
+
+def test_weighted_draft_rejects_bad_weights_before_enqueueing(dels):
+    L = dels.lib()
+    h = dels.LocalHead()
+    n = 4
+    good = (ctypes.c_float * n)(0.0, 0.5, 0.5, 0.5)
+    bad = (ctypes.c_float * n)(0.0, float("nan"), 0.5, 0.5)
+    args = lambda a, b, nn: (ctypes.byref(h), None, 0, None, a, b, 1, nn, 64, None, None, None, None, 0, None)
+    assert L.dels_draft_block_weighted(*args(None, ctypes.cast(good, ctypes.c_void_p), n)) == -1
+    assert L.dels_draft_block_weighted(*args(ctypes.cast(good, ctypes.c_void_p), ctypes.cast(bad, ctypes.c_void_p),
+                                             n)) == -2
+    assert L.dels_draft_block_weighted(*args(ctypes.cast(good, ctypes.c_void_p), ctypes.cast(good, ctypes.c_void_p),
+                                             0)) == -2

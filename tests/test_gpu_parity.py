@@ -292,6 +292,39 @@ def test_draft_fused_products_vocab_kernel_matches_oracle(name, stress, monkeypa
     print(name, stress, info)
 
 
+def _learned_weights(n):
+    """Per-position (alpha_j, beta_j) from the Appendix C table (positions 2..15
+    are j = 1..14; later positions keep the last printed value)."""
+    import os
+    path = os.path.join(os.path.dirname(__file__), "golden", "appendix_c_learned_weights.txt")
+    rows = [l.split() for l in open(path) if l.strip() and not l.startswith("#")]
+    tab = {int(p): (float(a), float(b)) for p, a, b in rows}
+    a, b = [0.0] * n, [0.0] * n
+    for j in range(1, n):
+        a[j], b[j] = tab[min(j + 1, max(tab))]
+    return a, b
+
+
+@pytest.mark.parametrize("name", ["gru", "gru_b64", "mlp2", "xfmr", "markov", "gru_f32", "tiny"])
+def test_draft_per_position_weights_match_oracle(name):
+    w = synth.stress(SMALL[name])
+    d = synth.make_inputs(w, device=DEV, target=False)
+    if name == "gru_b64":
+        d = _with_table(w, d)
+    a, b = _learned_weights(w.n)
+    W = {k[5:]: v for k, v in d.items() if k.startswith("head.")}
+    prior = dels.dels_prior_from_counts(d["counts"]).to(DEV)
+    dr = dels.Drafter(w.head, W, w.B, w.n, w.V)
+    tok, lp, gap = dr(d["long"], prior, a, b)
+    torch.cuda.synchronize()
+    assert dr.status() == 0
+    W = {k: v for k, v in W.items() if k != "input_table"}
+    tol = LP_TOL_F32 if w.head.wdtype == "f32" else LP_TOL_BF16
+    info = check_draft(tok.cpu().numpy(), lp.cpu().numpy(), gap.cpu().numpy(), _oracle_head(w, W), d["long"].cpu(),
+                       oracle.log_prior(d["counts"]), np.array(a), np.array(b), tol)
+    print(name, info)
+
+
 def test_draft_zero_weight_is_dflash_argmax():
     w = synth.with_sizes(synth.stress(synth.WORKLOADS["qwen3_8b_batched"]), B=8, n=5, V=2048, weight=0.0,
                          head_d_model=128, head_d_hidden=64, head_d_rank=64)
