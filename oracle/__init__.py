@@ -18,8 +18,8 @@ Speculative Drafting"):
 * Appendix A, local heads: the RNN head (target embedding -> one bias-free GRU
   layer -> SiLU(W_rank h) -> W_vocab r) and the Markov head
   (r = E_M(x_{i-1}), l_S = W_M r).
-* Appendix A, unigram prior: p0(v) = (c(v) + lambda) / sum(c + lambda),
-  l_P = log p0.
+* Appendix A, unigram prior: c(v) counts the loss-masked corpus tokens equal
+  to v; p0(v) = (c(v) + lambda) / sum(c + lambda), l_P = log p0.
 * Section 4.1 and Appendix B: the exact three-factor factorisation of
   p(x | y, z) (used by the tests to pin the alpha = beta = 1 case).
 * Appendix D: rate_i = P(acceptance length >= i).
@@ -41,6 +41,7 @@ factorisation) and ``heads`` (local heads and the block drafting loop).
 from .core import (  # noqa: F401
     to_f64,
     round_bf16,
+    count_masked_tokens,
     log_prior,
     lse,
     fuse,

@@ -48,6 +48,26 @@ def round_bf16(x: np.ndarray) -> np.ndarray:
 # unigram prior (Appendix A, "Unigram Prior Estimation")
 # ----------------------------------------------------------------------------
 
+def count_masked_tokens(tokens, loss_mask, V: int):
+    """c(v) = number of corpus positions t with loss_mask[t] == 1 and tokens[t] == v.
+
+    Only loss-masked (assistant-response) tokens are counted. A masked
+    position whose id lies outside [0, V) is not counted in c; it is reported
+    separately. Returns (c as int64 [V], masked in-range total, masked
+    out-of-range total).
+    """
+    t = np.asarray(tokens).reshape(-1).astype(np.int64)
+    m = np.asarray(loss_mask).reshape(-1)
+    if t.shape != m.shape:
+        raise ValueError("tokens and loss_mask must have the same length")
+    if V <= 0:
+        raise ValueError("V must be positive")
+    sel = t[m != 0]
+    ok = (sel >= 0) & (sel < V)
+    c = np.bincount(sel[ok], minlength=V).astype(np.int64)
+    return c, int(ok.sum()), int((~ok).sum())
+
+
 def log_prior(counts, lam: float = 1.0) -> np.ndarray:
     """l_P(v) = log( (c(v) + lambda) / sum_v' (c(v') + lambda) ), lambda = 1 by default."""
     c = to_f64(counts)

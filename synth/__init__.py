@@ -48,6 +48,8 @@ __all__ = [
     "make_long_logits",
     "make_target_logits",
     "make_counts",
+    "make_corpus",
+    "CORPUS_TOKENS",
     "make_combine_inputs",
     "make_planted_verify",
     "sweep_points",
@@ -224,6 +226,46 @@ def make_counts(w: Workload, total: float = 1e7) -> torch.Tensor:
     q = (rank + 1.0).pow(-1.1)
     q = q / q.sum()
     return torch.floor(q * total).to(torch.int64)
+
+
+# Size of the synthetic training corpus the prior is estimated from: 2^28
+# token positions (1.34 GB as int32 ids plus a byte mask), of the order of a
+# ShareGPT-style chat corpus of ~100K conversations.
+CORPUS_TOKENS = 1 << 28
+
+
+def make_corpus(V: int, N: int, seed: int, device="cpu", chunk: int = 1 << 25):
+    """A synthetic chat corpus of N token positions: (tokens int32 [N], loss_mask uint8 [N]).
+
+    Ids follow the Zipf(1.1) law of ``make_counts`` over the same seeded
+    frequency ranking, drawn by inverse-CDF lookup of uniform variates. The
+    mask alternates user spans (mask 0, lengths uniform in [8, 256]) with
+    assistant spans (mask 1, lengths uniform in [16, 768]), so about three
+    quarters of the positions carry loss, as in supervised chat data.
+    """
+    if N < 0 or V <= 0:
+        raise ValueError("need N >= 0 and V > 0")
+    g = _gen(seed * 7919 + 71, device)
+    by_rank = torch.argsort(_zipf_rank(V, seed, device))          # token id of each rank
+    q = (torch.arange(V, device=device, dtype=torch.float64) + 1.0).pow(-1.1)
+    cdf = torch.cumsum(q, 0)
+    cdf = cdf / cdf[-1]
+    tokens = torch.empty(N, dtype=torch.int32, device=device)
+    for a in range(0, N, chunk):
+        b = min(N, a + chunk)
+        u = torch.rand(b - a, generator=g, device=device, dtype=torch.float64)
+        r = torch.searchsorted(cdf, u).clamp_(max=V - 1)
+        tokens[a:b] = by_rank[r].to(torch.int32)
+    spans = 2 * (N // (2 * (8 + 16)) + 1)                         # enough spans to cover N
+    lo = torch.tensor([8, 16], device=device).repeat(spans // 2)
+    hi = torch.tensor([257, 769], device=device).repeat(spans // 2)
+    lens = lo + (torch.rand(spans, generator=g, device=device) * (hi - lo).to(torch.float32)).long()
+    lens = torch.minimum(lens, hi - 1)
+    vals = torch.tensor([0, 1], dtype=torch.uint8, device=device).repeat(spans // 2)
+    cum = torch.cumsum(lens, 0)
+    k = int(torch.searchsorted(cum, torch.tensor([N], device=device)).item()) + 1
+    mask = torch.repeat_interleave(vals[:k], lens[:k])[:N].contiguous()
+    return tokens, mask
 
 
 def make_inputs(w: Workload, device="cpu", target: bool = True) -> Dict[str, torch.Tensor]:

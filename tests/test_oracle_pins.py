@@ -33,6 +33,72 @@ def test_prior_closed_forms():
     np.testing.assert_allclose(lp, np.log(np.array([6, 2, 12]) / 20.0), atol=1e-15)
 
 
+def test_masked_counts_brute_force():
+    """c(v) counts only loss-masked positions; ids outside [0, V) are reported, not counted."""
+    rng = np.random.default_rng(11)
+    V, N = 37, 3001
+    tok = rng.integers(-3, V + 4, size=N).astype(np.int32)
+    mask = (rng.random(N) < 0.6).astype(np.uint8)
+    mask[::7] = 2                                   # any nonzero byte carries loss
+    c, n_in, n_out = oracle.count_masked_tokens(tok, mask, V)
+    ref = [0] * V
+    ref_in = ref_out = 0
+    for t, m in zip(tok.tolist(), mask.tolist()):
+        if m == 0:
+            continue
+        if 0 <= t < V:
+            ref[t] += 1
+            ref_in += 1
+        else:
+            ref_out += 1
+    assert c.tolist() == ref and (n_in, n_out) == (ref_in, ref_out)
+    assert c.dtype == np.int64 and c.shape == (V,)
+
+
+def test_masked_counts_invariants():
+    tok, mask = synth.make_corpus(1000, 20000, seed=3)
+    tok, mask = tok.numpy(), mask.numpy()
+    c, n_in, n_out = oracle.count_masked_tokens(tok, mask, 1000)
+    assert n_out == 0 and n_in == int(mask.sum()) == int(c.sum())
+    # the order of the corpus does not matter
+    perm = np.random.default_rng(0).permutation(tok.size)
+    c2, _, _ = oracle.count_masked_tokens(tok[perm], mask[perm], 1000)
+    np.testing.assert_array_equal(c, c2)
+    # counting a corpus in two pieces and adding gives the whole corpus's counts
+    ca, _, _ = oracle.count_masked_tokens(tok[:7777], mask[:7777], 1000)
+    cb, _, _ = oracle.count_masked_tokens(tok[7777:], mask[7777:], 1000)
+    np.testing.assert_array_equal(ca + cb, c)
+    # unmasked positions never count
+    c0, z_in, z_out = oracle.count_masked_tokens(tok, np.zeros_like(mask), 1000)
+    assert not c0.any() and z_in == z_out == 0
+    # an empty corpus
+    ce, e_in, e_out = oracle.count_masked_tokens(np.zeros(0, np.int32), np.zeros(0, np.uint8), 5)
+    assert ce.tolist() == [0] * 5 and e_in == e_out == 0
+
+
+def test_prior_from_a_balanced_corpus_is_uniform():
+    """Every id loss-masked exactly k times: p0 is uniform whatever lambda is."""
+    V, k = 50, 4
+    tok = np.tile(np.arange(V, dtype=np.int32), k)
+    tok = np.concatenate([tok, np.arange(V, dtype=np.int32)])     # unmasked tail
+    mask = np.concatenate([np.ones(V * k, np.uint8), np.zeros(V, np.uint8)])
+    c, _, _ = oracle.count_masked_tokens(tok, mask, V)
+    assert c.tolist() == [k] * V
+    for lam in (1.0, 0.25):
+        np.testing.assert_allclose(oracle.log_prior(c, lam), np.full(V, -math.log(V)), atol=1e-15)
+
+
+def test_synthetic_corpus_follows_its_zipf_law():
+    """The corpus generator's masked frequencies follow q(v) ~ (pi(v) + 1)^-1.1 of make_counts."""
+    w = synth.WORKLOADS["qwen3_8b_batched"]
+    tok, mask = synth.make_corpus(w.V, 1 << 20, w.seed)
+    c, n_in, _ = oracle.count_masked_tokens(tok.numpy(), mask.numpy(), w.V)
+    assert 0.7 < n_in / tok.numel() < 0.8
+    q = synth.make_counts(w, total=1.0 * n_in).numpy()        # floor(n_in * q(v))
+    top = np.argsort(-q)[:20]
+    np.testing.assert_allclose(c[top], q[top], rtol=0.05)
+
+
 def test_prior_normalises_and_orders():
     c = synth.make_counts(synth.WORKLOADS["qwen3_8b_batched"])
     lp = oracle.log_prior(c)
