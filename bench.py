@@ -52,6 +52,9 @@ def parse_args():
     p.add_argument("--sweep", action="store_true",
                    help="instead of the drafting step: HBM GB/s of dels_combine_argmax and dels_verify_block over "
                         "the combine/verify sweep grid (one JSON line per point)")
+    p.add_argument("--prior", action="store_true",
+                   help="instead of the drafting step: device unigram-prior estimation (masked token histogram, "
+                        "smoothing, log) over a 2^28-position synthetic chat corpus")
     p.add_argument("--no-input-table", action="store_true",
                    help="recompute the GRU input product W_ih E[x] at every position instead of reading the "
                         "precomputed table G = E W_ih^T")
@@ -535,12 +538,106 @@ def run_sweep(args):
     return 0
 
 
+def run_prior(args):
+    """Corpus positions per second of dels_prior_estimate (zero the counts,
+    count the loss-masked ids, write l_P) over the 2^28-position synthetic
+    corpus of synth.make_corpus (V = 151936). The corpus (1.34 GB) is larger
+    than L2, so no flush is needed between steps. The count kernel is also
+    timed alone (dels_prior_count, one launch) for the roofline: it reads
+    4 bytes of id and 1 byte of mask per position."""
+    import torch
+    import numpy as np
+    import synth
+    import paper_2607_07409_gb300 as dels
+    from paper_2607_07409_gb300 import replicas
+    world, rank, local = dist_setup(args.gpus)
+    dev = torch.device(f"cuda:{local}")
+    torch.cuda.set_device(dev)
+    peak, peak_kind = measured_peaks()
+    w = synth.WORKLOADS[WORKLOAD]
+    V, N = w.V, synth.CORPUS_TOKENS
+    tok, mask = synth.make_corpus(V, N, replicas.replica_seed(w.seed, rank), device=dev)
+    nbytes = dels.dels_prior_workspace_bytes(V)
+    ws = torch.zeros(nbytes, dtype=torch.uint8, device=dev)
+    out = torch.empty(V, dtype=torch.float32, device=dev)
+    counts = torch.empty(V, dtype=torch.int64, device=dev)
+    tally = torch.empty(2, dtype=torch.int64, device=dev)
+
+    def estimate():
+        r = dels.dels_prior_estimate(tok, mask, N, V, 1.0, out, counts, tally, ws, nbytes)
+        if r != 0:
+            raise dels.DelsError(r, "dels_prior_estimate")
+
+    acc = torch.zeros(V, dtype=torch.int64, device=dev)
+
+    def count_only():
+        r = dels.dels_prior_count(tok, mask, N, V, acc, None, ws, nbytes)
+        if r != 0:
+            raise dels.DelsError(r, "dels_prior_count")
+
+    def timed(fn, k):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        a.record()
+        for _ in range(k):
+            fn()
+        b.record()
+        b.synchronize()
+        return a.elapsed_time(b) * 1e-3 / k
+
+    for _ in range(args.warmup):
+        estimate()
+        count_only()
+    torch.cuda.synchronize()
+    replicas.barrier()
+    clk = ClockSampler(local)
+    with clk:
+        t_est = replicas.max_over_ranks(timed(estimate, args.steps))
+        t_cnt = replicas.max_over_ranks(timed(count_only, args.steps))
+    st = dels.dels_read_status(ws)
+    c = counts.cpu().numpy()
+    t = tally.cpu().numpy()
+    masked = int(mask.sum(dtype=torch.int64).item())
+    props = bool(st == 0 and t[0] == masked and t[1] == 0 and c.sum() == masked
+                 and np.isclose(np.exp(out.double().cpu().numpy()).sum(), 1.0, atol=1e-5))
+    # oracle on a bounded sample of the same corpus, on the host cores
+    cpu = None
+    if rank == 0 and not args.no_cpu_baseline:
+        import oracle
+        n_s = 1 << 25
+        ts, ms = tok[:n_s].cpu().numpy(), mask[:n_s].cpu().numpy()
+        t0 = time.perf_counter()
+        c_s, _, _ = oracle.count_masked_tokens(ts, ms, V)
+        oracle.log_prior(c_s)
+        dt = time.perf_counter() - t0
+        cpu = {"value": n_s / dt, "unit": "corpus positions/s", "cores": 1, "kind": "oracle",
+               "sample": f"first {n_s} positions of the corpus (count + log prior)"}
+    cnt_bytes = 5 * N
+    if rank == 0:
+        print(json.dumps({
+            "metric": "unigram prior estimation: corpus positions/s (masked histogram + smoothing + log)",
+            "value": world * N / t_est, "unit": "corpus positions/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": t_est * 1e3, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "int32 ids, u8 mask, u64 counts, f64 log", "data": "synthetic",
+            "config": {"workload": f"chat corpus N={N} V={V} Zipf(1.1) ids, ~75% loss-masked",
+                       "l2": "inputs larger than L2"},
+            "roofline": {"bound": "hbm", "kernel": "k_prior_count", "achieved": cnt_bytes / t_cnt / 1e9,
+                         "peak": peak, "unit": "GB/s", "frac": cnt_bytes / t_cnt / 1e9 / peak,
+                         "peak_source": peak_kind, "us_per_launch": t_cnt * 1e6, "algorithmic_bytes": cnt_bytes},
+            "gpu_launches": 2 * args.steps + args.steps,
+            "properties_ok": props, "clocks": clk.summary(), "cpu_baseline": cpu}), flush=True)
+    replicas.barrier()
+    return 0
+
+
 def main():
     args = parse_args()
     if args.impl == "reference":
         return run_reference(args)
     if args.sweep:
         return run_sweep(args)
+    if args.prior:
+        return run_prior(args)
     return run_ours(args)
 
 

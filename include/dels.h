@@ -62,7 +62,7 @@ enum {
   /* detected on the device; bits of the workspace status word */
   DELS_STATUS_NONFINITE = 1,       /* NaN or +inf logit, or a row that is all -inf */
   DELS_STATUS_TIMEOUT = 2,         /* a bounded device-side wait expired */
-  DELS_STATUS_BAD_TOKEN = 4        /* a draft token outside [0, V) */
+  DELS_STATUS_BAD_TOKEN = 4        /* a draft or loss-masked corpus token outside [0, V) */
 };
 
 typedef enum { DELS_F32 = 0, DELS_BF16 = 1 } dels_dtype;
@@ -289,6 +289,56 @@ int dels_read_status(void* workspace, dels_stream_t stream, int32_t* out_status)
  */
 int dels_prior_from_counts(const int64_t* counts, int V, double lambda, float* out_log_prior);
 
+/* ---- unigram prior estimation on the device (Appendix A) ----------------- */
+
+/*
+ * The prior the fusion subtracts is estimated once from the training corpus:
+ * c(v) counts the corpus positions that carry loss (assistant-response
+ * tokens) and hold token v; p0(v) = (c(v) + lambda) / sum_u (c(u) + lambda)
+ * with lambda = 1 by default; l_P(v) = log p0(v).
+ *
+ * Corpus layout: tokens [device] [N] int32 ids (4-byte aligned; any offset
+ * into a larger corpus is accepted, 16-byte alignment is fastest) and
+ * loss_mask [device] [N] uint8, one byte per position, nonzero = the position
+ * carries loss. Counts are uint64. A loss-masked position whose id lies
+ * outside [0, V) is not counted: it is tallied separately and sets
+ * DELS_STATUS_BAD_TOKEN in the workspace status word.
+ */
+size_t dels_prior_workspace_bytes(int V);
+
+/*
+ * Adds one corpus piece's loss-masked token counts to `counts`:
+ *   counts[v] += #{ t < N : loss_mask[t] != 0 and tokens[t] == v }.
+ * counts [device] [V] uint64, accumulated (zero it before the first piece);
+ * tally  [device] [2] uint64 or NULL, accumulated: tally[0] += positions
+ *        counted, tally[1] += loss-masked positions with an id outside [0, V).
+ * workspace [device]: at least 256 bytes (only its status word is used) or
+ * the dels_prior_workspace_bytes(V) buffer of the other prior calls.
+ * Limits: N >= 0 (N = 0 enqueues nothing), 1 <= V < 2^31.
+ */
+int dels_prior_count(const int32_t* tokens, const uint8_t* loss_mask, int64_t N, int V, uint64_t* counts,
+                     uint64_t* tally, void* workspace, size_t workspace_bytes, dels_stream_t stream);
+
+/*
+ * l_P from counts on the device: the sum of the counts, then
+ *   out_log_prior[v] = log(counts[v] + lambda) - log(sum_u counts[u] + V * lambda)
+ * evaluated in float64 and stored as float32 (within one float32 rounding of
+ * the exact value). counts [device] [V] uint64; out_log_prior [device] [V]
+ * float32; lambda > 0 and finite; workspace >= dels_prior_workspace_bytes(V).
+ */
+int dels_prior_log(const uint64_t* counts, int V, double lambda, float* out_log_prior, void* workspace,
+                   size_t workspace_bytes, dels_stream_t stream);
+
+/*
+ * Both steps for a corpus held in device memory: zeroes counts kept in the
+ * workspace, counts, and writes l_P. out_counts [device] [V] uint64 and
+ * out_tally [device] [2] uint64 (as for dels_prior_count) are optional copies.
+ * workspace >= dels_prior_workspace_bytes(V).
+ */
+int dels_prior_estimate(const int32_t* tokens, const uint8_t* loss_mask, int64_t N, int V, double lambda,
+                        float* out_log_prior, uint64_t* out_counts, uint64_t* out_tally, void* workspace,
+                        size_t workspace_bytes, dels_stream_t stream);
+
 /* ---- instrumentation (not part of the method) ---------------------------- */
 
 /* Kernel classes timed by the optional per-kernel profiler. */
@@ -301,7 +351,8 @@ enum {
   DELS_KCLASS_VERIFY = 5,        /* verification                                          */
   DELS_KCLASS_COMBINE = 6,       /* dels_combine_argmax                                   */
   DELS_KCLASS_DRAFT_BLOCK = 7,   /* persistent per-block drafting kernel (whole block)    */
-  DELS_KCLASS_COUNT = 8
+  DELS_KCLASS_PRIOR = 8,         /* unigram prior estimation (count, sum, log)            */
+  DELS_KCLASS_COUNT = 9
 };
 
 /*

@@ -28,6 +28,7 @@ __all__ = [
     "dels_profile_enable", "dels_profile_reset", "dels_profile_read", "KCLASS",
     "dels_gru_input_table_bytes", "dels_gru_build_input_table", "gru_input_table",
     "dels_selftest_timeout_bytes", "dels_selftest_timeout",
+    "dels_prior_workspace_bytes", "dels_prior_count", "dels_prior_log", "dels_prior_estimate", "estimate_prior",
     "make_head", "Drafter", "dtype_code",
 ]
 
@@ -74,6 +75,10 @@ _SIGS = {
     "dels_verify_block": (_i, [_vp, _vp, _i, _i, _i, _i, _vp, _vp, _vp, _vp, _sz, _vp]),
     "dels_read_status": (_i, [_vp, _vp, ctypes.POINTER(ctypes.c_int32)]),
     "dels_prior_from_counts": (_i, [_vp, _i, _d, _vp]),
+    "dels_prior_workspace_bytes": (_sz, [_i]),
+    "dels_prior_count": (_i, [_vp, _vp, ctypes.c_int64, _i, _vp, _vp, _vp, _sz, _vp]),
+    "dels_prior_log": (_i, [_vp, _i, _d, _vp, _vp, _sz, _vp]),
+    "dels_prior_estimate": (_i, [_vp, _vp, ctypes.c_int64, _i, _d, _vp, _vp, _vp, _vp, _sz, _vp]),
     "dels_status_string": (ctypes.c_char_p, [_i]),
     "dels_version": (_i, []),
     "dels_profile_enable": (_i, [_i]),
@@ -83,7 +88,7 @@ _SIGS = {
 
 # kernel classes of the optional profiler
 KCLASS = {"vocab_combine": 0, "head_gemm": 1, "head_misc": 2, "merge": 3, "pos0": 4, "verify": 5, "combine": 6,
-          "draft_block": 7}
+          "draft_block": 7, "prior": 8}
 
 
 def exported_symbols():
@@ -267,6 +272,51 @@ def dels_prior_from_counts(counts: torch.Tensor, lam: float = 1.0) -> torch.Tens
     _check(lib().dels_prior_from_counts(c.data_ptr(), c.numel(), float(lam), out.data_ptr()),
            "dels_prior_from_counts")
     return out
+
+
+def dels_prior_workspace_bytes(V: int) -> int:
+    return lib().dels_prior_workspace_bytes(V)
+
+
+def dels_prior_count(tokens, loss_mask, N: int, V: int, counts, tally, workspace, workspace_bytes: int,
+                     stream=None) -> int:
+    """counts/tally: int64 (uint64 bit pattern) device tensors, accumulated."""
+    return lib().dels_prior_count(_ptr(tokens), _ptr(loss_mask), N, V, _ptr(counts), _ptr(tally), _ptr(workspace),
+                                  workspace_bytes, _stream(stream))
+
+
+def dels_prior_log(counts, V: int, lam: float, out_log_prior, workspace, workspace_bytes: int, stream=None) -> int:
+    return lib().dels_prior_log(_ptr(counts), V, float(lam), _ptr(out_log_prior), _ptr(workspace), workspace_bytes,
+                                _stream(stream))
+
+
+def dels_prior_estimate(tokens, loss_mask, N: int, V: int, lam: float, out_log_prior, out_counts, out_tally,
+                        workspace, workspace_bytes: int, stream=None) -> int:
+    return lib().dels_prior_estimate(_ptr(tokens), _ptr(loss_mask), N, V, float(lam), _ptr(out_log_prior),
+                                     _ptr(out_counts), _ptr(out_tally), _ptr(workspace), workspace_bytes,
+                                     _stream(stream))
+
+
+def estimate_prior(tokens: torch.Tensor, loss_mask: torch.Tensor, V: int, lam: float = 1.0, stream=None):
+    """Device unigram prior of a corpus: (log prior float32 [V], counts int64 [V],
+    tally int64 [2] = positions counted, loss-masked ids outside [0, V))."""
+    if tokens.dtype != torch.int32 or loss_mask.dtype not in (torch.uint8, torch.bool):
+        raise ValueError("tokens must be int32 and loss_mask uint8")
+    if tokens.numel() != loss_mask.numel():
+        raise ValueError("tokens and loss_mask must have the same length")
+    if not (tokens.is_contiguous() and loss_mask.is_contiguous()):
+        raise ValueError("tokens and loss_mask must be contiguous")
+    dev = tokens.device
+    nbytes = dels_prior_workspace_bytes(V)
+    if nbytes == 0:
+        raise DelsError(-2, "dels_prior_workspace_bytes")
+    ws = torch.zeros(nbytes, dtype=torch.uint8, device=dev)
+    out = torch.empty(V, dtype=torch.float32, device=dev)
+    counts = torch.empty(V, dtype=torch.int64, device=dev)
+    tally = torch.empty(2, dtype=torch.int64, device=dev)
+    _check(dels_prior_estimate(tokens, loss_mask.view(torch.uint8), tokens.numel(), V, lam, out, counts, tally, ws,
+                               nbytes, stream), "dels_prior_estimate")
+    return out, counts, tally
 
 
 def dels_profile_enable(on: bool) -> None:

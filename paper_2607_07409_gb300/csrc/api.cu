@@ -584,6 +584,147 @@ int dels_prior_from_counts(const int64_t* counts, int V, double lambda, float* o
   return DELS_OK;
 }
 
+// ------------------------------------------------ unigram prior (Appendix A)
+
+namespace {
+
+struct PriorWs {
+  unsigned long long* counts;   // [V]
+  unsigned long long* tally;    // [2]
+  unsigned long long* partials; // [kPriorMaxPartials]
+  unsigned* ticket;
+  unsigned long long* total;
+  size_t bytes;
+};
+
+PriorWs prior_ws_layout(void* ws, int V) {
+  PriorWs w{};
+  size_t off = kHeaderBytes;
+  w.counts = at<unsigned long long>(ws, off);
+  off = round_up(off + (size_t)V * 8, 256);
+  w.tally = at<unsigned long long>(ws, off);
+  off = round_up(off + 16, 256);
+  w.partials = at<unsigned long long>(ws, off);
+  off = round_up(off + (size_t)kPriorMaxPartials * 8, 256);
+  w.ticket = at<unsigned>(ws, off);
+  w.total = at<unsigned long long>(ws, off + 8);
+  w.bytes = round_up(off + 16, 256);
+  return w;
+}
+
+// Splits [0, N) into a scalar head, a vector range (tokens + head 16-byte
+// aligned, mask + head 4-byte aligned, a multiple of 512 positions) and a
+// scalar tail; pointers that cannot be aligned together get no vector range.
+void prior_split(const int32_t* tokens, const uint8_t* mask, long long N, long long& head, long long& nvec) {
+  head = (long long)((16 - (reinterpret_cast<uintptr_t>(tokens) & 15u)) & 15u) / 4;
+  nvec = 0;
+  if (head >= N || ((reinterpret_cast<uintptr_t>(mask) + (uintptr_t)head) & 3u) != 0) {
+    head = 0;
+    return;
+  }
+  nvec = (N - head) / 512 * 512;
+}
+
+int prior_count_impl(const int32_t* tokens, const uint8_t* loss_mask, long long N, int V, unsigned long long* counts,
+                     unsigned long long* tally, int* status, int sms, cudaStream_t s) {
+  if (N == 0) return DELS_OK;
+  PriorCountArgs a{};
+  a.tokens = tokens;
+  a.mask = loss_mask;
+  a.N = N;
+  prior_split(tokens, loss_mask, N, a.head, a.nvec);
+  a.V = V;
+  a.counts = counts;
+  a.tally = tally;
+  a.status = status;
+  PROF(DELS_KCLASS_PRIOR);
+  return launch_prior_count(a, sms, s) == cudaSuccess ? DELS_OK : DELS_ERR_CUDA;
+}
+
+}  // namespace
+
+size_t dels_prior_workspace_bytes(int V) {
+  if (V < 1) return 0;
+  return prior_ws_layout(nullptr, V).bytes;
+}
+
+int dels_prior_count(const int32_t* tokens, const uint8_t* loss_mask, int64_t N, int V, uint64_t* counts,
+                     uint64_t* tally, void* workspace, size_t workspace_bytes, dels_stream_t stream) {
+  if (N < 0 || V < 1) return DELS_ERR_BAD_SHAPE;
+  if (!workspace || workspace_bytes < kHeaderBytes) return DELS_ERR_WORKSPACE;
+  if (!counts || (N > 0 && (!tokens || !loss_mask))) return DELS_ERR_NULL_POINTER;
+  if ((reinterpret_cast<uintptr_t>(tokens) & 3u) || (reinterpret_cast<uintptr_t>(counts) & 7u) ||
+      (reinterpret_cast<uintptr_t>(tally) & 7u) || !aligned16(workspace))
+    return DELS_ERR_ALIGNMENT;
+  if (N == 0) return DELS_OK;
+  const int sms = device_sm_count();
+  if (sms <= 0) return DELS_ERR_CUDA;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  return prior_count_impl(tokens, loss_mask, N, V, reinterpret_cast<unsigned long long*>(counts),
+                          reinterpret_cast<unsigned long long*>(tally), at<int>(workspace, 0), sms, s);
+}
+
+int dels_prior_log(const uint64_t* counts, int V, double lambda, float* out_log_prior, void* workspace,
+                   size_t workspace_bytes, dels_stream_t stream) {
+  if (V < 1 || !(lambda > 0.0) || !std::isfinite(lambda)) return DELS_ERR_BAD_SHAPE;
+  if (!counts || !out_log_prior) return DELS_ERR_NULL_POINTER;
+  if (!workspace) return DELS_ERR_WORKSPACE;
+  if ((reinterpret_cast<uintptr_t>(counts) & 7u) || (reinterpret_cast<uintptr_t>(out_log_prior) & 3u) ||
+      !aligned16(workspace))
+    return DELS_ERR_ALIGNMENT;
+  PriorWs w = prior_ws_layout(workspace, V);
+  if (workspace_bytes < w.bytes) return DELS_ERR_WORKSPACE;
+  const int sms = device_sm_count();
+  if (sms <= 0) return DELS_ERR_CUDA;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  PriorLogArgs a{};
+  a.counts = reinterpret_cast<const unsigned long long*>(counts);
+  a.V = V;
+  a.lambda = lambda;
+  a.partials = w.partials;
+  a.ticket = w.ticket;
+  a.total = w.total;
+  a.out = out_log_prior;
+  PROF(DELS_KCLASS_PRIOR);
+  if (launch_prior_total(a, sms, s) != cudaSuccess) return DELS_ERR_CUDA;
+  if (launch_prior_log(a, sms, s) != cudaSuccess) return DELS_ERR_CUDA;
+  return DELS_OK;
+}
+
+int dels_prior_estimate(const int32_t* tokens, const uint8_t* loss_mask, int64_t N, int V, double lambda,
+                        float* out_log_prior, uint64_t* out_counts, uint64_t* out_tally, void* workspace,
+                        size_t workspace_bytes, dels_stream_t stream) {
+  if (N < 0 || V < 1 || !(lambda > 0.0) || !std::isfinite(lambda)) return DELS_ERR_BAD_SHAPE;
+  if (!out_log_prior || (N > 0 && (!tokens || !loss_mask))) return DELS_ERR_NULL_POINTER;
+  if (!workspace) return DELS_ERR_WORKSPACE;
+  if ((reinterpret_cast<uintptr_t>(tokens) & 3u) || (reinterpret_cast<uintptr_t>(out_log_prior) & 3u) ||
+      (reinterpret_cast<uintptr_t>(out_counts) & 7u) || (reinterpret_cast<uintptr_t>(out_tally) & 7u) ||
+      !aligned16(workspace))
+    return DELS_ERR_ALIGNMENT;
+  PriorWs w = prior_ws_layout(workspace, V);
+  if (workspace_bytes < w.bytes) return DELS_ERR_WORKSPACE;
+  const int sms = device_sm_count();
+  if (sms <= 0) return DELS_ERR_CUDA;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  // counts and tally start from zero (they sit next to each other)
+  const size_t zero_bytes = reinterpret_cast<uint8_t*>(w.tally + 2) - reinterpret_cast<uint8_t*>(w.counts);
+  if (cudaMemsetAsync(w.counts, 0, zero_bytes, s) != cudaSuccess) return DELS_ERR_CUDA;
+  const int rc = prior_count_impl(tokens, loss_mask, N, V, w.counts, w.tally, at<int>(workspace, 0), sms, s);
+  if (rc != DELS_OK) return rc;
+  PriorLogArgs a{};
+  a.counts = w.counts;
+  a.V = V;
+  a.lambda = lambda;
+  a.total = w.tally;   // tally[0] = the number of counted positions = sum_v c(v)
+  a.tally = w.tally;
+  a.out = out_log_prior;
+  a.counts_out = reinterpret_cast<unsigned long long*>(out_counts);
+  a.tally_out = reinterpret_cast<unsigned long long*>(out_tally);
+  PROF(DELS_KCLASS_PRIOR);
+  if (launch_prior_log(a, sms, s) != cudaSuccess) return DELS_ERR_CUDA;
+  return DELS_OK;
+}
+
 int dels_read_status(void* workspace, dels_stream_t stream, int32_t* out_status) {
   if (!workspace || !out_status) return DELS_ERR_NULL_POINTER;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);

@@ -263,4 +263,36 @@ bool encode_tmap_3d(CUtensorMap* m, const void* base, CUtensorMapDataType dt, in
                     uint64_t d1, uint64_t d2, uint64_t pitch1_bytes, uint64_t pitch2_bytes, uint32_t b0,
                     uint32_t b1, uint32_t b2, CUtensorMapSwizzle swz);
 
+// ---- unigram prior estimation (Appendix A) -----------------------------------
+constexpr int kPriorMaxPartials = 1024;    // CTAs of the two-level count sum
+
+struct PriorCountArgs {
+  const int32_t* tokens;          // [N]
+  const uint8_t* mask;            // [N], nonzero = loss-masked
+  long long N;
+  long long head;                 // positions before the vector range (0..3)
+  long long nvec;                 // vector-range length, a multiple of 512
+  int V;
+  unsigned long long* counts;     // [V], accumulated
+  unsigned long long* tally;      // [2] or null: masked in-range, masked out-of-range
+  int* status;
+};
+
+struct PriorLogArgs {
+  const unsigned long long* counts;   // [V]
+  int V;
+  double lambda;
+  unsigned long long* partials;       // [kPriorMaxPartials]
+  unsigned* ticket;
+  unsigned long long* total;          // sum_v counts[v] (written by k_prior_total, or the tally)
+  const unsigned long long* tally;    // [2] copied to tally_out when both are set
+  float* out;                         // [V] log prior
+  unsigned long long* counts_out;     // [V] or null
+  unsigned long long* tally_out;      // [2] or null
+};
+
+cudaError_t launch_prior_count(const PriorCountArgs& a, int sms, cudaStream_t s);
+cudaError_t launch_prior_total(const PriorLogArgs& a, int sms, cudaStream_t s);
+cudaError_t launch_prior_log(const PriorLogArgs& a, int sms, cudaStream_t s);
+
 }  // namespace dels

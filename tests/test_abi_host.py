@@ -131,3 +131,37 @@ def test_weighted_draft_rejects_bad_weights_before_enqueueing(dels):
                                              n)) == -2
     assert L.dels_draft_block_weighted(*args(ctypes.cast(good, ctypes.c_void_p), ctypes.cast(good, ctypes.c_void_p),
                                              0)) == -2
+
+
+def test_prior_entry_points_reject_bad_arguments_before_enqueueing(dels):
+    L = dels.lib()
+    V = 1000
+    need = dels.dels_prior_workspace_bytes(V)
+    assert need >= 256 + 8 * V + 16 + 8 * 1024
+    assert dels.dels_prior_workspace_bytes(0) == 0
+    ws = ctypes.create_string_buffer(need + 16)
+    wsp = (ctypes.addressof(ws) + 15) // 16 * 16
+    buf = ctypes.create_string_buffer(1 << 16)
+    p = (ctypes.addressof(buf) + 15) // 16 * 16
+    # dels_prior_count(tokens, mask, N, V, counts, tally, ws, bytes, stream)
+    assert L.dels_prior_count(p, p, -1, V, p, None, wsp, need, None) == -2
+    assert L.dels_prior_count(p, p, 10, 0, p, None, wsp, need, None) == -2
+    assert L.dels_prior_count(None, p, 10, V, p, None, wsp, need, None) == -1
+    assert L.dels_prior_count(p, None, 10, V, p, None, wsp, need, None) == -1
+    assert L.dels_prior_count(p, p, 10, V, None, None, wsp, need, None) == -1
+    assert L.dels_prior_count(p + 2, p, 10, V, p, None, wsp, need, None) == -4     # ids not 4-byte aligned
+    assert L.dels_prior_count(p, p, 10, V, p + 4, None, wsp, need, None) == -4     # counts not 8-byte aligned
+    assert L.dels_prior_count(p, p, 10, V, p, None, None, need, None) == -5
+    assert L.dels_prior_count(p, p, 10, V, p, None, wsp, 100, None) == -5
+    assert L.dels_prior_count(None, None, 0, V, p, None, wsp, need, None) == 0    # empty corpus: nothing to do
+    # dels_prior_log(counts, V, lambda, out, ws, bytes, stream)
+    for lam in (0.0, -1.0, float("inf"), float("nan")):
+        assert L.dels_prior_log(p, V, lam, p, wsp, need, None) == -2
+    assert L.dels_prior_log(None, V, 1.0, p, wsp, need, None) == -1
+    assert L.dels_prior_log(p, V, 1.0, None, wsp, need, None) == -1
+    assert L.dels_prior_log(p, V, 1.0, p, wsp, need - 1, None) == -5
+    # dels_prior_estimate(tokens, mask, N, V, lambda, out, counts, tally, ws, bytes, stream)
+    assert L.dels_prior_estimate(p, p, 10, V, 0.0, p, None, None, wsp, need, None) == -2
+    assert L.dels_prior_estimate(p, p, 10, V, 1.0, None, None, None, wsp, need, None) == -1
+    assert L.dels_prior_estimate(p, p, 10, V, 1.0, p, p + 4, None, wsp, need, None) == -4
+    assert L.dels_prior_estimate(p, p, 10, V, 1.0, p, None, None, wsp, need - 256, None) == -5
