@@ -557,7 +557,7 @@ def run_prior(args):
     w = synth.WORKLOADS[WORKLOAD]
     V, N = w.V, synth.CORPUS_TOKENS
     tok, mask = synth.make_corpus(V, N, replicas.replica_seed(w.seed, rank), device=dev)
-    nbytes = dels.dels_prior_workspace_bytes(V)
+    nbytes = dels.dels_prior_workspace_bytes(V, N)
     ws = torch.zeros(nbytes, dtype=torch.uint8, device=dev)
     out = torch.empty(V, dtype=torch.float32, device=dev)
     counts = torch.empty(V, dtype=torch.int64, device=dev)

@@ -304,7 +304,7 @@ int dels_prior_from_counts(const int64_t* counts, int V, double lambda, float* o
  * outside [0, V) is not counted: it is tallied separately and sets
  * DELS_STATUS_BAD_TOKEN in the workspace status word.
  */
-size_t dels_prior_workspace_bytes(int V);
+size_t dels_prior_workspace_bytes(int V, int64_t N);
 
 /*
  * Adds one corpus piece's loss-masked token counts to `counts`:
@@ -312,8 +312,11 @@ size_t dels_prior_workspace_bytes(int V);
  * counts [device] [V] uint64, accumulated (zero it before the first piece);
  * tally  [device] [2] uint64 or NULL, accumulated: tally[0] += positions
  *        counted, tally[1] += loss-masked positions with an id outside [0, V).
- * workspace [device]: at least 256 bytes (only its status word is used) or
- * the dels_prior_workspace_bytes(V) buffer of the other prior calls.
+ * workspace [device] >= dels_prior_workspace_bytes(V, N) (a workspace sized
+ * for the longest piece serves every piece).
+ * Large vocabularies count long pieces in two steps: the first positions
+ * exactly, then the rest with the ids that are most frequent in `counts` so
+ * far held on chip; the result is the exact count either way.
  * Limits: N >= 0 (N = 0 enqueues nothing), 1 <= V < 2^31.
  */
 int dels_prior_count(const int32_t* tokens, const uint8_t* loss_mask, int64_t N, int V, uint64_t* counts,
@@ -324,7 +327,7 @@ int dels_prior_count(const int32_t* tokens, const uint8_t* loss_mask, int64_t N,
  *   out_log_prior[v] = log(counts[v] + lambda) - log(sum_u counts[u] + V * lambda)
  * evaluated in float64 and stored as float32 (within one float32 rounding of
  * the exact value). counts [device] [V] uint64; out_log_prior [device] [V]
- * float32; lambda > 0 and finite; workspace >= dels_prior_workspace_bytes(V).
+ * float32; lambda > 0 and finite; workspace >= dels_prior_workspace_bytes(V, 0).
  */
 int dels_prior_log(const uint64_t* counts, int V, double lambda, float* out_log_prior, void* workspace,
                    size_t workspace_bytes, dels_stream_t stream);
@@ -333,7 +336,7 @@ int dels_prior_log(const uint64_t* counts, int V, double lambda, float* out_log_
  * Both steps for a corpus held in device memory: zeroes counts kept in the
  * workspace, counts, and writes l_P. out_counts [device] [V] uint64 and
  * out_tally [device] [2] uint64 (as for dels_prior_count) are optional copies.
- * workspace >= dels_prior_workspace_bytes(V).
+ * workspace >= dels_prior_workspace_bytes(V, N).
  */
 int dels_prior_estimate(const int32_t* tokens, const uint8_t* loss_mask, int64_t N, int V, double lambda,
                         float* out_log_prior, uint64_t* out_counts, uint64_t* out_tally, void* workspace,

@@ -75,7 +75,7 @@ _SIGS = {
     "dels_verify_block": (_i, [_vp, _vp, _i, _i, _i, _i, _vp, _vp, _vp, _vp, _sz, _vp]),
     "dels_read_status": (_i, [_vp, _vp, ctypes.POINTER(ctypes.c_int32)]),
     "dels_prior_from_counts": (_i, [_vp, _i, _d, _vp]),
-    "dels_prior_workspace_bytes": (_sz, [_i]),
+    "dels_prior_workspace_bytes": (_sz, [_i, ctypes.c_int64]),
     "dels_prior_count": (_i, [_vp, _vp, ctypes.c_int64, _i, _vp, _vp, _vp, _sz, _vp]),
     "dels_prior_log": (_i, [_vp, _i, _d, _vp, _vp, _sz, _vp]),
     "dels_prior_estimate": (_i, [_vp, _vp, ctypes.c_int64, _i, _d, _vp, _vp, _vp, _vp, _sz, _vp]),
@@ -274,8 +274,8 @@ def dels_prior_from_counts(counts: torch.Tensor, lam: float = 1.0) -> torch.Tens
     return out
 
 
-def dels_prior_workspace_bytes(V: int) -> int:
-    return lib().dels_prior_workspace_bytes(V)
+def dels_prior_workspace_bytes(V: int, N: int) -> int:
+    return lib().dels_prior_workspace_bytes(V, N)
 
 
 def dels_prior_count(tokens, loss_mask, N: int, V: int, counts, tally, workspace, workspace_bytes: int,
@@ -307,7 +307,7 @@ def estimate_prior(tokens: torch.Tensor, loss_mask: torch.Tensor, V: int, lam: f
     if not (tokens.is_contiguous() and loss_mask.is_contiguous()):
         raise ValueError("tokens and loss_mask must be contiguous")
     dev = tokens.device
-    nbytes = dels_prior_workspace_bytes(V)
+    nbytes = dels_prior_workspace_bytes(V, tokens.numel())
     if nbytes == 0:
         raise DelsError(-2, "dels_prior_workspace_bytes")
     ws = torch.zeros(nbytes, dtype=torch.uint8, device=dev)

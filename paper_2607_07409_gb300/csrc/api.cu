@@ -589,15 +589,22 @@ int dels_prior_from_counts(const int64_t* counts, int V, double lambda, float* o
 namespace {
 
 struct PriorWs {
-  unsigned long long* counts;   // [V]
-  unsigned long long* tally;    // [2]
-  unsigned long long* partials; // [kPriorMaxPartials]
+  unsigned long long* counts;   // [V] (dels_prior_estimate)
+  unsigned long long* tally;    // [2] (dels_prior_estimate)
+  unsigned long long* partials; // [kPriorMaxPartials] (sum of the counts)
   unsigned* ticket;
   unsigned long long* total;
+  // hot/cold counting (when the plan uses it)
+  uint32_t* entries;            // [nent]
+  int32_t* slot_id;             // [K]
+  unsigned* n_hot;
+  unsigned* hot_partials;       // [ctas][K]
+  unsigned* cold_len;           // [ctas]
+  int32_t* cold_buf;            // [ctas][cold_cap]
   size_t bytes;
 };
 
-PriorWs prior_ws_layout(void* ws, int V) {
+PriorWs prior_ws_layout(void* ws, int V, const PriorPlan& p) {
   PriorWs w{};
   size_t off = kHeaderBytes;
   w.counts = at<unsigned long long>(ws, off);
@@ -608,60 +615,135 @@ PriorWs prior_ws_layout(void* ws, int V) {
   off = round_up(off + (size_t)kPriorMaxPartials * 8, 256);
   w.ticket = at<unsigned>(ws, off);
   w.total = at<unsigned long long>(ws, off + 8);
-  w.bytes = round_up(off + 16, 256);
+  off = round_up(off + 16, 256);
+  if (p.use_hot) {
+    w.entries = at<uint32_t>(ws, off);
+    off = round_up(off + (size_t)p.nent * 4, 256);
+    w.slot_id = at<int32_t>(ws, off);
+    off = round_up(off + (size_t)p.K * 4, 256);
+    w.n_hot = at<unsigned>(ws, off);
+    off = round_up(off + 4, 256);
+    w.hot_partials = at<unsigned>(ws, off);
+    off = round_up(off + (size_t)p.ctas * p.K * 4, 256);
+    w.cold_len = at<unsigned>(ws, off);
+    off = round_up(off + (size_t)p.ctas * 4, 256);
+    w.cold_buf = at<int32_t>(ws, off);
+    off = round_up(off + (size_t)p.ctas * p.cold_cap * 4, 256);
+  }
+  w.bytes = off;
   return w;
 }
 
 // Splits [0, N) into a scalar head, a vector range (tokens + head 16-byte
 // aligned, mask + head 4-byte aligned, a multiple of 512 positions) and a
 // scalar tail; pointers that cannot be aligned together get no vector range.
-void prior_split(const int32_t* tokens, const uint8_t* mask, long long N, long long& head, long long& nvec) {
-  head = (long long)((16 - (reinterpret_cast<uintptr_t>(tokens) & 15u)) & 15u) / 4;
-  nvec = 0;
-  if (head >= N || ((reinterpret_cast<uintptr_t>(mask) + (uintptr_t)head) & 3u) != 0) {
-    head = 0;
-    return;
+PriorRange prior_range(const int32_t* tokens, const uint8_t* mask, long long begin, long long n) {
+  PriorRange r{};
+  r.tokens = tokens + begin;
+  r.mask = mask + begin;
+  r.n = n;
+  r.head = (long long)((16 - (reinterpret_cast<uintptr_t>(r.tokens) & 15u)) & 15u) / 4;
+  r.nvec = 0;
+  if (r.head >= n || ((reinterpret_cast<uintptr_t>(r.mask) + (uintptr_t)r.head) & 3u) != 0) {
+    r.head = 0;
+    return r;
   }
-  nvec = (N - head) / 512 * 512;
+  r.nvec = (n - r.head) / 512 * 512;
+  return r;
 }
 
+// Adds the loss-masked counts of positions [0, N) to `counts` (see the
+// kernels' file for the two counting schemes).
 int prior_count_impl(const int32_t* tokens, const uint8_t* loss_mask, long long N, int V, unsigned long long* counts,
-                     unsigned long long* tally, int* status, int sms, cudaStream_t s) {
+                     unsigned long long* tally, int* status, const PriorPlan& p, const PriorWs& w, int sms,
+                     cudaStream_t s) {
   if (N == 0) return DELS_OK;
-  PriorCountArgs a{};
-  a.tokens = tokens;
-  a.mask = loss_mask;
-  a.N = N;
-  prior_split(tokens, loss_mask, N, a.head, a.nvec);
-  a.V = V;
-  a.counts = counts;
-  a.tally = tally;
-  a.status = status;
-  PROF(DELS_KCLASS_PRIOR);
-  return launch_prior_count(a, sms, s) == cudaSuccess ? DELS_OK : DELS_ERR_CUDA;
+  PriorSliceArgs sa{};
+  sa.V = V;
+  sa.slices = p.slices;
+  sa.slice = p.slice;
+  sa.counts = counts;
+  sa.tally = tally;
+  sa.status = status;
+  auto slices_over = [&](long long begin, long long n, int max_members) {
+    for (long long b = begin; b < begin + n; b += kPriorChunk) {
+      sa.range = prior_range(tokens, loss_mask, b, std::min(kPriorChunk, begin + n - b));
+      if (launch_prior_slices(sa, false, p.slice_smem, max_members, sms, s) != cudaSuccess) return false;
+    }
+    return true;
+  };
+  if (!p.use_hot) return slices_over(0, N, 1 << 30) ? DELS_OK : DELS_ERR_CUDA;
+  // a prefix, exactly, then the hot set from the counts so far
+  if (!slices_over(0, p.prefix, 24)) return DELS_ERR_CUDA;
+  PriorSelectArgs se{};
+  se.counts = counts;
+  se.V = V;
+  se.K = p.K;
+  se.nent = p.nent;
+  se.cache_bytes = p.select_cache;
+  se.entries = w.entries;
+  se.slot_id = w.slot_id;
+  se.n_hot = w.n_hot;
+  if (launch_prior_select(se, s) != cudaSuccess) return DELS_ERR_CUDA;
+  PriorHotArgs ha{};
+  ha.V = V;
+  ha.K = p.K;
+  ha.nent = p.nent;
+  ha.ctas = p.ctas;
+  ha.entries = w.entries;
+  ha.slot_id = w.slot_id;
+  ha.n_hot = w.n_hot;
+  ha.partials = w.hot_partials;
+  ha.cold_buf = w.cold_buf;
+  ha.cold_len = w.cold_len;
+  ha.cold_cap = p.cold_cap;
+  ha.counts = counts;
+  ha.tally = tally;
+  ha.status = status;
+  PriorSliceArgs ca = sa;
+  ca.tally = nullptr;
+  ca.cold_buf = w.cold_buf;
+  ca.cold_len = w.cold_len;
+  ca.cold_regions = p.ctas;
+  ca.cold_cap = p.cold_cap;
+  for (long long b = p.prefix; b < N; b += kPriorChunk) {
+    ha.range = prior_range(tokens, loss_mask, b, std::min(kPriorChunk, N - b));
+    if (launch_prior_hot(ha, p.hot_smem, s) != cudaSuccess) return DELS_ERR_CUDA;
+    if (launch_prior_slices(ca, true, p.slice_smem, 24, sms, s) != cudaSuccess) return DELS_ERR_CUDA;
+  }
+  return DELS_OK;
 }
 
 }  // namespace
 
-size_t dels_prior_workspace_bytes(int V) {
-  if (V < 1) return 0;
-  return prior_ws_layout(nullptr, V).bytes;
+size_t dels_prior_workspace_bytes(int V, int64_t N) {
+  if (V < 1 || N < 0) return 0;
+  const int sms = device_sm_count();
+  const PriorPlan p = plan_prior(V, N, sms);
+  if (!p.ok) return 0;
+  return prior_ws_layout(nullptr, V, p).bytes;
 }
 
 int dels_prior_count(const int32_t* tokens, const uint8_t* loss_mask, int64_t N, int V, uint64_t* counts,
                      uint64_t* tally, void* workspace, size_t workspace_bytes, dels_stream_t stream) {
   if (N < 0 || V < 1) return DELS_ERR_BAD_SHAPE;
-  if (!workspace || workspace_bytes < kHeaderBytes) return DELS_ERR_WORKSPACE;
+  if (!workspace) return DELS_ERR_WORKSPACE;
   if (!counts || (N > 0 && (!tokens || !loss_mask))) return DELS_ERR_NULL_POINTER;
   if ((reinterpret_cast<uintptr_t>(tokens) & 3u) || (reinterpret_cast<uintptr_t>(counts) & 7u) ||
       (reinterpret_cast<uintptr_t>(tally) & 7u) || !aligned16(workspace))
     return DELS_ERR_ALIGNMENT;
+  if (workspace_bytes < (size_t)kHeaderBytes) return DELS_ERR_WORKSPACE;
   if (N == 0) return DELS_OK;
   const int sms = device_sm_count();
   if (sms <= 0) return DELS_ERR_CUDA;
+  const PriorPlan p = plan_prior(V, N, sms);
+  if (!p.ok) return DELS_ERR_CUDA;
+  const PriorWs w = prior_ws_layout(workspace, V, p);
+  if (workspace_bytes < w.bytes) return DELS_ERR_WORKSPACE;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  PROF(DELS_KCLASS_PRIOR);
   return prior_count_impl(tokens, loss_mask, N, V, reinterpret_cast<unsigned long long*>(counts),
-                          reinterpret_cast<unsigned long long*>(tally), at<int>(workspace, 0), sms, s);
+                          reinterpret_cast<unsigned long long*>(tally), at<int>(workspace, 0), p, w, sms, s);
 }
 
 int dels_prior_log(const uint64_t* counts, int V, double lambda, float* out_log_prior, void* workspace,
@@ -672,10 +754,13 @@ int dels_prior_log(const uint64_t* counts, int V, double lambda, float* out_log_
   if ((reinterpret_cast<uintptr_t>(counts) & 7u) || (reinterpret_cast<uintptr_t>(out_log_prior) & 3u) ||
       !aligned16(workspace))
     return DELS_ERR_ALIGNMENT;
-  PriorWs w = prior_ws_layout(workspace, V);
-  if (workspace_bytes < w.bytes) return DELS_ERR_WORKSPACE;
+  if (workspace_bytes < (size_t)kHeaderBytes + (size_t)V * 8) return DELS_ERR_WORKSPACE;
   const int sms = device_sm_count();
   if (sms <= 0) return DELS_ERR_CUDA;
+  const PriorPlan p = plan_prior(V, 0, sms);
+  if (!p.ok) return DELS_ERR_CUDA;
+  const PriorWs w = prior_ws_layout(workspace, V, p);
+  if (workspace_bytes < w.bytes) return DELS_ERR_WORKSPACE;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   PriorLogArgs a{};
   a.counts = reinterpret_cast<const unsigned long long*>(counts);
@@ -701,15 +786,19 @@ int dels_prior_estimate(const int32_t* tokens, const uint8_t* loss_mask, int64_t
       (reinterpret_cast<uintptr_t>(out_counts) & 7u) || (reinterpret_cast<uintptr_t>(out_tally) & 7u) ||
       !aligned16(workspace))
     return DELS_ERR_ALIGNMENT;
-  PriorWs w = prior_ws_layout(workspace, V);
-  if (workspace_bytes < w.bytes) return DELS_ERR_WORKSPACE;
+  if (workspace_bytes < (size_t)kHeaderBytes + (size_t)V * 8) return DELS_ERR_WORKSPACE;
   const int sms = device_sm_count();
   if (sms <= 0) return DELS_ERR_CUDA;
+  const PriorPlan p = plan_prior(V, N, sms);
+  if (!p.ok) return DELS_ERR_CUDA;
+  const PriorWs w = prior_ws_layout(workspace, V, p);
+  if (workspace_bytes < w.bytes) return DELS_ERR_WORKSPACE;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  PROF(DELS_KCLASS_PRIOR);
   // counts and tally start from zero (they sit next to each other)
   const size_t zero_bytes = reinterpret_cast<uint8_t*>(w.tally + 2) - reinterpret_cast<uint8_t*>(w.counts);
   if (cudaMemsetAsync(w.counts, 0, zero_bytes, s) != cudaSuccess) return DELS_ERR_CUDA;
-  const int rc = prior_count_impl(tokens, loss_mask, N, V, w.counts, w.tally, at<int>(workspace, 0), sms, s);
+  const int rc = prior_count_impl(tokens, loss_mask, N, V, w.counts, w.tally, at<int>(workspace, 0), p, w, sms, s);
   if (rc != DELS_OK) return rc;
   PriorLogArgs a{};
   a.counts = w.counts;
@@ -720,7 +809,6 @@ int dels_prior_estimate(const int32_t* tokens, const uint8_t* loss_mask, int64_t
   a.out = out_log_prior;
   a.counts_out = reinterpret_cast<unsigned long long*>(out_counts);
   a.tally_out = reinterpret_cast<unsigned long long*>(out_tally);
-  PROF(DELS_KCLASS_PRIOR);
   if (launch_prior_log(a, sms, s) != cudaSuccess) return DELS_ERR_CUDA;
   return DELS_OK;
 }

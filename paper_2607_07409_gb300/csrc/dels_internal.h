@@ -264,17 +264,61 @@ bool encode_tmap_3d(CUtensorMap* m, const void* base, CUtensorMapDataType dt, in
                     uint32_t b1, uint32_t b2, CUtensorMapSwizzle swz);
 
 // ---- unigram prior estimation (Appendix A) -----------------------------------
-constexpr int kPriorMaxPartials = 1024;    // CTAs of the two-level count sum
+constexpr int kPriorMaxPartials = 1024;            // CTAs of the two-level count sum
+constexpr long long kPriorHotMinN = 1ll << 24;     // shorter ranges: slice histograms only
+constexpr long long kPriorChunk = 1ll << 36;       // positions per hot pass (per-CTA bins stay < 2^32)
 
-struct PriorCountArgs {
-  const int32_t* tokens;          // [N]
-  const uint8_t* mask;            // [N], nonzero = loss-masked
-  long long N;
-  long long head;                 // positions before the vector range (0..3)
-  long long nvec;                 // vector-range length, a multiple of 512
+// Positions [0, n) of tokens / mask; [head, head + nvec) takes the vector
+// path (tokens + head 16-byte aligned, mask + head 4-byte aligned, nvec a
+// multiple of 512).
+struct PriorRange {
+  const int32_t* tokens;
+  const uint8_t* mask;        // nonzero = loss-masked
+  long long n;
+  long long head;
+  long long nvec;
+};
+
+struct PriorSliceArgs {
+  PriorRange range;
   int V;
-  unsigned long long* counts;     // [V], accumulated
-  unsigned long long* tally;      // [2] or null: masked in-range, masked out-of-range
+  int slices;                       // P
+  int slice;                        // ids per slice (bins per CTA)
+  unsigned long long* counts;       // [V], accumulated
+  unsigned long long* tally;        // [2] or null
+  int* status;
+  const int32_t* cold_buf;          // cold source: [cold_regions][cold_cap]
+  const unsigned* cold_len;         // [cold_regions]
+  long long cold_regions;
+  long long cold_cap;
+};
+
+struct PriorSelectArgs {
+  const unsigned long long* counts;   // [V]
+  int V;
+  int K;                              // hot slots
+  int nent;                           // remap words: ceil(V / 16)
+  size_t cache_bytes;                 // nent * 16 byte copy of the counts in smem, or 0
+  uint32_t* entries;                  // [nent]
+  int32_t* slot_id;                   // [K]
+  unsigned* n_hot;
+};
+
+struct PriorHotArgs {
+  PriorRange range;
+  int V;
+  int K;
+  int nent;
+  int ctas;
+  const uint32_t* entries;
+  const int32_t* slot_id;
+  const unsigned* n_hot;
+  unsigned* partials;                 // [ctas][K]
+  int32_t* cold_buf;                  // [ctas][cold_cap]
+  unsigned* cold_len;                 // [ctas]
+  long long cold_cap;
+  unsigned long long* counts;
+  unsigned long long* tally;
   int* status;
 };
 
@@ -291,7 +335,24 @@ struct PriorLogArgs {
   unsigned long long* tally_out;      // [2] or null
 };
 
-cudaError_t launch_prior_count(const PriorCountArgs& a, int sms, cudaStream_t s);
+// How a count call runs for (V, N) on this device.
+struct PriorPlan {
+  bool ok;
+  int slices, slice;          // slice histograms: P slices of `slice` ids
+  size_t slice_smem;
+  bool use_hot;               // hot/cold path
+  int nent, K;                // remap words, hot slots
+  size_t hot_smem, select_cache;
+  int ctas;                   // CTAs of the hot pass (one per SM)
+  long long prefix;           // positions counted by the slices before the hot set is chosen
+  long long cold_cap;         // cold-buffer entries per CTA
+};
+
+PriorPlan plan_prior(int V, long long N, int sms);
+cudaError_t launch_prior_slices(const PriorSliceArgs& a, bool cold, size_t smem, int max_members, int sms,
+                                cudaStream_t s);
+cudaError_t launch_prior_select(const PriorSelectArgs& a, cudaStream_t s);
+cudaError_t launch_prior_hot(const PriorHotArgs& a, size_t smem, cudaStream_t s);
 cudaError_t launch_prior_total(const PriorLogArgs& a, int sms, cudaStream_t s);
 cudaError_t launch_prior_log(const PriorLogArgs& a, int sms, cudaStream_t s);
 

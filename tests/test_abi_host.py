@@ -136,9 +136,9 @@ def test_weighted_draft_rejects_bad_weights_before_enqueueing(dels):
 def test_prior_entry_points_reject_bad_arguments_before_enqueueing(dels):
     L = dels.lib()
     V = 1000
-    need = dels.dels_prior_workspace_bytes(V)
-    assert need >= 256 + 8 * V + 16 + 8 * 1024
-    assert dels.dels_prior_workspace_bytes(0) == 0
+    assert dels.dels_prior_workspace_bytes(0, 10) == 0
+    assert dels.dels_prior_workspace_bytes(V, -1) == 0
+    need = 1 << 16                                  # enough for every check below to come first
     ws = ctypes.create_string_buffer(need + 16)
     wsp = (ctypes.addressof(ws) + 15) // 16 * 16
     buf = ctypes.create_string_buffer(1 << 16)
@@ -159,9 +159,9 @@ def test_prior_entry_points_reject_bad_arguments_before_enqueueing(dels):
         assert L.dels_prior_log(p, V, lam, p, wsp, need, None) == -2
     assert L.dels_prior_log(None, V, 1.0, p, wsp, need, None) == -1
     assert L.dels_prior_log(p, V, 1.0, None, wsp, need, None) == -1
-    assert L.dels_prior_log(p, V, 1.0, p, wsp, need - 1, None) == -5
+    assert L.dels_prior_log(p, V, 1.0, p, wsp, 256 + 8 * V - 1, None) == -5
     # dels_prior_estimate(tokens, mask, N, V, lambda, out, counts, tally, ws, bytes, stream)
     assert L.dels_prior_estimate(p, p, 10, V, 0.0, p, None, None, wsp, need, None) == -2
     assert L.dels_prior_estimate(p, p, 10, V, 1.0, None, None, None, wsp, need, None) == -1
     assert L.dels_prior_estimate(p, p, 10, V, 1.0, p, p + 4, None, wsp, need, None) == -4
-    assert L.dels_prior_estimate(p, p, 10, V, 1.0, p, None, None, wsp, need - 256, None) == -5
+    assert L.dels_prior_estimate(p, p, 10, V, 1.0, p, None, None, wsp, 256 + 8 * V - 1, None) == -5

@@ -17,8 +17,8 @@ pytestmark = pytest.mark.gpu
 DEV = "cuda:0"
 
 
-def _ws(V):
-    n = dels.dels_prior_workspace_bytes(V)
+def _ws(V, N):
+    n = dels.dels_prior_workspace_bytes(V, N)
     assert n > 0
     return torch.zeros(n, dtype=torch.uint8, device=DEV), n
 
@@ -66,7 +66,7 @@ def test_out_of_range_ids_are_tallied_and_flagged():
     tok, mask = _corpus(V, N, 5, bad=37)
     c_ref, n_in, n_out = oracle.count_masked_tokens(tok.numpy(), mask.numpy(), V)
     assert n_out == 37
-    ws, nbytes = _ws(V)
+    ws, nbytes = _ws(V, N)
     out = torch.empty(V, dtype=torch.float32, device=DEV)
     counts = torch.empty(V, dtype=torch.int64, device=DEV)
     tally = torch.empty(2, dtype=torch.int64, device=DEV)
@@ -87,7 +87,7 @@ def test_unaligned_corpus_pieces(tok_off, mask_off):
     n = N - 5
     c_ref, n_in, n_out = oracle.count_masked_tokens(tok[tok_off:tok_off + n].numpy(),
                                                     mask[mask_off:mask_off + n].numpy(), V)
-    ws, nbytes = _ws(V)
+    ws, nbytes = _ws(V, n)
     counts = torch.zeros(V, dtype=torch.int64, device=DEV)
     tally = torch.zeros(2, dtype=torch.int64, device=DEV)
     r = dels.dels_prior_count(t_dev[tok_off:], m_dev[mask_off:], n, V, counts, tally, ws, nbytes)
@@ -101,7 +101,7 @@ def test_pieces_accumulate_then_log_equals_one_call():
     V, N = 151936, 300000
     tok, mask = _corpus(V, N, 7)
     t_dev, m_dev = tok.to(DEV), mask.to(DEV)
-    ws, nbytes = _ws(V)
+    ws, nbytes = _ws(V, N)
     counts = torch.zeros(V, dtype=torch.int64, device=DEV)
     tally = torch.zeros(2, dtype=torch.int64, device=DEV)
     cuts = [0, 12345, 12346, 200000, N]
@@ -155,3 +155,55 @@ def test_full_corpus_counts_match_oracle():
     np.testing.assert_array_equal(c, c_ref)
     assert tally.tolist() == [n_in, n_out]
     _check_log_prior(out, c_ref, 1.0)
+
+
+# ------------------------------------------------------------- the hot/cold path
+# (large vocabularies over long ranges: a prefix counted exactly, the most
+# frequent ids so far on chip, the others through per-CTA cold buffers)
+
+HOT_N = (1 << 24) + 1234
+
+
+def test_hot_cold_path_matches_oracle_with_bad_ids():
+    V = 151936
+    tok, mask = _corpus(V, HOT_N, 8, bad=101)
+    c_ref, n_in, n_out = oracle.count_masked_tokens(tok.numpy(), mask.numpy(), V)
+    ws, nbytes = _ws(V, HOT_N)
+    out = torch.empty(V, dtype=torch.float32, device=DEV)
+    counts = torch.empty(V, dtype=torch.int64, device=DEV)
+    tally = torch.empty(2, dtype=torch.int64, device=DEV)
+    assert dels.dels_prior_estimate(tok.to(DEV), mask.to(DEV), HOT_N, V, 1.0, out, counts, tally, ws, nbytes) == 0
+    assert dels.dels_read_status(ws) == dels.DELS_STATUS_BAD_TOKEN
+    np.testing.assert_array_equal(counts.cpu().numpy(), c_ref)
+    assert tally.cpu().tolist() == [n_in, n_out] and n_out == 101
+    _check_log_prior(out, c_ref, 1.0)
+
+
+def test_hot_cold_path_when_the_prefix_misleads():
+    """The prefix holds one id only, the rest is uniform over V: almost every
+    later position is cold and the cold buffers overflow into direct adds."""
+    V = 151936
+    g = torch.Generator().manual_seed(9)
+    tok = torch.randint(0, V, (HOT_N,), generator=g, dtype=torch.int32)
+    tok[: 1 << 23] = 77
+    mask = (torch.rand(HOT_N, generator=g) < 0.9).to(torch.uint8)
+    c_ref, n_in, n_out = oracle.count_masked_tokens(tok.numpy(), mask.numpy(), V)
+    out, c, tally = _estimate(tok.to(DEV), mask.to(DEV), V)
+    np.testing.assert_array_equal(c, c_ref)
+    assert tally.tolist() == [n_in, n_out]
+
+
+def test_hot_cold_pieces_on_top_of_earlier_counts():
+    """A second long piece chooses its hot set from counts that already hold the first."""
+    V = 151936
+    tok, mask = _corpus(V, 2 * HOT_N, 10)
+    t_dev, m_dev = tok.to(DEV), mask.to(DEV)
+    ws, nbytes = _ws(V, HOT_N)
+    counts = torch.zeros(V, dtype=torch.int64, device=DEV)
+    tally = torch.zeros(2, dtype=torch.int64, device=DEV)
+    for a in (0, HOT_N):
+        assert dels.dels_prior_count(t_dev[a:], m_dev[a:], HOT_N, V, counts, tally, ws, nbytes) == 0
+    torch.cuda.synchronize()
+    c_ref, n_in, _ = oracle.count_masked_tokens(tok.numpy(), mask.numpy(), V)
+    np.testing.assert_array_equal(counts.cpu().numpy(), c_ref)
+    assert tally.cpu().tolist() == [n_in, 0]
