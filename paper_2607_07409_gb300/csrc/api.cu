@@ -594,13 +594,14 @@ struct PriorWs {
   unsigned long long* partials; // [kPriorMaxPartials] (sum of the counts)
   unsigned* ticket;
   unsigned long long* total;
-  // hot/cold counting (when the plan uses it)
+  // hot ids on chip (when the plan uses them)
+  unsigned* hist;               // [kPriorHistBuckets]
+  unsigned* cta_total;          // [select CTAs]
+  unsigned* n_hot;
   uint32_t* entries;            // [nent]
   int32_t* slot_id;             // [K]
-  unsigned* n_hot;
-  unsigned* hot_partials;       // [ctas][K]
-  unsigned* cold_len;           // [ctas]
-  int32_t* cold_buf;            // [ctas][cold_cap]
+  int32_t* stage;               // [nent * 15]
+  unsigned* hot_partials;       // [ctas][(K + 1) / 2]
   size_t bytes;
 };
 
@@ -617,18 +618,20 @@ PriorWs prior_ws_layout(void* ws, int V, const PriorPlan& p) {
   w.total = at<unsigned long long>(ws, off + 8);
   off = round_up(off + 16, 256);
   if (p.use_hot) {
+    w.hist = at<unsigned>(ws, off);
+    off = round_up(off + (size_t)kPriorHistBuckets * 4, 256);
+    w.cta_total = at<unsigned>(ws, off);
+    off = round_up(off + (size_t)p.select_ctas * 4, 256);
+    w.n_hot = at<unsigned>(ws, off);
+    off = round_up(off + 4, 256);
     w.entries = at<uint32_t>(ws, off);
     off = round_up(off + (size_t)p.nent * 4, 256);
     w.slot_id = at<int32_t>(ws, off);
     off = round_up(off + (size_t)p.K * 4, 256);
-    w.n_hot = at<unsigned>(ws, off);
-    off = round_up(off + 4, 256);
+    w.stage = at<int32_t>(ws, off);
+    off = round_up(off + (size_t)p.nent * 15 * 4, 256);
     w.hot_partials = at<unsigned>(ws, off);
-    off = round_up(off + (size_t)p.ctas * p.K * 4, 256);
-    w.cold_len = at<unsigned>(ws, off);
-    off = round_up(off + (size_t)p.ctas * 4, 256);
-    w.cold_buf = at<int32_t>(ws, off);
-    off = round_up(off + (size_t)p.ctas * p.cold_cap * 4, 256);
+    off = round_up(off + (size_t)p.ctas * ((p.K + 1) / 2) * 4, 256);
   }
   w.bytes = off;
   return w;
@@ -668,7 +671,7 @@ int prior_count_impl(const int32_t* tokens, const uint8_t* loss_mask, long long 
   auto slices_over = [&](long long begin, long long n, int max_members) {
     for (long long b = begin; b < begin + n; b += kPriorChunk) {
       sa.range = prior_range(tokens, loss_mask, b, std::min(kPriorChunk, begin + n - b));
-      if (launch_prior_slices(sa, false, p.slice_smem, max_members, sms, s) != cudaSuccess) return false;
+      if (launch_prior_slices(sa, p.slice_smem, max_members, sms, s) != cudaSuccess) return false;
     }
     return true;
   };
@@ -680,11 +683,13 @@ int prior_count_impl(const int32_t* tokens, const uint8_t* loss_mask, long long 
   se.V = V;
   se.K = p.K;
   se.nent = p.nent;
-  se.cache_bytes = p.select_cache;
+  se.hist = w.hist;
   se.entries = w.entries;
+  se.stage = w.stage;
+  se.cta_total = w.cta_total;
   se.slot_id = w.slot_id;
   se.n_hot = w.n_hot;
-  if (launch_prior_select(se, s) != cudaSuccess) return DELS_ERR_CUDA;
+  if (launch_prior_select(se, p.select_ctas, s) != cudaSuccess) return DELS_ERR_CUDA;
   PriorHotArgs ha{};
   ha.V = V;
   ha.K = p.K;
@@ -694,22 +699,12 @@ int prior_count_impl(const int32_t* tokens, const uint8_t* loss_mask, long long 
   ha.slot_id = w.slot_id;
   ha.n_hot = w.n_hot;
   ha.partials = w.hot_partials;
-  ha.cold_buf = w.cold_buf;
-  ha.cold_len = w.cold_len;
-  ha.cold_cap = p.cold_cap;
   ha.counts = counts;
   ha.tally = tally;
   ha.status = status;
-  PriorSliceArgs ca = sa;
-  ca.tally = nullptr;
-  ca.cold_buf = w.cold_buf;
-  ca.cold_len = w.cold_len;
-  ca.cold_regions = p.ctas;
-  ca.cold_cap = p.cold_cap;
   for (long long b = p.prefix; b < N; b += kPriorChunk) {
     ha.range = prior_range(tokens, loss_mask, b, std::min(kPriorChunk, N - b));
     if (launch_prior_hot(ha, p.hot_smem, s) != cudaSuccess) return DELS_ERR_CUDA;
-    if (launch_prior_slices(ca, true, p.slice_smem, 24, sms, s) != cudaSuccess) return DELS_ERR_CUDA;
   }
   return DELS_OK;
 }

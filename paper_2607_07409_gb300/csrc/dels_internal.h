@@ -265,8 +265,9 @@ bool encode_tmap_3d(CUtensorMap* m, const void* base, CUtensorMapDataType dt, in
 
 // ---- unigram prior estimation (Appendix A) -----------------------------------
 constexpr int kPriorMaxPartials = 1024;            // CTAs of the two-level count sum
+constexpr int kPriorHistBuckets = 3776;            // count buckets of the hot-set choice
 constexpr long long kPriorHotMinN = 1ll << 24;     // shorter ranges: slice histograms only
-constexpr long long kPriorChunk = 1ll << 36;       // positions per hot pass (per-CTA bins stay < 2^32)
+constexpr long long kPriorChunk = 1ll << 36;       // positions per launch (per-thread tallies stay < 2^32)
 
 // Positions [0, n) of tokens / mask; [head, head + nvec) takes the vector
 // path (tokens + head 16-byte aligned, mask + head 4-byte aligned, nvec a
@@ -287,19 +288,17 @@ struct PriorSliceArgs {
   unsigned long long* counts;       // [V], accumulated
   unsigned long long* tally;        // [2] or null
   int* status;
-  const int32_t* cold_buf;          // cold source: [cold_regions][cold_cap]
-  const unsigned* cold_len;         // [cold_regions]
-  long long cold_regions;
-  long long cold_cap;
 };
 
 struct PriorSelectArgs {
   const unsigned long long* counts;   // [V]
   int V;
   int K;                              // hot slots
-  int nent;                           // remap words: ceil(V / 16)
-  size_t cache_bytes;                 // nent * 16 byte copy of the counts in smem, or 0
+  int nent;                           // remap words: ceil(V / 15)
+  unsigned* hist;                     // [kPriorHistBuckets], zero on entry and on exit
   uint32_t* entries;                  // [nent]
+  int32_t* stage;                     // [nent * 15] hot ids per CTA, before placement
+  unsigned* cta_total;                // [CTAs] hot ids per CTA
   int32_t* slot_id;                   // [K]
   unsigned* n_hot;
 };
@@ -313,10 +312,7 @@ struct PriorHotArgs {
   const uint32_t* entries;
   const int32_t* slot_id;
   const unsigned* n_hot;
-  unsigned* partials;                 // [ctas][K]
-  int32_t* cold_buf;                  // [ctas][cold_cap]
-  unsigned* cold_len;                 // [ctas]
-  long long cold_cap;
+  unsigned* partials;                 // [ctas][(K + 1) / 2] words of two 16-bit bins
   unsigned long long* counts;
   unsigned long long* tally;
   int* status;
@@ -340,18 +336,17 @@ struct PriorPlan {
   bool ok;
   int slices, slice;          // slice histograms: P slices of `slice` ids
   size_t slice_smem;
-  bool use_hot;               // hot/cold path
+  bool use_hot;               // hot ids on chip
   int nent, K;                // remap words, hot slots
-  size_t hot_smem, select_cache;
+  size_t hot_smem;
   int ctas;                   // CTAs of the hot pass (one per SM)
+  int select_ctas;            // CTAs of the hot-set choice
   long long prefix;           // positions counted by the slices before the hot set is chosen
-  long long cold_cap;         // cold-buffer entries per CTA
 };
 
 PriorPlan plan_prior(int V, long long N, int sms);
-cudaError_t launch_prior_slices(const PriorSliceArgs& a, bool cold, size_t smem, int max_members, int sms,
-                                cudaStream_t s);
-cudaError_t launch_prior_select(const PriorSelectArgs& a, cudaStream_t s);
+cudaError_t launch_prior_slices(const PriorSliceArgs& a, size_t smem, int max_members, int sms, cudaStream_t s);
+cudaError_t launch_prior_select(const PriorSelectArgs& a, int ctas, cudaStream_t s);
 cudaError_t launch_prior_hot(const PriorHotArgs& a, size_t smem, cudaStream_t s);
 cudaError_t launch_prior_total(const PriorLogArgs& a, int sms, cudaStream_t s);
 cudaError_t launch_prior_log(const PriorLogArgs& a, int sms, cudaStream_t s);

@@ -13,16 +13,18 @@
 // * Slice histograms (k_prior_slices): the vocabulary is cut into P slices
 //   that each fit; P groups of CTAs read the same positions, each group
 //   counting one slice. Used alone when P = 1 (small vocabularies) or when
-//   the range is short, and for the steps below.
-// * Hot/cold (large vocabularies, long corpora): a short prefix is counted
-//   exactly by the slices; the K ids with the largest counts so far become
-//   the hot set (k_prior_select), addressed through a 16-ids-per-word remap
-//   (16 presence bits + the number of hot ids before the word). The main pass
-//   (k_prior_hot) counts hot ids in shared memory and appends the others to
-//   a per-CTA cold buffer; the per-CTA hot bins are then summed
-//   (k_prior_hot_reduce) and the cold buffer is counted by the slices.
-//   Every position is counted exactly once whichever ids are hot; the hot
-//   set only decides the speed.
+//   the range is short.
+// * Hot ids on chip (large vocabularies, long corpora): a short prefix is
+//   counted exactly by the slices; the ids with the largest counts so far
+//   become the hot set, at most K of them (k_prior_hist, k_prior_mark,
+//   k_prior_place: a count histogram, presence bits, slot numbers). A remap
+//   word covers 15 ids: 15 presence bits and the 17-bit slot number of the
+//   first hot one. The main pass (k_prior_hot) counts hot ids in 16-bit
+//   shared-memory bins, two to a word (about 95K of them), which hand 2^15
+//   to the global count each time they reach it; the few cold ids go to the
+//   global counts directly. The per-CTA bins are summed at the end
+//   (k_prior_hot_reduce). Every position is counted exactly once whichever
+//   ids are hot; the hot set only decides the speed.
 //
 // The log step is a map over V after a two-level sum of the counts.
 #include <algorithm>
@@ -37,7 +39,10 @@ constexpr int kThreads = 1024;               // smem-bound kernels: one CTA per 
 constexpr int kWarps = kThreads / 32;
 constexpr int kMapThreads = 256;             // the V-sized maps (sum, log)
 constexpr int kWarpSpan = 512;               // positions a warp takes per vector step
-constexpr int kSelectBuckets = 3776;         // count buckets of the hot-set choice (32 x 118)
+constexpr int kSelectBuckets = kPriorHistBuckets;   // count buckets of the hot-set choice (32 x 118)
+constexpr int kIdsPerWord = 15;              // remap word: 15 presence bits + a 17-bit slot number
+constexpr unsigned kFlush = 0x8000u;         // a 16-bit hot bin hands this to the global count
+constexpr int kLogTable = 256;               // log(c + lambda) tabulated for counts below this
 
 struct Tally {   // per thread; a thread sees far fewer than 2^32 positions per launch
   unsigned in = 0, out = 0;
@@ -52,6 +57,9 @@ __device__ __forceinline__ unsigned long long warp_sum_u64(unsigned long long x)
 __device__ __forceinline__ int int4_at(const int4& v, int k) {
   return k == 0 ? v.x : k == 1 ? v.y : k == 2 ? v.z : v.w;
 }
+
+// id / 15 for any 32-bit id: multiply by ceil(2^35 / 15) and keep bits 35 and up
+__device__ __forceinline__ unsigned div15(unsigned id) { return __umulhi(id, 0x88888889u) >> 3; }
 
 // byte k of w, zero-extended (k a compile-time constant after unrolling)
 __device__ __forceinline__ uint32_t mask_byte(uint32_t w, int k) { return __byte_perm(w, 0u, 0x4440u | (unsigned)k); }
@@ -113,10 +121,7 @@ __device__ __forceinline__ void visit(const PriorRange& r, long long worker, lon
 
 // Slice histograms. CTA b counts slice b % P of the vocabulary over the
 // positions its group member index b / P takes; the bins are added to the
-// 64-bit counts at the end (coalesced atomics). Source: the corpus range
-// (COLD = false; group 0 keeps the tallies) or the per-CTA cold buffers of
-// k_prior_hot (COLD = true; every entry is an in-range id).
-template <bool COLD>
+// 64-bit counts at the end (coalesced atomics). Group 0 keeps the tallies.
 __global__ void __launch_bounds__(kThreads) k_prior_slices(PriorSliceArgs a) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   unsigned* bins = reinterpret_cast<unsigned*>(smem_raw);
@@ -130,53 +135,21 @@ __global__ void __launch_bounds__(kThreads) k_prior_slices(PriorSliceArgs a) {
   __syncthreads();
   pdl_wait();
   Tally t;
-  if (!COLD) {
-    // every group sees every position; group 0's tallies are the ones kept
-    visit<false>(a.range, member * kWarps + (threadIdx.x >> 5), members * kWarps,
-                 [&](int id, uint32_t m, bool) {
-                   const bool masked = m != 0u;
-                   const bool in_range = (unsigned)id < (unsigned)a.V;
-                   t.in += (masked && in_range) ? 1u : 0u;
-                   t.out += (masked && !in_range) ? 1u : 0u;
-                   const unsigned u = (unsigned)(id - lo);   // < nb only for in-range ids of the slice
-                   if (masked && u < (unsigned)nb) atomicAdd(bins + u, 1u);
-                 });
-    if (g != 0) t = Tally{};
-  } else {
-    // regions start 16-byte aligned (cold_cap is a multiple of 4 entries)
-    for (long long rgn = member; rgn < a.cold_regions; rgn += members) {
-      const long long len = min((long long)__ldcg(a.cold_len + rgn), a.cold_cap);
-      const int32_t* buf = a.cold_buf + rgn * a.cold_cap;
-      const int4* b4 = reinterpret_cast<const int4*>(buf);
-      const long long n4 = len / 4;
-      constexpr int U = 4;
-      for (long long i0 = threadIdx.x; i0 < n4; i0 += U * kThreads) {
-        int4 v[U];
-#pragma unroll
-        for (int k = 0; k < U; ++k) {
-          const long long i = i0 + (long long)k * kThreads;
-          v[k] = i < n4 ? __ldcg(b4 + i) : make_int4(-1, -1, -1, -1);
-        }
-#pragma unroll
-        for (int k = 0; k < U; ++k)
-#pragma unroll
-          for (int c = 0; c < 4; ++c) {
-            const unsigned u = (unsigned)(int4_at(v[k], c) - lo);
-            if (u < (unsigned)nb) atomicAdd(bins + u, 1u);
-          }
-      }
-      for (long long i = n4 * 4 + threadIdx.x; i < len; i += kThreads) {
-        const unsigned u = (unsigned)(__ldcg(buf + i) - lo);
-        if (u < (unsigned)nb) atomicAdd(bins + u, 1u);
-      }
-    }
-  }
+  visit<false>(a.range, member * kWarps + (threadIdx.x >> 5), members * kWarps, [&](int id, uint32_t m, bool) {
+    const bool masked = m != 0u;
+    const bool in_range = (unsigned)id < (unsigned)a.V;
+    t.in += (masked && in_range) ? 1u : 0u;
+    t.out += (masked && !in_range) ? 1u : 0u;
+    const unsigned u = (unsigned)(id - lo);   // < nb only for in-range ids of the slice
+    if (masked && u < (unsigned)nb) atomicAdd(bins + u, 1u);
+  });
+  if (g != 0) t = Tally{};
   __syncthreads();
   for (int b = threadIdx.x; b < nb; b += kThreads) {
     const unsigned c = bins[b];
     if (c) atomicAdd(a.counts + lo + b, (unsigned long long)c);
   }
-  if (!COLD) flush_tally(t, a.tally, a.status, red);
+  flush_tally(t, a.tally, a.status, red);
 }
 
 // Count buckets of the hot-set choice: exact below 2048, then 32 buckets per
@@ -194,51 +167,36 @@ __device__ __forceinline__ unsigned long long bucket_low(int b) {
   return (1ull << lg) | ((unsigned long long)sub << (lg - 5));
 }
 
-// The hot set: the ids whose count so far is at least T, for the smallest
-// bucket boundary T >= 1 that keeps the set within K slots (so it never
-// exceeds K), as the remap entries[e] = presence bits of ids 16e..16e+15 in
-// the low half and the number of hot ids before id 16e in the high half,
-// plus slot_id[s] = the id of hot slot s. One CTA; the counts are read once
-// into a byte copy min(c, 255) in shared memory, which decides presence when
-// T <= 255 (otherwise the counts are read again).
-__global__ void __launch_bounds__(kThreads) k_prior_select(PriorSelectArgs a) {
-  extern __shared__ __align__(16) unsigned char c8[];   // [nent * 16] when a.cache_bytes
-  __shared__ unsigned hist[kSelectBuckets];
-  __shared__ unsigned wsum[kWarps];
-  __shared__ unsigned wbase[kWarps];
-  __shared__ unsigned thr_bucket;
-  __shared__ unsigned run_base;
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  for (int i = threadIdx.x; i < kSelectBuckets; i += kThreads) hist[i] = 0u;
-  if (a.cache_bytes)
-    for (int i = a.V + threadIdx.x; i < a.nent * 16; i += kThreads) c8[i] = 0;
-  if (threadIdx.x == 0) run_base = 0u;
+// Step 1 of the hot-set choice: the histogram of count buckets, into the
+// global hist (zero on entry; k_prior_place clears it again). Most ids have
+// tiny counts, so buckets 0..7 are counted per thread instead of with
+// shared-memory atomics on a handful of addresses.
+__global__ void __launch_bounds__(kThreads) k_prior_hist(PriorSelectArgs a) {
+  __shared__ unsigned h[kSelectBuckets];
+  const int lane = threadIdx.x & 31;
+  for (int i = threadIdx.x; i < kSelectBuckets; i += kThreads) h[i] = 0u;
   __syncthreads();
   pdl_wait();
-  // most ids have tiny counts: buckets 0..7 are counted per thread (no
-  // shared-memory atomics on a handful of addresses), the rest in smem
-  constexpr int U = 8, kSmall = 8;
+  constexpr int U = 4, kSmall = 8;
   unsigned small[kSmall];
 #pragma unroll
   for (int j = 0; j < kSmall; ++j) small[j] = 0u;
-  for (int v0 = threadIdx.x; v0 < a.V; v0 += U * kThreads) {
+  const int stride = gridDim.x * kThreads;
+  for (int v0 = blockIdx.x * kThreads + threadIdx.x; v0 < a.V; v0 += U * stride) {
     unsigned long long c[U];
 #pragma unroll
     for (int k = 0; k < U; ++k) {
-      const int v = v0 + k * kThreads;
+      const int v = v0 + k * stride;
       c[k] = v < a.V ? __ldcg(a.counts + v) : ~0ull;
     }
 #pragma unroll
     for (int k = 0; k < U; ++k) {
-      const int v = v0 + k * kThreads;
-      if (v < a.V) {
-        if (c[k] < (unsigned long long)kSmall) {
+      if (v0 + k * stride >= a.V) continue;
+      if (c[k] < (unsigned long long)kSmall) {
 #pragma unroll
-          for (int j = 0; j < kSmall; ++j) small[j] += c[k] == (unsigned long long)j ? 1u : 0u;
-        } else {
-          atomicAdd(hist + count_bucket(c[k]), 1u);
-        }
-        if (a.cache_bytes) c8[v] = (unsigned char)min(c[k], 255ull);
+        for (int j = 0; j < kSmall; ++j) small[j] += c[k] == (unsigned long long)j ? 1u : 0u;
+      } else {
+        atomicAdd(h + count_bucket(c[k]), 1u);
       }
     }
   }
@@ -247,63 +205,84 @@ __global__ void __launch_bounds__(kThreads) k_prior_select(PriorSelectArgs a) {
     unsigned x = small[j];
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
-    if (lane == 0 && x) atomicAdd(hist + j, x);
+    if (lane == 0 && x) atomicAdd(h + j, x);
   }
+  __syncthreads();
+  for (int i = threadIdx.x; i < kSelectBuckets; i += kThreads)
+    if (h[i]) atomicAdd(a.hist + i, h[i]);
+}
+
+// The smallest bucket boundary T >= 1 with #{v : c(v) >= T} <= K, from a
+// shared-memory copy of the histogram (run by warp 0).
+__device__ unsigned long long hot_threshold(const unsigned* hist, int K) {
+  const int lane = threadIdx.x & 31;
+  constexpr int per = kSelectBuckets / 32;
+  unsigned s = 0;
+  for (int i = 0; i < per; ++i) s += hist[lane * per + i];
+  unsigned S = s;   // #{bucket >= per * lane}
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const unsigned y = __shfl_down_sync(0xffffffffu, S, o);
+    if (lane + o < 32) S += y;
+  }
+  unsigned S_next = __shfl_down_sync(0xffffffffu, S, 1);
+  if (lane == 31) S_next = 0u;
+  int t = 0;
+  if (S > (unsigned)K && S_next <= (unsigned)K) {
+    // the crossing lies in this lane's buckets
+    unsigned above = S_next;
+    for (int i = per - 1; i >= 0; --i) {
+      const unsigned h = hist[lane * per + i];
+      if (above + h > (unsigned)K) {
+        t = lane * per + i + 1;
+        break;
+      }
+      above += h;
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) t = max(t, __shfl_xor_sync(0xffffffffu, t, o));
+  return bucket_low(max(t, 1));
+}
+
+// Step 2: presence bits. CTA c owns remap words [c * per, (c + 1) * per);
+// hot ids get slot numbers counted from the CTA's first word (the CTA's own
+// base is added by k_prior_place), and are listed in stage[15 * first word ..].
+__global__ void __launch_bounds__(kThreads) k_prior_mark(PriorSelectArgs a) {
+  __shared__ unsigned hs[kSelectBuckets];
+  __shared__ unsigned wsum[kWarps];
+  __shared__ unsigned wbase[kWarps];
+  __shared__ unsigned long long thr;
+  __shared__ unsigned run_base;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  pdl_wait();
+  for (int i = threadIdx.x; i < kSelectBuckets; i += kThreads) hs[i] = __ldcg(a.hist + i);
   __syncthreads();
   if (warp == 0) {
-    // lane L holds buckets [per L, per L + per); S = #{c : bucket >= per L}
-    constexpr int per = kSelectBuckets / 32;
-    unsigned s = 0;
-    for (int i = 0; i < per; ++i) s += hist[lane * per + i];
-    unsigned S = s;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const unsigned y = __shfl_down_sync(0xffffffffu, S, o);
-      if (lane + o < 32) S += y;
+    const unsigned long long T = hot_threshold(hs, a.K);
+    if (lane == 0) {
+      thr = T;
+      run_base = 0u;
     }
-    unsigned S_next = __shfl_down_sync(0xffffffffu, S, 1);
-    if (lane == 31) S_next = 0u;
-    int t = 0;
-    if (S > (unsigned)a.K && S_next <= (unsigned)a.K) {
-      // the crossing lies in this lane's range: smallest t with #{bucket >= t} <= K
-      unsigned above = S_next;
-      for (int b = lane * per + per - 1; b >= lane * per; --b) {
-        if (above + hist[b] > (unsigned)a.K) {
-          t = b + 1;
-          break;
-        }
-        above += hist[b];
-      }
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) t = max(t, __shfl_xor_sync(0xffffffffu, t, o));
-    if (lane == 0) thr_bucket = (unsigned)max(t, 1);
   }
   __syncthreads();
-  const unsigned long long T = bucket_low((int)thr_bucket);
-  const bool from_cache = a.cache_bytes && T <= 255ull;
-  // rounds of kThreads entries; thread i takes entry r * kThreads + i
-  for (int e0 = 0; e0 < a.nent; e0 += kThreads) {
-    const int e = e0 + threadIdx.x;
+  const unsigned long long T = thr;
+  const int per = (a.nent + gridDim.x - 1) / gridDim.x;
+  const int w_begin = min(a.nent, (int)blockIdx.x * per), w_end = min(a.nent, w_begin + per);
+  int32_t* stage = a.stage + (long long)w_begin * kIdsPerWord;
+  for (int w0 = w_begin; w0 < w_end; w0 += kThreads) {
+    const int w = w0 + threadIdx.x;
     unsigned bits = 0;
-    if (e < a.nent) {
-      if (from_cache) {
-        const uint4 q = *reinterpret_cast<const uint4*>(c8 + (size_t)e * 16);
-        const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+    if (w < w_end) {
+      unsigned long long c[kIdsPerWord];
 #pragma unroll
-        for (int j = 0; j < 16; ++j)
-          if (((w[j >> 2] >> (8 * (j & 3))) & 0xFFu) >= (uint32_t)T) bits |= 1u << j;
-      } else {
-        unsigned long long c[16];
-#pragma unroll
-        for (int j = 0; j < 16; ++j) {
-          const int v = e * 16 + j;
-          c[j] = v < a.V ? __ldcg(a.counts + v) : 0ull;
-        }
-#pragma unroll
-        for (int j = 0; j < 16; ++j)
-          if (c[j] >= T) bits |= 1u << j;
+      for (int j = 0; j < kIdsPerWord; ++j) {
+        const int v = w * kIdsPerWord + j;
+        c[j] = v < a.V ? __ldcg(a.counts + v) : 0ull;
       }
+#pragma unroll
+      for (int j = 0; j < kIdsPerWord; ++j)
+        if (c[j] >= T) bits |= 1u << j;
     }
     const unsigned cnt = __popc(bits);
     unsigned incl = cnt;
@@ -315,66 +294,105 @@ __global__ void __launch_bounds__(kThreads) k_prior_select(PriorSelectArgs a) {
     if (lane == 31) wsum[warp] = incl;
     __syncthreads();
     if (warp == 0) {
-      const unsigned w0 = wsum[lane];
-      unsigned w = w0;
+      const unsigned x0 = wsum[lane];
+      unsigned x = x0;
 #pragma unroll
       for (int o = 1; o < 32; o <<= 1) {
-        const unsigned y = __shfl_up_sync(0xffffffffu, w, o);
-        if (lane >= o) w += y;
+        const unsigned y = __shfl_up_sync(0xffffffffu, x, o);
+        if (lane >= o) x += y;
       }
-      wbase[lane] = w - w0;
+      wbase[lane] = x - x0;
     }
     __syncthreads();
-    unsigned base = run_base + wbase[warp] + incl - cnt;
-    if (e < a.nent) {
-      a.entries[e] = bits | (base << 16);
-      while (bits) {
-        const int j = __ffs(bits) - 1;
-        bits &= bits - 1u;
-        if (base < (unsigned)a.K) a.slot_id[base] = e * 16 + j;
-        ++base;
-      }
+    unsigned base = run_base + wbase[warp] + incl - cnt;   // local slot of this word's first hot id
+    if (w < w_end) {
+      a.entries[w] = bits | (base << kIdsPerWord);
+      for (unsigned b = bits; b; b &= b - 1u) stage[base++] = w * kIdsPerWord + (__ffs(b) - 1);
     }
     __syncthreads();
     if (threadIdx.x == kThreads - 1) run_base = base;
     __syncthreads();
   }
-  if (threadIdx.x == 0) *a.n_hot = min(run_base, (unsigned)a.K);
+  if (threadIdx.x == 0) a.cta_total[blockIdx.x] = run_base;
 }
 
-// Main pass over a long range: loss-masked hot ids are counted in shared
-// memory, other in-range ids are appended to this CTA's cold buffer (past
-// its capacity they go to the global counts directly). Writes the CTA's hot
-// bins to partials[blockIdx.x][0..K) and its cold length.
+// Step 3: each CTA adds its base (the hot ids of the CTAs before it) to its
+// remap words and moves its staged ids to slot_id. A word whose slots would
+// not all fit in K (never, when the histogram is right) is left with no hot
+// ids, so its ids are counted as cold. CTA 0 clears the histogram.
+__global__ void __launch_bounds__(kMapThreads) k_prior_place(PriorSelectArgs a) {
+  __shared__ unsigned base_s, total_s;
+  pdl_wait();
+  if (threadIdx.x < 32) {
+    const int lane = threadIdx.x;
+    unsigned before = 0, total = 0;
+    for (int c = lane; c < (int)gridDim.x; c += 32) {
+      const unsigned x = __ldcg(a.cta_total + c);
+      total += x;
+      if (c < (int)blockIdx.x) before += x;
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      before += __shfl_xor_sync(0xffffffffu, before, o);
+      total += __shfl_xor_sync(0xffffffffu, total, o);
+    }
+    if (lane == 0) {
+      base_s = before;
+      total_s = total;
+    }
+  }
+  __syncthreads();
+  const unsigned base = base_s;
+  const int per = (a.nent + gridDim.x - 1) / gridDim.x;
+  const int w_begin = min(a.nent, (int)blockIdx.x * per), w_end = min(a.nent, w_begin + per);
+  for (int w = w_begin + threadIdx.x; w < w_end; w += kMapThreads) {
+    const uint32_t e = __ldcg(a.entries + w);
+    const unsigned bits = e & ((1u << kIdsPerWord) - 1u);
+    const unsigned slot0 = base + (e >> kIdsPerWord);
+    a.entries[w] = slot0 + __popc(bits) <= (unsigned)a.K ? (bits | (slot0 << kIdsPerWord)) : 0u;
+  }
+  const unsigned mine = __ldcg(a.cta_total + blockIdx.x);
+  const int32_t* stage = a.stage + (long long)w_begin * kIdsPerWord;
+  for (unsigned i = threadIdx.x; i < mine; i += kMapThreads)
+    if (base + i < (unsigned)a.K) a.slot_id[base + i] = __ldcg(stage + i);
+  if (blockIdx.x == 0) {
+    if (threadIdx.x == 0) *a.n_hot = min(total_s, (unsigned)a.K);
+    for (int i = threadIdx.x; i < kSelectBuckets; i += kMapThreads) a.hist[i] = 0u;
+  }
+}
+
+// Main pass over a long range: loss-masked hot ids are counted in 16-bit
+// shared-memory bins (two per word; a bin that reaches 2^15 hands 2^15 to the
+// global count, so it never carries into its neighbour), the others go to the
+// global counts directly. Writes the CTA's bin words to partials.
 __global__ void __launch_bounds__(kThreads, 1) k_prior_hot(PriorHotArgs a) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   uint32_t* ent = reinterpret_cast<uint32_t*>(smem_raw);
-  unsigned* bins = ent + a.nent;
+  unsigned* words = ent + a.nent;
   __shared__ unsigned long long red[2 * kWarps];
-  __shared__ unsigned cursor;
+  const int kw = (a.K + 1) / 2;
   pdl_wait();
   for (int i = threadIdx.x; i < a.nent; i += kThreads) ent[i] = __ldcg(a.entries + i);
-  for (int i = threadIdx.x; i < a.K; i += kThreads) bins[i] = 0u;
-  if (threadIdx.x == 0) cursor = 0u;
+  for (int i = threadIdx.x; i < kw; i += kThreads) words[i] = 0u;
   __syncthreads();
   const int lane = threadIdx.x & 31;
-  int32_t* cold = a.cold_buf + (long long)blockIdx.x * a.cold_cap;
-  const unsigned cap = (unsigned)a.cold_cap;
   Tally t;
-  auto put_cold = [&](unsigned slot, int id) {
-    if (slot < cap) cold[slot] = id;
-    else atomicAdd(a.counts + id, 1ull);
-  };
-  // true: hot (counted here); false: a loss-masked in-range id that is cold
-  auto count_hot = [&](int id) -> bool {
-    const uint32_t e = ent[id >> 4];
-    const uint32_t bit = 1u << (id & 15);
-    const uint32_t slot = (e >> 16) + __popc(e & (bit - 1u));
-    if ((e & bit) && slot < (uint32_t)a.K) {
-      atomicAdd(bins + slot, 1u);
-      return true;
+  // one loss-masked in-range id
+  auto count_one = [&](int id) {
+    const unsigned q = div15((unsigned)id);
+    const uint32_t e = ent[q];
+    const uint32_t bit = 1u << ((unsigned)id - q * kIdsPerWord);
+    const uint32_t slot = (e >> kIdsPerWord) + __popc(e & (bit - 1u));
+    if ((e & bit) != 0u && slot < (uint32_t)a.K) {
+      const unsigned sh = (slot & 1u) << 4;
+      const unsigned old = atomicAdd(words + (slot >> 1), 1u << sh);
+      if (((old >> sh) & 0xFFFFu) == kFlush - 1u) {
+        atomicSub(words + (slot >> 1), kFlush << sh);
+        atomicAdd(a.counts + id, (unsigned long long)kFlush);
+      }
+    } else {
+      atomicAdd(a.counts + id, 1ull);
     }
-    return false;
   };
   const PriorRange& r = a.range;
   const long long worker = (long long)blockIdx.x * kWarps + (threadIdx.x >> 5);
@@ -390,41 +408,18 @@ __global__ void __launch_bounds__(kThreads, 1) k_prior_hot(PriorHotArgs a) {
     for (int k = 0; k < 4; ++k) tk[k] = __ldcs(tv + w0 + 32 * k);
 #pragma unroll
     for (int k = 0; k < 4; ++k) mk[k] = __ldcs(mv + w0 + 32 * k);
-    uint32_t cold_bits = 0;
+    uint32_t valid_bits = 0, bad_bits = 0;
 #pragma unroll
     for (int q = 0; q < 16; ++q) {
-      // straight-line and predicated: no branch per position
       const int id = int4_at(tk[q >> 2], q & 3);
       const bool masked = mask_byte(mk[q >> 2], q & 3) != 0u;
       const bool in_range = (unsigned)id < (unsigned)a.V;
-      const bool valid = masked && in_range;
-      t.in += valid ? 1u : 0u;
-      t.out += (masked && !in_range) ? 1u : 0u;
-      uint32_t e = 0;
-      if (valid) e = ent[id >> 4];
-      const uint32_t bit = 1u << (id & 15);
-      const uint32_t slot = (e >> 16) + __popc(e & (bit - 1u));
-      const bool hot = (e & bit) != 0u && slot < (uint32_t)a.K;
-      if (hot) atomicAdd(bins + slot, 1u);
-      cold_bits |= (valid && !hot) ? (1u << q) : 0u;
+      valid_bits |= (masked && in_range) ? (1u << q) : 0u;
+      bad_bits |= (masked && !in_range) ? (1u << q) : 0u;
+      if (masked && in_range) count_one(id);
     }
-    // one cursor add per warp step: lanes take consecutive runs of the cold buffer
-    const unsigned n = __popc(cold_bits);
-    unsigned incl = n;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const unsigned y = __shfl_up_sync(0xffffffffu, incl, o);
-      if (lane >= o) incl += y;
-    }
-    const unsigned total = __shfl_sync(0xffffffffu, incl, 31);
-    if (total) {
-      unsigned base = 0;
-      if (lane == 31) base = atomicAdd(&cursor, total);
-      base = __shfl_sync(0xffffffffu, base, 31) + incl - n;
-#pragma unroll
-      for (int q = 0; q < 16; ++q)
-        if ((cold_bits >> q) & 1u) put_cold(base++, int4_at(tk[q >> 2], q & 3));
-    }
+    t.in += __popc(valid_bits);
+    t.out += __popc(bad_bits);
   }
   const long long rest = r.n - r.nvec;
   for (long long j = worker * 32 + lane; j < rest; j += nworkers * 32) {
@@ -436,27 +431,36 @@ __global__ void __launch_bounds__(kThreads, 1) k_prior_hot(PriorHotArgs a) {
       continue;
     }
     ++t.in;
-    if (!count_hot(id)) put_cold(atomicAdd(&cursor, 1u), id);
+    count_one(id);
   }
   __syncthreads();
-  unsigned* out = a.partials + (long long)blockIdx.x * a.K;
-  for (int i = threadIdx.x; i < a.K; i += kThreads) out[i] = bins[i];
-  if (threadIdx.x == 0) a.cold_len[blockIdx.x] = min(cursor, cap);
+  unsigned* out = a.partials + (long long)blockIdx.x * kw;
+  for (int i = threadIdx.x; i < kw; i += kThreads) out[i] = words[i];
   flush_tally(t, a.tally, a.status, red);
 }
 
-// counts[slot_id[s]] += sum over CTAs of partials[cta][s], for the n_hot slots.
+// counts[slot_id[s]] += the sum over CTAs of bin s (the 16-bit halves of the
+// partial words), for the n_hot slots.
 __global__ void __launch_bounds__(kMapThreads) k_prior_hot_reduce(PriorHotArgs a) {
   pdl_wait();
   const unsigned n_hot = min(__ldcg(a.n_hot), (unsigned)a.K);
-  for (long long s = (long long)blockIdx.x * kMapThreads + threadIdx.x; s < n_hot;
-       s += (long long)gridDim.x * kMapThreads) {
-    unsigned long long sum = 0;
-    for (int c = 0; c < a.ctas; ++c) sum += __ldcg(a.partials + (long long)c * a.K + s);
-    if (sum) {
-      const int id = __ldcg(a.slot_id + s);
-      a.counts[id] += sum;
+  const long long kw = (a.K + 1) / 2;
+  for (long long w = (long long)blockIdx.x * kMapThreads + threadIdx.x; 2 * w < n_hot;
+       w += (long long)gridDim.x * kMapThreads) {
+    unsigned long long lo = 0, hi = 0;
+    constexpr int U = 8;
+    for (int c0 = 0; c0 < a.ctas; c0 += U) {
+      unsigned x[U];
+#pragma unroll
+      for (int k = 0; k < U; ++k) x[k] = c0 + k < a.ctas ? __ldcg(a.partials + (long long)(c0 + k) * kw + w) : 0u;
+#pragma unroll
+      for (int k = 0; k < U; ++k) {
+        lo += x[k] & 0xFFFFu;
+        hi += x[k] >> 16;
+      }
     }
+    if (lo) a.counts[__ldcg(a.slot_id + 2 * w)] += lo;
+    if (hi && 2 * w + 1 < n_hot) a.counts[__ldcg(a.slot_id + 2 * w + 1)] += hi;
   }
 }
 
@@ -491,16 +495,23 @@ __global__ void __launch_bounds__(kMapThreads) k_prior_total(PriorLogArgs a) {
 }
 
 // l_P(v) = log(c(v) + lambda) - log(sum_u c(u) + V lambda), in float64,
-// stored as float32. Optionally copies the counts and the tally out (the
+// stored as float32; log(c + lambda) of the small counts (most ids) comes
+// from a per-CTA table. Optionally copies the counts and the tally out (the
 // one-call estimate keeps both in its workspace).
 __global__ void __launch_bounds__(kMapThreads) k_prior_log(PriorLogArgs a) {
-  pdl_wait();
+  __shared__ double tab[kLogTable];
+  __shared__ double log_s_sh;
   const double lam = a.lambda;
-  const double log_s = log((double)__ldcg(a.total) + (double)a.V * lam);
+  for (int i = threadIdx.x; i < kLogTable; i += kMapThreads) tab[i] = log((double)i + lam);
+  pdl_wait();
+  if (threadIdx.x == 0) log_s_sh = log((double)__ldcg(a.total) + (double)a.V * lam);
+  __syncthreads();
+  const double log_s = log_s_sh;
   const long long stride = (long long)gridDim.x * kMapThreads;
   for (long long v = (long long)blockIdx.x * kMapThreads + threadIdx.x; v < a.V; v += stride) {
     const unsigned long long c = __ldcg(a.counts + v);
-    a.out[v] = (float)(log((double)c + lam) - log_s);
+    const double lc = c < (unsigned long long)kLogTable ? tab[c] : log((double)c + lam);
+    a.out[v] = (float)(lc - log_s);
     if (a.counts_out) a.counts_out[v] = c;
   }
   if (a.tally_out && blockIdx.x == 0 && threadIdx.x < 2) a.tally_out[threadIdx.x] = __ldcg(a.tally + threadIdx.x);
@@ -520,19 +531,15 @@ int max_smem_optin() {
 
 // CTAs per SM that one k_prior_slices launch can keep resident
 int slices_per_sm(size_t smem) {
-  static size_t set_for[2] = {0, 0};
-  int per_sm = 0;
-  for (int c = 0; c < 2; ++c) {
-    void (*k)(PriorSliceArgs) = c ? k_prior_slices<true> : k_prior_slices<false>;
-    if (set_for[c] < smem) {
-      if (cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess) return 0;
-      set_for[c] = smem;
-    }
-    int v = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, k, kThreads, smem) != cudaSuccess) return 0;
-    per_sm = c ? std::min(per_sm, v) : v;
+  static size_t set_for = 0;
+  if (set_for < smem) {
+    if (cudaFuncSetAttribute(k_prior_slices, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
+      return 0;
+    set_for = smem;
   }
-  return per_sm;
+  int v = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, k_prior_slices, kThreads, smem) != cudaSuccess) return 0;
+  return v;
 }
 
 }  // namespace
@@ -546,44 +553,35 @@ PriorPlan plan_prior(int V, long long N, int sms) {
   p.slices = (V + bins_max - 1) / bins_max;
   p.slice = (V + p.slices - 1) / p.slices;
   p.slice_smem = (size_t)p.slice * 4;
-  // hot/cold: the remap and as many hot bins as fit beside it (slot numbers
-  // live in the 16-bit high half of a remap entry)
-  p.nent = (V + 15) / 16;
+  // hot ids: the remap and as many 16-bit bins as fit beside it (slot
+  // numbers have 17 bits in a remap word)
+  p.nent = (V + kIdsPerWord - 1) / kIdsPerWord;
   const long long hot_bytes = (long long)smem - 2048 - (long long)p.nent * 4;
-  p.K = hot_bytes > 0 ? (int)std::min<long long>(hot_bytes / 4 / 32 * 32, 65504) : 0;
-  p.hot_smem = (size_t)(p.nent + p.K) * 4;
-  const size_t cache = (size_t)p.nent * 16;
-  p.select_cache = cache + 8192 + 16 * 1024 <= (size_t)smem ? cache : 0;   // beside the static hist
+  p.K = hot_bytes > 0 ? (int)std::min<long long>(hot_bytes / 2 / 64 * 64, (1 << 17) - 64) : 0;
+  p.hot_smem = (size_t)p.nent * 4 + (size_t)(p.K + 1) / 2 * 4;
   p.ctas = sms;
-  p.use_hot = p.slices > 1 && p.K >= 4096 && N >= kPriorHotMinN;
-  if (p.use_hot) {
-    p.prefix = std::min<long long>(N, std::max<long long>(kPriorHotMinN / 4, N / 64));
-    const long long main_n = std::min<long long>(N - p.prefix, kPriorChunk);
-    p.cold_cap = (std::max<long long>(4096, (main_n / 8 + sms - 1) / sms) + 127) / 128 * 128;
-  }
+  p.select_ctas = std::min(sms, kPriorMaxPartials);
+  // a CTA of the hot-set choice numbers its hot ids locally in the 17-bit field
+  const long long words_per_cta = (p.nent + p.select_ctas - 1) / p.select_ctas;
+  p.use_hot = p.slices > 1 && p.K >= 4096 && N >= kPriorHotMinN && words_per_cta * kIdsPerWord < (1 << 17);
+  if (p.use_hot) p.prefix = std::min<long long>(N, std::max<long long>(kPriorHotMinN / 4, N / 64));
   p.ok = true;
   return p;
 }
 
-cudaError_t launch_prior_slices(const PriorSliceArgs& a, bool cold, size_t smem, int max_members, int sms,
-                                cudaStream_t s) {
+cudaError_t launch_prior_slices(const PriorSliceArgs& a, size_t smem, int max_members, int sms, cudaStream_t s) {
   const int per_sm = slices_per_sm(smem);
   if (per_sm < 1 || per_sm * sms < a.slices) return cudaErrorInvalidConfiguration;
   const int members = std::max(1, std::min(per_sm * sms / a.slices, max_members));
-  const dim3 grid((unsigned)(members * a.slices));
-  return cold ? launch_pdl(k_prior_slices<true>, grid, dim3(kThreads), smem, s, a)
-              : launch_pdl(k_prior_slices<false>, grid, dim3(kThreads), smem, s, a);
+  return launch_pdl(k_prior_slices, dim3((unsigned)(members * a.slices)), dim3(kThreads), smem, s, a);
 }
 
-cudaError_t launch_prior_select(const PriorSelectArgs& a, cudaStream_t s) {
-  static size_t set_for = 0;
-  const size_t smem = a.cache_bytes;
-  if (set_for < smem) {
-    cudaError_t e = cudaFuncSetAttribute(k_prior_select, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    set_for = smem;
-  }
-  return launch_pdl(k_prior_select, dim3(1), dim3(kThreads), smem, s, a);
+cudaError_t launch_prior_select(const PriorSelectArgs& a, int ctas, cudaStream_t s) {
+  cudaError_t e = launch_pdl(k_prior_hist, dim3((unsigned)ctas), dim3(kThreads), 0, s, a);
+  if (e != cudaSuccess) return e;
+  e = launch_pdl(k_prior_mark, dim3((unsigned)ctas), dim3(kThreads), 0, s, a);
+  if (e != cudaSuccess) return e;
+  return launch_pdl(k_prior_place, dim3((unsigned)ctas), dim3(kMapThreads), 0, s, a);
 }
 
 cudaError_t launch_prior_hot(const PriorHotArgs& a, size_t smem, cudaStream_t s) {
@@ -595,7 +593,8 @@ cudaError_t launch_prior_hot(const PriorHotArgs& a, size_t smem, cudaStream_t s)
   }
   cudaError_t e = launch_pdl(k_prior_hot, dim3((unsigned)a.ctas), dim3(kThreads), smem, s, a);
   if (e != cudaSuccess) return e;
-  const int blocks = std::max(1, std::min(a.ctas * 4, (a.K + kMapThreads - 1) / kMapThreads));
+  const int kw = (a.K + 1) / 2;
+  const int blocks = std::max(1, std::min(a.ctas * 4, (kw + kMapThreads - 1) / kMapThreads));
   return launch_pdl(k_prior_hot_reduce, dim3((unsigned)blocks), dim3(kMapThreads), 0, s, a);
 }
 
@@ -606,8 +605,8 @@ cudaError_t launch_prior_total(const PriorLogArgs& a, int sms, cudaStream_t s) {
 }
 
 cudaError_t launch_prior_log(const PriorLogArgs& a, int sms, cudaStream_t s) {
-  long long blocks = ((long long)a.V + kMapThreads - 1) / kMapThreads;
-  blocks = std::max<long long>(1, std::min<long long>(blocks, (long long)sms * 4));
+  long long blocks = ((long long)a.V + 4 * kMapThreads - 1) / (4 * kMapThreads);
+  blocks = std::max<long long>(1, std::min<long long>(blocks, (long long)sms));
   return launch_pdl(k_prior_log, dim3((unsigned)blocks), dim3(kMapThreads), 0, s, a);
 }
 
