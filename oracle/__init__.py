@@ -14,7 +14,10 @@ Speculative Drafting"):
 * Algorithm 1: x_0 decoded from softmax(l_L^(0)) alone; for j = 1..s the local
   head runs over x_{0:j-1}, its logits are fused, and x_j is decoded from the
   softmax of the fused logits; the block is then verified by the target.
-  Decode at temperature 0 is the argmax (lowest vocabulary index on ties).
+  Decode at temperature 0 is the argmax (lowest vocabulary index on ties);
+  at temperature 1 it is a draw from the softmax by the Gumbel-max rule, with
+  Philox4x64-10 uniforms, and the block is verified by lossless speculative
+  sampling (accept with probability min(1, p/q), resample the residual).
 * Appendix A, local heads: the RNN head (target embedding -> one bias-free GRU
   layer -> SiLU(W_rank h) -> W_vocab r) and the Markov head
   (r = E_M(x_{i-1}), l_S = W_M r).
@@ -48,6 +51,14 @@ from .core import (  # noqa: F401
     greedy_decode,
     combine_argmax,
     verify_greedy,
+    philox4x64_10,
+    uniforms,
+    gumbel,
+    sample_decode,
+    verify_sampled,
+    STREAM_DRAFT,
+    STREAM_ACCEPT,
+    STREAM_RESIDUAL,
     acceptance_rates,
     poe_factors,
 )

@@ -142,6 +142,140 @@ def combine_argmax(long, short, prior, alpha: float, beta: float):
 
 
 # ----------------------------------------------------------------------------
+# temperature-1 Decode (Algorithm 1, x_j ~ softmax(l^(j))) and its random numbers
+# ----------------------------------------------------------------------------
+# The random numbers come from Philox4x64-10, the counter-based generator of
+# Salmon, Moraes, Dror and Shaw ("Parallel random numbers: as easy as 1, 2, 3",
+# SC 2011): ten rounds of two 64x64 -> 128-bit products on a 4-word counter
+# under a 2-word key that is bumped by two Weyl constants between rounds.
+# The drafting and verification kernels implement the same definition, so
+# both sides draw identical uniforms from (seed, step, request, position,
+# stream, vocabulary index).
+
+PHILOX_M0, PHILOX_M1 = 0xD2E7470EE14C6C93, 0xCA5A826395121157
+PHILOX_W0, PHILOX_W1 = 0x9E3779B97F4A7C15, 0xBB67AE8584CAA73B
+STREAM_DRAFT, STREAM_ACCEPT, STREAM_RESIDUAL = 0, 1, 2
+_M32 = np.uint64(0xFFFFFFFF)
+
+
+def _mulhilo64(a, m: int):
+    """(high, low) 64-bit halves of the 128-bit products a * m, a uint64 array."""
+    a = np.asarray(a, dtype=np.uint64)
+    m = np.uint64(m)
+    s32 = np.uint64(32)
+    a_lo, a_hi = a & _M32, a >> s32
+    m_lo, m_hi = m & _M32, m >> s32
+    p0, p1, p2, p3 = a_lo * m_lo, a_lo * m_hi, a_hi * m_lo, a_hi * m_hi
+    mid = (p0 >> s32) + (p1 & _M32) + (p2 & _M32)
+    hi = p3 + (p1 >> s32) + (p2 >> s32) + (mid >> s32)
+    with np.errstate(over="ignore"):
+        lo = a * m
+    return hi, lo
+
+
+def philox4x64_10(c0, c1, c2, c3, k0: int, k1: int):
+    """Philox4x64-10 of counters (c0, c1, c2, c3) (uint64 arrays, broadcast) under key (k0, k1)."""
+    x = [np.asarray(c, dtype=np.uint64) for c in np.broadcast_arrays(c0, c1, c2, c3)]
+    k0, k1 = np.uint64(k0 & 0xFFFFFFFFFFFFFFFF), np.uint64(k1 & 0xFFFFFFFFFFFFFFFF)
+    with np.errstate(over="ignore"):
+        for _ in range(10):
+            hi0, lo0 = _mulhilo64(x[0], PHILOX_M0)
+            hi1, lo1 = _mulhilo64(x[2], PHILOX_M1)
+            x = [hi1 ^ x[1] ^ k0, lo1, hi0 ^ x[3] ^ k1, lo0]
+            k0 = k0 + np.uint64(PHILOX_W0)
+            k1 = k1 + np.uint64(PHILOX_W1)
+    return x
+
+
+def uniforms(seed: int, step: int, b: int, j: int, stream: int, v):
+    """The uniform variates U(0, 1) of vocabulary indices v (array) for request
+    b, position j and stream (0 drafting, 1 acceptance, 2 residual/bonus).
+
+    Counter (v // 8, j, b, stream), key (seed, step); the 4 output words give 8
+    32-bit halves (high half first), and a half h gives u = (floor(h / 2^9) +
+    1/2) / 2^23, an exact float32 in [2^-24, 1 - 2^-24].
+    """
+    v = np.asarray(v, dtype=np.int64)
+    words = philox4x64_10((v >> 3).astype(np.uint64), np.uint64(j), np.uint64(b), np.uint64(stream), seed, step)
+    w = np.select([(v & 7) >> 1 == k for k in range(4)], words)
+    half = np.where((v & 1) == 0, w >> np.uint64(32), w & _M32)
+    return ((half >> np.uint64(9)).astype(np.float64) + 0.5) / float(1 << 23)
+
+
+def gumbel(u):
+    """Standard Gumbel variates g = -log(-log(u))."""
+    return -np.log(-np.log(np.asarray(u, dtype=np.float64)))
+
+
+def sample_decode(l, g):
+    """Temperature-1 Decode of one row by the Gumbel-max rule: x = argmax(l + g)
+    (lowest index on exact ties) is a draw from softmax(l) when g are i.i.d.
+    standard Gumbel. Returns (x, logp = l[x] - LSE(l), key gap = k[x] - max_{v != x} k[v],
+    LSE(l))."""
+    l = np.asarray(l, dtype=np.float64)
+    if np.any(np.isnan(l)) or np.any(l == np.inf):
+        raise ValueError("non-finite logits")
+    k = l + np.asarray(g, dtype=np.float64)
+    x = int(np.argmax(k))
+    z = lse(l)
+    rest = np.concatenate([k[:x], k[x + 1:]])
+    gap = float(k[x] - np.max(rest)) if rest.size else np.inf
+    return x, float(l[x] - z), gap, z
+
+
+def verify_sampled(draft, draft_logits, target, seed: int, step: int):
+    """Lossless speculative sampling (Leviathan et al. 2023; Chen et al. 2023)
+    of a block drafted at temperature 1.
+
+    draft [B, n] tokens; draft_logits [B, n, V] the logits each token was drawn
+    from (row j: softmax gives q_j); target [B, n+1, V] (softmax gives p_j).
+    For j = 0..n-1: accept x_j when u_j < p_j(x_j) / q_j(x_j), u_j the
+    acceptance uniform of (b, j); at the first rejection the bonus token is
+    drawn from the residual max(0, p_j - q_j) (normalised) by the Gumbel-max
+    rule with the residual stream at position j; when all n are accepted it
+    is drawn from p_n the same way at position n.
+
+    Returns (accept [B], bonus [B], info) with info["margin"][b] the distance
+    |u - p/q| of the deciding test (the smallest over the accepted positions
+    and the rejected one) and info["bonus_gap"][b] the key gap of the bonus draw.
+    """
+    D = np.asarray(draft, dtype=np.int64)
+    Q = to_f64(draft_logits)
+    T = to_f64(target)
+    B, n = D.shape
+    V = T.shape[2]
+    if Q.shape != (B, n, V) or T.shape[:2] != (B, n + 1):
+        raise ValueError("draft_logits must be [B, n, V] and target [B, n+1, V]")
+    vidx = np.arange(V)
+    accept = np.zeros(B, np.int64)
+    bonus = np.zeros(B, np.int64)
+    margin = np.full(B, np.inf)
+    bonus_gap = np.zeros(B)
+    for b in range(B):
+        a = n
+        for j in range(n):
+            p = np.exp(T[b, j] - lse(T[b, j]))
+            q = np.exp(Q[b, j] - lse(Q[b, j]))
+            x = D[b, j]
+            u = float(uniforms(seed, step, b, j, STREAM_ACCEPT, np.array([0]))[0])
+            ratio = p[x] / q[x]
+            margin[b] = min(margin[b], abs(u - ratio))
+            if not u < ratio:
+                a = j
+                w = np.maximum(p - q, 0.0)
+                with np.errstate(divide="ignore"):
+                    key = np.log(w) + gumbel(uniforms(seed, step, b, j, STREAM_RESIDUAL, vidx))
+                break
+        if a == n:
+            key = T[b, n] + gumbel(uniforms(seed, step, b, n, STREAM_RESIDUAL, vidx))
+        accept[b] = a
+        bonus[b] = int(np.argmax(key))
+        rest = np.delete(key, bonus[b])
+        bonus_gap[b] = float(key[bonus[b]] - np.max(rest)) if rest.size else np.inf
+    return accept, bonus, {"margin": margin, "bonus_gap": bonus_gap}
+
+
+# ----------------------------------------------------------------------------
 # verification (Algorithm 1, greedy verification by one target forward)
 # ----------------------------------------------------------------------------
 

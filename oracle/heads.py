@@ -17,7 +17,8 @@ from typing import Dict, Optional
 import numpy as np
 from scipy.special import erf
 
-from .core import to_f64, round_bf16, fuse, greedy_decode, lse
+from .core import (to_f64, round_bf16, fuse, greedy_decode, lse, sample_decode, gumbel, uniforms,
+                   STREAM_DRAFT)
 
 
 def _sigmoid(x):
@@ -224,10 +225,16 @@ class DraftResult:
     fused_max: Optional[np.ndarray] = None  # [B, n] maximum fused value (forced mode)
     logp_at: Optional[np.ndarray] = None    # [B, n] log softmax at the forced token
     short_rows: Optional[Dict] = None       # {(b, j): l_S row} when requested
+    lse: Optional[np.ndarray] = None        # [B, n] LSE of the fused row (temperature 1)
+    fused: Optional[np.ndarray] = None      # [B, n, V] fused rows (temperature 1, keep_fused)
 
 
-def draft_block(head, long, prior, alpha, beta, forced=None, keep_short=()):
-    """Algorithm 1 (temperature 0) for one block of B independent rows.
+def draft_block(head, long, prior, alpha, beta, forced=None, keep_short=(), sample=None, keep_fused=False):
+    """Algorithm 1 for one block of B independent rows, at temperature 0
+    (``sample=None``: Decode = argmax) or temperature 1 (``sample=(seed,
+    step)``: Decode draws x_j from softmax(l^(j)) by the Gumbel-max rule,
+    x_j = argmax(l^(j) + g), g the drafting-stream Gumbel variates of (b, j);
+    ``gap`` and the forced-mode values then refer to the keys l + g).
 
     long [B, n, V] long-context logits; prior [V] log unigram prior.
     Position 0: x_0 = argmax l_L^(0) (no local head, no prior term).
@@ -256,18 +263,30 @@ def draft_block(head, long, prior, alpha, beta, forced=None, keep_short=()):
     logp_at = np.zeros((B, n)) if forced is not None else None
     forced = None if forced is None else np.asarray(forced, dtype=np.int64)
     kept = {}
+    lse_out = np.zeros((B, n)) if sample is not None else None
+    fused_out = np.zeros((B, n, V)) if (sample is not None and keep_fused) else None
+    vidx = np.arange(V)
 
     def row_long(b, j):
         return to_f64(L[b, j])
 
     def record(b, j, f):
-        x, lp, g = greedy_decode(f)
+        if sample is None:
+            x, lp, g = greedy_decode(f)
+            key = f
+        else:
+            gv = gumbel(uniforms(sample[0], sample[1], b, j, STREAM_DRAFT, vidx))
+            x, lp, g, z = sample_decode(f, gv)
+            key = f + gv
+            lse_out[b, j] = z
+            if fused_out is not None:
+                fused_out[b, j] = f
         amax[b, j], logp[b, j], gap[b, j] = x, lp, g
         if forced is not None:
             xf = int(forced[b, j])
             tokens[b, j] = xf
-            fused_at[b, j] = f[xf]
-            fused_max[b, j] = f[x]
+            fused_at[b, j] = key[xf]
+            fused_max[b, j] = key[x]
             logp_at[b, j] = f[xf] - lse(f)
         else:
             tokens[b, j] = x
@@ -284,4 +303,4 @@ def draft_block(head, long, prior, alpha, beta, forced=None, keep_short=()):
             if (b, j) in keep_short:
                 kept[(b, j)] = S[b].copy()
             record(b, j, f)
-    return DraftResult(tokens, logp, gap, amax, fused_at, fused_max, logp_at, kept or None)
+    return DraftResult(tokens, logp, gap, amax, fused_at, fused_max, logp_at, kept or None, lse_out, fused_out)

@@ -520,3 +520,127 @@ def test_per_position_weights_brute_force_enumeration():
             if ok:
                 consistent.append(blk)
         assert consistent == [tuple(res.tokens[bb])]
+
+
+# ------------------------------------------- temperature 1 (Algorithm 1 Decode ~ softmax)
+
+def test_philox_matches_numpys_philox4x64():
+    """Philox4x64-10 against numpy's Philox bit generator (which adds one to the
+    counter before each block of four outputs)."""
+    rng = np.random.default_rng(5)
+    for _ in range(20):
+        c = [int(x) for x in rng.integers(1, 2 ** 63, size=4, dtype=np.int64)]
+        k = [int(x) for x in rng.integers(0, 2 ** 63, size=2, dtype=np.int64)]
+        bg = np.random.Philox(counter=np.array([c[0] - 1, c[1], c[2], c[3]], dtype=np.uint64),
+                              key=np.array(k, dtype=np.uint64))
+        want = [int(x) for x in bg.random_raw(4)]
+        got = [int(x) for x in oracle.philox4x64_10(np.uint64(c[0]), c[1], c[2], c[3], k[0], k[1])]
+        assert got == want
+
+
+def test_uniforms_lie_on_the_float32_grid_inside_the_unit_interval():
+    u = oracle.uniforms(11, 2, 3, 4, oracle.STREAM_DRAFT, np.arange(4096))
+    scaled = u * 2.0 ** 23 - 0.5
+    assert np.all(scaled == np.round(scaled)) and np.all((u > 0) & (u < 1))
+    assert np.all(u.astype(np.float32).astype(np.float64) == u)
+    assert abs(u.mean() - 0.5) < 0.02
+    # different streams, positions, requests and steps give different variates
+    base = oracle.uniforms(11, 2, 3, 4, 0, np.arange(64))
+    for args in ((11, 2, 3, 4, 1), (11, 2, 3, 5, 0), (11, 2, 4, 4, 0), (11, 3, 3, 4, 0), (12, 2, 3, 4, 0)):
+        assert not np.array_equal(base, oracle.uniforms(*args, np.arange(64)))
+
+
+def _chi2_p(counts, probs):
+    from scipy.stats import chisquare
+    counts = np.asarray(counts, dtype=np.float64)
+    return chisquare(counts, counts.sum() * np.asarray(probs)).pvalue
+
+
+def test_gumbel_max_draws_follow_the_softmax():
+    l = np.array([0.0, 1.0, -1.0, 2.0, 0.5, -3.0])
+    p = np.exp(l - sps.logsumexp(l))
+    counts = np.zeros(l.size)
+    for step in range(6000):
+        g = oracle.gumbel(oracle.uniforms(21, step, 0, 0, oracle.STREAM_DRAFT, np.arange(l.size)))
+        x, lp, gap, z = oracle.sample_decode(l, g)
+        counts[x] += 1
+        assert lp == pytest.approx(l[x] - sps.logsumexp(l)) and z == pytest.approx(sps.logsumexp(l))
+        assert gap >= 0
+    assert _chi2_p(counts, p) > 1e-3
+
+
+def test_speculative_sampling_is_lossless():
+    """The first token the block emits (x_0 if accepted, else the residual draw)
+    is distributed as the target's p_0, whatever the draft's q_0; x_0 is
+    accepted with probability sum_v min(p, q)."""
+    ql = np.array([1.5, 0.0, -0.5, 0.7, -2.0])
+    pl = np.array([0.2, 0.9, -0.3, -1.0, 0.4])
+    pn = np.zeros(5)
+    p = np.exp(pl - sps.logsumexp(pl))
+    q = np.exp(ql - sps.logsumexp(ql))
+    first = np.zeros(5)
+    accepted = 0
+    steps = 6000
+    for step in range(steps):
+        g = oracle.gumbel(oracle.uniforms(33, step, 0, 0, oracle.STREAM_DRAFT, np.arange(5)))
+        x0 = int(np.argmax(ql + g))
+        acc, bonus, info = oracle.verify_sampled([[x0]], ql[None, None, :], np.stack([pl, pn])[None], 33, step)
+        if acc[0] == 1:
+            accepted += 1
+            first[x0] += 1
+        else:
+            first[bonus[0]] += 1
+    assert _chi2_p(first, p) > 1e-3
+    rate = np.minimum(p, q).sum()
+    assert abs(accepted / steps - rate) < 4 * np.sqrt(rate * (1 - rate) / steps)
+
+
+def test_speculative_sampling_special_cases():
+    V = 7
+    rng = np.random.default_rng(2)
+    ql = rng.normal(size=(1, 3, V))
+    # the target equals the draft: every token is accepted, the bonus comes from p_n
+    T = np.concatenate([ql, rng.normal(size=(1, 1, V))], axis=1)
+    for step in range(50):
+        d = [[int(np.argmax(ql[0, j] + oracle.gumbel(oracle.uniforms(4, step, 0, j, 0, np.arange(V)))))
+              for j in range(3)]]
+        acc, bonus, _ = oracle.verify_sampled(d, ql, T, 4, step)
+        key = T[0, 3] + oracle.gumbel(oracle.uniforms(4, step, 0, 3, oracle.STREAM_RESIDUAL, np.arange(V)))
+        assert acc[0] == 3 and bonus[0] == int(np.argmax(key))
+    # a draft token the target rules out (p = 0) is always rejected, and the
+    # residual never gives it back
+    T2 = T.copy()
+    T2[0, 0, 2] = -np.inf
+    for step in range(50):
+        acc, bonus, _ = oracle.verify_sampled([[2, 0, 0]], ql, T2, 5, step)
+        assert acc[0] == 0 and bonus[0] != 2
+
+
+def test_draft_block_temperature_one_draws_with_the_drafting_stream():
+    """Temperature 1: every position is argmax(l + g) of the same fused row as
+    temperature 0, g the drafting-stream variates of (b, j); with a huge gap
+    it agrees with the greedy draft."""
+    base = synth.WORKLOADS["tiny"]
+    w = synth.with_sizes(base, B=2, n=5)
+    d = synth.make_inputs(w)
+    W = {k[5:]: v for k, v in d.items() if k.startswith("head.")}
+    prior = oracle.log_prior(d["counts"])
+    head = oracle.make_head(w.head, W)
+    res = oracle.draft_block(head, d["long"], prior, 0.5, 0.5, sample=(9, 1), keep_fused=True)
+    L = oracle.to_f64(d["long"])
+    for b in range(2):
+        for j in range(5):
+            f = res.fused[b, j]
+            if j == 0:
+                np.testing.assert_array_equal(f, L[b, 0])
+            g = oracle.gumbel(oracle.uniforms(9, 1, b, j, oracle.STREAM_DRAFT, np.arange(w.V)))
+            assert res.tokens[b, j] == int(np.argmax(f + g))
+            assert res.lse[b, j] == pytest.approx(sps.logsumexp(f))
+            assert res.logp[b, j] == pytest.approx(f[res.tokens[b, j]] - sps.logsumexp(f))
+    # the same run forced onto its own tokens reproduces them
+    forced = oracle.draft_block(head, d["long"], prior, 0.5, 0.5, forced=res.tokens, sample=(9, 1))
+    np.testing.assert_array_equal(forced.argmax, res.tokens)
+    # scaled-up logits: the Gumbel noise cannot move the argmax
+    big = oracle.draft_block(head, L * 1e4, prior, 0.0, 0.0, sample=(9, 1))
+    greedy = oracle.draft_block(head, L * 1e4, prior, 0.0, 0.0)
+    np.testing.assert_array_equal(big.tokens, greedy.tokens)
