@@ -253,6 +253,38 @@ int dels_combine_argmax_noalloc(const void* long_logits, const void* short_logit
                                 int32_t* out_token, float* out_logprob, float* out_top2_gap,
                                 dels_stream_t stream);
 
+/* ---- temperature 1 (Algorithm 1 with Decode = a draw from the softmax) --- */
+
+/*
+ * Random numbers. Every uniform is drawn from Philox4x64-10 (Salmon et al.,
+ * "Parallel random numbers: as easy as 1, 2, 3", SC 2011) under the key
+ * (seed, step) with the counter (v / 8, j, b, stream) for vocabulary index v,
+ * block position j, request b and stream (0 drafting, 1 acceptance tests, 2
+ * residual / bonus draws); the 4 output words give 8 32-bit halves, high half
+ * first, for v = 8 (v / 8) .. + 7, and a half h gives u = (floor(h / 2^9) +
+ * 1/2) / 2^23. Draws use the Gumbel-max rule: x = argmax_v (l_v + g_v),
+ * g = -log(-log u). Give each block its own `step`.
+ *
+ * dels_draft_block_sampled: as dels_draft_block_weighted, but every position
+ * is drawn: x_0 ~ softmax(l_L^(0)), x_j ~ softmax(l^(j)).
+ *   out_logprob  [device] [B, n] float32 log softmax(l^(j))[x_j] (required: the
+ *                verification's q_j(x_j));
+ *   out_key_gap  [device] [B, n] float32 key gap k[x_j] - max_{v != x_j} k[v], or NULL;
+ *   draft_state  [device] >= dels_draft_state_bytes(head, B, n), 16-byte aligned,
+ *                or NULL: what dels_verify_block_sampled needs to rebuild a
+ *                rejected position's draft distribution (the LSE of every
+ *                fused row and the vocabulary-projection input of every
+ *                position j >= 1); contents private to the library.
+ *   alpha, beta  [host] [n] float32 per-position weights (entry 0 unused).
+ * Requires d_rank * (2 for bf16 heads, 4 for float32 heads) to be a multiple of 16.
+ */
+size_t dels_draft_state_bytes(const dels_local_head* head, int B, int n);
+int dels_draft_block_sampled(const dels_local_head* head, const void* long_logits, dels_dtype logit_dtype,
+                             const float* log_prior, const float* alpha, const float* beta, int B, int n, int V,
+                             uint64_t seed, uint64_t step, int32_t* out_tokens, float* out_logprob,
+                             float* out_key_gap, void* draft_state, size_t state_bytes, void* workspace,
+                             size_t workspace_bytes, dels_stream_t stream);
+
 /* ---- greedy verification (Algorithm 1, last two steps) ------------------ */
 
 size_t dels_verify_workspace_bytes(int B, int n, int V, dels_dtype dtype);

@@ -22,6 +22,7 @@ __all__ = [
     "DELS_STATUS_NONFINITE", "DELS_STATUS_TIMEOUT", "DELS_STATUS_BAD_TOKEN",
     "DelsError", "LocalHead", "lib", "library_path", "exported_symbols",
     "dels_draft_workspace_bytes", "dels_draft_block", "dels_draft_block_weighted",
+    "dels_draft_state_bytes", "dels_draft_block_sampled",
     "dels_combine_workspace_bytes", "dels_combine_argmax", "dels_combine_argmax_noalloc",
     "dels_verify_workspace_bytes", "dels_verify_block",
     "dels_read_status", "dels_prior_from_counts", "dels_status_string", "dels_version",
@@ -68,6 +69,9 @@ _SIGS = {
                               _vp]),
     "dels_draft_block_weighted": (_i, [ctypes.POINTER(LocalHead), _vp, _i, _vp, _vp, _vp, _i, _i, _i, _vp, _vp, _vp,
                                        _vp, _sz, _vp]),
+    "dels_draft_state_bytes": (_sz, [ctypes.POINTER(LocalHead), _i, _i]),
+    "dels_draft_block_sampled": (_i, [ctypes.POINTER(LocalHead), _vp, _i, _vp, _vp, _vp, _i, _i, _i, ctypes.c_uint64,
+                                      ctypes.c_uint64, _vp, _vp, _vp, _vp, _sz, _vp, _sz, _vp]),
     "dels_combine_workspace_bytes": (_sz, [_i, _i, _i]),
     "dels_combine_argmax": (_i, [_vp, _vp, _i, _vp, _f, _f, _i, _i, _vp, _vp, _vp, _vp, _sz, _vp]),
     "dels_combine_argmax_noalloc": (_i, [_vp, _vp, _i, _vp, _f, _f, _i, _i, _vp, _vp, _vp, _vp]),
@@ -225,6 +229,30 @@ def dels_draft_block_weighted(head: LocalHead, long_logits, logit_dtype: int, lo
                                            ctypes.cast(a, ctypes.c_void_p), ctypes.cast(b, ctypes.c_void_p), B, n, V,
                                            _ptr(out_tokens), _ptr(out_logprob), _ptr(out_top2_gap),
                                            _ptr(workspace), workspace_bytes, _stream(stream))
+
+
+def _host_floats(xs, n):
+    xs = [float(x) for x in xs]
+    if len(xs) != n:
+        raise ValueError(f"expected {n} per-position weights")
+    arr = (ctypes.c_float * n)(*xs)
+    return arr, ctypes.cast(arr, ctypes.c_void_p)
+
+
+def dels_draft_state_bytes(head: LocalHead, B: int, n: int) -> int:
+    return lib().dels_draft_state_bytes(ctypes.byref(head), B, n)
+
+
+def dels_draft_block_sampled(head: LocalHead, long_logits, logit_dtype: int, log_prior, alpha, beta, B: int, n: int,
+                             V: int, seed: int, step: int, out_tokens, out_logprob, out_key_gap, draft_state,
+                             state_bytes: int, workspace, workspace_bytes: int, stream=None) -> int:
+    """Temperature-1 drafting; ``alpha``/``beta`` are sequences of n floats (host)."""
+    a, ap = _host_floats(alpha, n)
+    b, bp = _host_floats(beta, n)
+    return lib().dels_draft_block_sampled(ctypes.byref(head), _ptr(long_logits), logit_dtype, _ptr(log_prior), ap, bp,
+                                          B, n, V, int(seed), int(step), _ptr(out_tokens), _ptr(out_logprob),
+                                          _ptr(out_key_gap), _ptr(draft_state), state_bytes, _ptr(workspace),
+                                          workspace_bytes, _stream(stream))
 
 
 def dels_combine_workspace_bytes(rows: int, V: int, dtype: int) -> int:
@@ -392,6 +420,20 @@ class Drafter:
                                     self.n, self.V, self.tokens, self.logprob, self.gap, self.workspace,
                                     self.ws_bytes, stream), "dels_draft_block")
         return self.tokens, self.logprob, self.gap
+
+    def sample(self, long_logits: torch.Tensor, log_prior: torch.Tensor, alpha, beta, seed: int, step: int,
+               stream=None):
+        """Temperature-1 block: returns (tokens, logprob, key gap, draft state)."""
+        a = list(alpha) if hasattr(alpha, "__len__") else [alpha] * self.n
+        b = list(beta) if hasattr(beta, "__len__") else [beta] * self.n
+        if getattr(self, "state", None) is None:
+            self.state_bytes = dels_draft_state_bytes(self.head, self.B, self.n)
+            self.state = torch.zeros(self.state_bytes, dtype=torch.uint8, device=self.device)
+        _check(dels_draft_block_sampled(self.head, long_logits, dtype_code(long_logits), log_prior, a, b, self.B,
+                                        self.n, self.V, seed, step, self.tokens, self.logprob, self.gap, self.state,
+                                        self.state_bytes, self.workspace, self.ws_bytes, stream),
+               "dels_draft_block_sampled")
+        return self.tokens, self.logprob, self.gap, self.state
 
     def status(self, stream=None) -> int:
         return dels_read_status(self.workspace, stream)

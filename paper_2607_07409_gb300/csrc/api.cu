@@ -476,10 +476,31 @@ T* at(void* ws, size_t off) {
 // Position 0: x_0 = argmax l_L[b, 0, :] as per-chunk records (no merge);
 // returns the number of records per request.
 int position0_rows(const void* long_logits, dels_dtype ldt, int B, int n, int V, void* partials, int partial_ld,
-                   int* status, int sms, cudaStream_t s, int* count) {
+                   int* status, int sms, cudaStream_t s, int* count, const SampleArgs* smp = nullptr) {
   RowsArgs a{};
   const int es = ldt == DELS_F32 ? 4 : 2;
   RowsPlan p = plan_rows(B, V, es, sms, true, partial_ld);
+  if (smp && smp->on) {
+    // temperature 1: x_0 is drawn from softmax(l_L^(0)) (Gumbel-max records)
+    SampleRowsArgs sa{};
+    sa.src = long_logits;
+    sa.ld = (long long)n * V;
+    sa.rows = B;
+    sa.rows_per_request = 1;
+    sa.j0 = 0;
+    sa.V = V;
+    sa.chunk_cols = (int)round_up((size_t)p.chunk_cols, 8);
+    sa.nchunks = (V + sa.chunk_cols - 1) / sa.chunk_cols;
+    sa.vec = ((sa.ld * es) % 16 == 0 && aligned16(long_logits)) ? 1 : 0;
+    sa.seed = smp->seed;
+    sa.step = smp->step;
+    sa.stream = 0;
+    sa.partials = partials;
+    sa.partial_ld = partial_ld;
+    *count = sa.nchunks;
+    { PROF(DELS_KCLASS_POS0); DELS_CUDA(launch_sample_rows(sa, ldt == DELS_F32, s)); }
+    return DELS_OK;
+  }
   a.longp = long_logits;
   a.rows = B;
   a.V = V;
@@ -499,7 +520,8 @@ int position0_rows(const void* long_logits, dels_dtype ldt, int B, int n, int V,
 int draft_position0(const void* long_logits, dels_dtype ldt, int B, int n, int V, void* partials, int partial_ld,
                     int* status, const MergeArgs& merge_base, int sms, cudaStream_t s) {
   int count = 0;
-  const int r = position0_rows(long_logits, ldt, B, n, V, partials, partial_ld, status, sms, s, &count);
+  const int r = position0_rows(long_logits, ldt, B, n, V, partials, partial_ld, status, sms, s, &count,
+                               &merge_base.smp);
   if (r != DELS_OK) return r;
   MergeArgs m = merge_base;
   m.count = count;
@@ -1025,7 +1047,8 @@ namespace {
 int draft_block_impl(const dels_local_head* head, const void* long_logits, dels_dtype logit_dtype,
                      const float* log_prior, float alpha, float beta, const float* alpha_j, const float* beta_j,
                      int B, int n, int V, int32_t* out_tokens, float* out_logprob, float* out_top2_gap,
-                     void* workspace, size_t workspace_bytes, dels_stream_t stream) {
+                     void* workspace, size_t workspace_bytes, dels_stream_t stream,
+                     const SampleArgs* smp = nullptr) {
   auto aw = [&](int j) { return alpha_j ? alpha_j[j] : alpha; };
   auto bw = [&](int j) { return beta_j ? beta_j[j] : beta; };
   int r = validate_draft(head, long_logits, logit_dtype, log_prior, B, n, V, out_tokens, out_logprob, out_top2_gap);
@@ -1055,6 +1078,11 @@ int draft_block_impl(const dels_local_head* head, const void* long_logits, dels_
   mb.table = head->emb;
   mb.table_f32 = bf ? 0 : 1;
   mb.window = 1;
+  // temperature 1 (the kept inputs' source is set per head below)
+  const SampleArgs sm = smp ? *smp : SampleArgs{};
+  mb.smp = sm;
+  mb.smp.R = head->d_rank;
+  mb.smp.r_bytes = es;
 
   switch (head->kind) {
     case DELS_HEAD_GRU: {
@@ -1066,7 +1094,8 @@ int draft_block_impl(const dels_local_head* head, const void* long_logits, dels_
       void* rr = at<void>(workspace, L.r);
       mb.D = D;
       mb.dest = eg;
-      if (bf && persistent_enabled() && !alpha_j && !beta_j && B <= sms && R <= 256) {
+      mb.smp.src_r = rr;
+      if (bf && persistent_enabled() && !alpha_j && !beta_j && !sm.on && B <= sms && R <= 256) {
         // one cooperative launch for the whole block
         Gemm gg, gr, gv;
         if (!plan_store(gg, B, 3 * H, eg, head->w[0], D, hb, head->w[1], H, 128, L.gru_s0, L.gru_s1, ACT_NONE,
@@ -1119,7 +1148,7 @@ int draft_block_impl(const dels_local_head* head, const void* long_logits, dels_
         }
       }
       const float* G = static_cast<const float*>(head->w[3]);
-      if (bf && G && fused_products_enabled() && B <= 64) {
+      if (bf && G && fused_products_enabled() && !sm.on && B <= 64) {
         // Input-table path, fused variant (DELS_DRAFT_FUSED=1): two launches
         // per position —
         //   gates(j)        merge x_{j-1} from the previous position's records,
@@ -1215,7 +1244,8 @@ int draft_block_impl(const dels_local_head* head, const void* long_logits, dels_
         mb.table = nullptr;
         if (n == 1) return draft_position0(long_logits, logit_dtype, B, n, V, partials, L.partial_ld, status, mb, sms, s);
         int count = 0;
-        r = position0_rows(long_logits, logit_dtype, B, n, V, partials, L.partial_ld, status, sms, s, &count);
+        r = position0_rows(long_logits, logit_dtype, B, n, V, partials, L.partial_ld, status, sms, s, &count,
+                           &mb.smp);
         if (r != DELS_OK) return r;
         Gemm gr, gh, gv;
         if (!plan_store(gr, B, R, hb, head->w[2], H, nullptr, nullptr, 0, kRankTile, kRankSplits, 0, ACT_SILU,
@@ -1254,6 +1284,7 @@ int draft_block_impl(const dels_local_head* head, const void* long_logits, dels_
         ga.h = h;
         ga.h_bf16 = hb;
         ga.status = status;
+        ga.smp = mb.smp;
         for (int j = 1; j < n; ++j) {
           ga.count = j == 1 ? count : gv.grid;
           ga.jprev = j - 1;
@@ -1263,8 +1294,9 @@ int draft_block_impl(const dels_local_head* head, const void* long_logits, dels_
             DELS_CUDA(launch_tc_gemm(gr.a, &gr.mA0, &gr.mB0, &gr.mA1, &gr.mB1, &gr.mL, gr.grid, gr.smem, s,
                                      j + 1 < n ? &hh : nullptr)); }
           gv.a.j = j;
-        gv.a.alpha = aw(j);
-        gv.a.beta = bw(j);
+          gv.a.sample = sm.on;
+          gv.a.seed = sm.seed;
+          gv.a.step = sm.step;
           gv.a.alpha = aw(j);
           gv.a.beta = bw(j);
           { PROF(DELS_KCLASS_VOCAB_COMBINE); DELS_CUDA(run(gv, s)); }
@@ -1300,8 +1332,9 @@ int draft_block_impl(const dels_local_head* head, const void* long_logits, dels_
           { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_gru_gates(gpart, gg.a.seg_splits[0], gg.a.seg_splits[1], B, H, h, hb, s)); }
           { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run(gr, s)); }
           gv.a.j = j;
-        gv.a.alpha = aw(j);
-        gv.a.beta = bw(j);
+          gv.a.sample = sm.on;
+          gv.a.seed = sm.seed;
+          gv.a.step = sm.step;
           gv.a.alpha = aw(j);
           gv.a.beta = bw(j);
           { PROF(DELS_KCLASS_VOCAB_COMBINE); DELS_CUDA(run(gv, s)); }
@@ -1327,7 +1360,7 @@ int draft_block_impl(const dels_local_head* head, const void* long_logits, dels_
                                              static_cast<const uint8_t*>(long_logits) +
                                                  (size_t)j * V * (logit_dtype == DELS_F32 ? 4 : 2),
                                              logit_dtype == DELS_F32, (long long)n * V, log_prior, aw(j), bw(j), B, V,
-                                             partials, L.partial_ld, nch, status, s)); }
+                                             partials, L.partial_ld, nch, status, s, &sm, j)); }
           MergeArgs m = mb;
           m.count = nch;
           m.j = j;
@@ -1347,6 +1380,7 @@ int draft_block_impl(const dels_local_head* head, const void* long_logits, dels_
       mb.D = D;
       mb.window = W;
       mb.dest = u;
+      mb.smp.src_r = feat;
       r = draft_position0(long_logits, logit_dtype, B, n, V, partials, L.partial_ld, status, mb, sms, s);
       if (r != DELS_OK || n == 1) return r;
       if (bf) {
@@ -1371,8 +1405,9 @@ int draft_block_impl(const dels_local_head* head, const void* long_logits, dels_
                                            static_cast<uint16_t*>(h2), Hd, s)); }
           }
           gv.a.j = j;
-        gv.a.alpha = aw(j);
-        gv.a.beta = bw(j);
+          gv.a.sample = sm.on;
+          gv.a.seed = sm.seed;
+          gv.a.step = sm.step;
           gv.a.alpha = aw(j);
           gv.a.beta = bw(j);
           { PROF(DELS_KCLASS_VOCAB_COMBINE); DELS_CUDA(run(gv, s)); }
@@ -1395,7 +1430,7 @@ int draft_block_impl(const dels_local_head* head, const void* long_logits, dels_
                                              static_cast<const uint8_t*>(long_logits) +
                                                  (size_t)j * V * (logit_dtype == DELS_F32 ? 4 : 2),
                                              logit_dtype == DELS_F32, (long long)n * V, log_prior, aw(j), bw(j), B, V,
-                                             partials, L.partial_ld, nch, status, s)); }
+                                             partials, L.partial_ld, nch, status, s, &sm, j)); }
           MergeArgs m = mb;
           m.count = nch;
           m.j = j;
@@ -1422,6 +1457,7 @@ int draft_block_impl(const dels_local_head* head, const void* long_logits, dels_
       uint16_t* feat = at<uint16_t>(workspace, L.feat);
       mb.D = D;
       mb.dest = ex;
+      mb.smp.src_r = feat;
       r = draft_position0(long_logits, logit_dtype, B, n, V, partials, L.partial_ld, status, mb, sms, s);
       if (r != DELS_OK || n == 1) return r;
       Gemm gq, gk, gvv, go, g1, g2, gv;
@@ -1462,6 +1498,9 @@ int draft_block_impl(const dels_local_head* head, const void* long_logits, dels_
         { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_splitk_finish(xpart, g2.a.total_splits, B, D, uu, ACT_NONE, y, D, nullptr, 0, s)); }
         { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_rmsnorm_bf16(y, B, D, D, feat, s)); }
         gv.a.j = j;
+          gv.a.sample = sm.on;
+          gv.a.seed = sm.seed;
+          gv.a.step = sm.step;
         gv.a.alpha = aw(j);
         gv.a.beta = bw(j);
         { PROF(DELS_KCLASS_VOCAB_COMBINE); DELS_CUDA(run(gv, s)); }
@@ -1478,6 +1517,7 @@ int draft_block_impl(const dels_local_head* head, const void* long_logits, dels_
       void* feat = at<void>(workspace, L.mk);
       mb.D = R;
       mb.dest = feat;
+      mb.smp.src_r = feat;
       r = draft_position0(long_logits, logit_dtype, B, n, V, partials, L.partial_ld, status, mb, sms, s);
       if (r != DELS_OK || n == 1) return r;
       Gemm gv;
@@ -1489,8 +1529,9 @@ int draft_block_impl(const dels_local_head* head, const void* long_logits, dels_
         int count;
         if (bf) {
           gv.a.j = j;
-        gv.a.alpha = aw(j);
-        gv.a.beta = bw(j);
+          gv.a.sample = sm.on;
+          gv.a.seed = sm.seed;
+          gv.a.step = sm.step;
           gv.a.alpha = aw(j);
           gv.a.beta = bw(j);
           { PROF(DELS_KCLASS_VOCAB_COMBINE); DELS_CUDA(run(gv, s)); }
@@ -1501,7 +1542,7 @@ int draft_block_impl(const dels_local_head* head, const void* long_logits, dels_
                                              static_cast<const uint8_t*>(long_logits) +
                                                  (size_t)j * V * (logit_dtype == DELS_F32 ? 4 : 2),
                                              logit_dtype == DELS_F32, (long long)n * V, log_prior, aw(j), bw(j), B, V,
-                                             partials, L.partial_ld, nch, status, s)); }
+                                             partials, L.partial_ld, nch, status, s, &sm, j)); }
           count = nch;
         }
         MergeArgs m = mb;
@@ -1528,6 +1569,37 @@ int dels_draft_block(const dels_local_head* head, const void* long_logits, dels_
                      dels_stream_t stream) {
   return draft_block_impl(head, long_logits, logit_dtype, log_prior, alpha, beta, nullptr, nullptr, B, n, V,
                           out_tokens, out_logprob, out_top2_gap, workspace, workspace_bytes, stream);
+}
+
+size_t dels_draft_state_bytes(const dels_local_head* head, int B, int n) {
+  if (!head || B < 0 || n < 1) return 0;
+  const size_t es = head->wdtype == DELS_BF16 ? 2 : 4;
+  return round_up((size_t)B * n * 4, 256) + (size_t)B * n * (size_t)head->d_rank * es;
+}
+
+int dels_draft_block_sampled(const dels_local_head* head, const void* long_logits, dels_dtype logit_dtype,
+                             const float* log_prior, const float* alpha, const float* beta, int B, int n, int V,
+                             uint64_t seed, uint64_t step, int32_t* out_tokens, float* out_logprob,
+                             float* out_key_gap, void* draft_state, size_t state_bytes, void* workspace,
+                             size_t workspace_bytes, dels_stream_t stream) {
+  if (!head || !alpha || !beta || !out_logprob) return DELS_ERR_NULL_POINTER;
+  if (n < 1 || n > 32 || B < 0) return DELS_ERR_BAD_SHAPE;
+  for (int j = 0; j < n; ++j)
+    if (!std::isfinite(alpha[j]) || !std::isfinite(beta[j])) return DELS_ERR_BAD_SHAPE;
+  const size_t es = head->wdtype == DELS_BF16 ? 2 : 4;
+  if (((size_t)head->d_rank * es) % 16 != 0) return DELS_ERR_UNSUPPORTED;
+  if (draft_state) {
+    if (state_bytes < dels_draft_state_bytes(head, B, n)) return DELS_ERR_WORKSPACE;
+    if (!aligned16(draft_state)) return DELS_ERR_ALIGNMENT;
+  }
+  SampleArgs sm{};
+  sm.on = 1;
+  sm.seed = seed;
+  sm.step = step;
+  sm.out_lse = static_cast<float*>(draft_state);
+  sm.state_r = draft_state ? static_cast<uint8_t*>(draft_state) + round_up((size_t)B * n * 4, 256) : nullptr;
+  return draft_block_impl(head, long_logits, logit_dtype, log_prior, 0.f, 0.f, alpha, beta, B, n, V, out_tokens,
+                          out_logprob, out_key_gap, workspace, workspace_bytes, stream, &sm);
 }
 
 int dels_draft_block_weighted(const dels_local_head* head, const void* long_logits, dels_dtype logit_dtype,

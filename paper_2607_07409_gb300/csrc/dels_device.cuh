@@ -170,6 +170,128 @@ __device__ __forceinline__ void write_decode(const RowAcc& r, long long out_i, i
   if (gap) gap[out_i] = ok ? (r.m - r.second) : NAN;
 }
 
+// ----------------------------------------------------------------------------
+// temperature 1: Gumbel-max draws with Philox4x64-10 uniforms
+// ----------------------------------------------------------------------------
+// Philox4x64-10 (Salmon, Moraes, Dror and Shaw, "Parallel random numbers: as
+// easy as 1, 2, 3", SC 2011): ten rounds of two 64 x 64 -> 128-bit products
+// on a 4-word counter, the key bumped by two Weyl constants between rounds.
+constexpr uint64_t kPhiloxM0 = 0xD2E7470EE14C6C93ull, kPhiloxM1 = 0xCA5A826395121157ull;
+constexpr uint64_t kPhiloxW0 = 0x9E3779B97F4A7C15ull, kPhiloxW1 = 0xBB67AE8584CAA73Bull;
+enum { kStreamDraft = 0, kStreamAccept = 1, kStreamResidual = 2 };
+
+__device__ __forceinline__ void philox4x64_10(uint64_t (&x)[4], uint64_t k0, uint64_t k1) {
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    const uint64_t hi0 = __umul64hi(kPhiloxM0, x[0]), lo0 = kPhiloxM0 * x[0];
+    const uint64_t hi1 = __umul64hi(kPhiloxM1, x[2]), lo1 = kPhiloxM1 * x[2];
+    const uint64_t y0 = hi1 ^ x[1] ^ k0, y2 = hi0 ^ x[3] ^ k1;
+    x[0] = y0;
+    x[1] = lo1;
+    x[2] = y2;
+    x[3] = lo0;
+    k0 += kPhiloxW0;
+    k1 += kPhiloxW1;
+  }
+}
+
+// A 32-bit half h gives u = (floor(h / 2^9) + 1/2) / 2^23, exact in float32.
+__device__ __forceinline__ float uniform_from_bits(uint32_t h) {
+  return (float)(2u * (h >> 9) + 1u) * 5.9604644775390625e-08f;   // (2k + 1) * 2^-24
+}
+
+// Standard Gumbel variate -log(-log u): the inner log at full precision (it
+// decides how close to 1 u may be), the outer one through the fast log.
+__device__ __forceinline__ float gumbel_from_bits(uint32_t h) { return -__logf(-logf(uniform_from_bits(h))); }
+
+// Counter (v / 8, j, b, stream), key (seed, step): the 8 uniforms of
+// vocabulary indices 8c .. 8c + 7 are the halves of the 4 output words, high
+// half first.
+__device__ __forceinline__ void philox_block(uint64_t seed, uint64_t step, int b, int j, int stream, long long c,
+                                             uint64_t (&x)[4]) {
+  x[0] = (uint64_t)c;
+  x[1] = (uint64_t)j;
+  x[2] = (uint64_t)b;
+  x[3] = (uint64_t)stream;
+  philox4x64_10(x, seed, step);
+}
+
+__device__ __forceinline__ void gumbel8(uint64_t seed, uint64_t step, int b, int j, int stream, long long c,
+                                        float (&g)[8]) {
+  uint64_t x[4];
+  philox_block(seed, step, b, j, stream, c, x);
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    g[2 * k] = gumbel_from_bits((uint32_t)(x[k] >> 32));
+    g[2 * k + 1] = gumbel_from_bits((uint32_t)x[k]);
+  }
+}
+
+__device__ __forceinline__ uint32_t philox_half_at(uint64_t seed, uint64_t step, int b, int j, int stream,
+                                                   long long v) {
+  uint64_t x[4];
+  philox_block(seed, step, b, j, stream, v >> 3, x);
+  const int w = (int)((v & 7) >> 1);
+  const uint64_t word = w == 0 ? x[0] : w == 1 ? x[1] : w == 2 ? x[2] : x[3];
+  return (v & 1) ? (uint32_t)word : (uint32_t)(word >> 32);
+}
+
+__device__ __forceinline__ float gumbel_at(uint64_t seed, uint64_t step, int b, int j, int stream, long long v) {
+  return gumbel_from_bits(philox_half_at(seed, step, b, j, stream, v));
+}
+
+__device__ __forceinline__ float uniform_at(uint64_t seed, uint64_t step, int b, int j, int stream, long long v) {
+  return uniform_from_bits(philox_half_at(seed, step, b, j, stream, v));
+}
+
+// A record of temperature-1 drafting holds the largest key k = l + g, its
+// index and the runner-up key, and s = sum_v exp(l_v - k_max): the key max
+// is at least l_v + g_v, and g > -2.82 for these uniforms, so no term
+// exceeds e^2.82. LSE(l) = k_max + log s and log softmax(l)[x] = -g_x - log s.
+__device__ __forceinline__ bool rowacc_valid_sampled(const RowAcc& a) {
+  return a.m > -INFINITY && a.m < INFINITY && a.s == a.s && a.s > 0.f && a.s < INFINITY;
+}
+
+__device__ __forceinline__ void write_decode_sampled(const RowAcc& r, long long out_i, int32_t* tok, float* lp,
+                                                     float* gap, float* lse, int* status, float g_idx) {
+  const bool ok = rowacc_valid_sampled(r);
+  if (!ok) raise_status(status, DELS_STATUS_NONFINITE);
+  tok[out_i] = ok ? r.idx : -1;
+  const float ls = logf(r.s);
+  if (lp) lp[out_i] = ok ? -g_idx - ls : NAN;
+  if (gap) gap[out_i] = ok ? (r.m - r.second) : NAN;
+  if (lse) lse[out_i] = ok ? r.m + ls : NAN;
+}
+
+// Decode of a merged record of position j for request b at either temperature;
+// returns the token (-1 for an invalid row).
+__device__ __forceinline__ int decode_record(const RowAcc& x, const SampleArgs& smp, int b, int n, int j,
+                                             int32_t* tok, float* lp, float* gap, int* status) {
+  const long long o = (long long)b * n + j;
+  if (!smp.on) {
+    write_decode(x, o, tok, lp, gap, status);
+    return rowacc_valid(x) ? x.idx : -1;
+  }
+  const bool ok = rowacc_valid_sampled(x);
+  const float gx = ok ? gumbel_at(smp.seed, smp.step, b, j, kStreamDraft, x.idx) : 0.f;
+  write_decode_sampled(x, o, tok, lp, gap, smp.out_lse, status, gx);
+  return ok ? x.idx : -1;
+}
+
+// Temperature-1 drafting keeps the vocabulary-projection input of every
+// position j >= 1 for the verification's residual row: row b of `src_r`
+// ([B][R] elements of r_bytes) goes to state_r[b][j]. Called by one CTA per
+// request with all its threads.
+__device__ __forceinline__ void keep_draft_input(const SampleArgs& smp, int b, int n, int j) {
+  if (!smp.on || !smp.state_r || j < 1) return;
+  const int vecs = smp.R * smp.r_bytes / 16;   // R * r_bytes is a multiple of 16
+  const uint4* src = reinterpret_cast<const uint4*>(static_cast<const uint8_t*>(smp.src_r) +
+                                                    (long long)b * smp.R * smp.r_bytes);
+  uint4* dst = reinterpret_cast<uint4*>(static_cast<uint8_t*>(smp.state_r) +
+                                        ((long long)b * n + j) * smp.R * smp.r_bytes);
+  for (int i = threadIdx.x; i < vecs; i += blockDim.x) dst[i] = __ldcg(src + i);
+}
+
 // Argmax-only update (verification): value and lowest index.
 __device__ __forceinline__ void argmax_push(float x, int v, float& best, int& idx, bool& nan_seen) {
   const bool gt = x > best;

@@ -91,6 +91,31 @@ cudaError_t launch_combine_rows(const RowsArgs& a, dels_dtype dt, bool vec, bool
 cudaError_t launch_verify_rows(const RowsArgs& a, dels_dtype dt, bool vec, cudaStream_t s);
 
 // ---- draft merge + gather of the next local-head input ----------------------
+// Temperature-1 drafting (on = 0: temperature 0). The uniforms of (request
+// b, position j, stream, vocabulary index) come from Philox4x64-10 under the
+// key (seed, step).
+struct SampleArgs {
+  int on;
+  unsigned long long seed, step;
+  float* out_lse;                // [B, n] LSE of the fused row, or null
+  void* state_r;                 // [B][n][R] kept vocabulary-projection inputs, or null
+  const void* src_r;             // [B][R] the current position's input
+  int R, r_bytes;                // elements per row and bytes per element
+};
+
+// Records of Gumbel-max keys over logit rows (temperature 1).
+struct SampleRowsArgs {
+  const void* src;               // row r starts at src + r * ld (elements)
+  long long ld;
+  int rows, rows_per_request, j0;
+  int V, chunk_cols, nchunks, vec;
+  unsigned long long seed, step;
+  int stream;
+  void* partials;                // [rows][partial_ld] RowAcc
+  int partial_ld;
+};
+cudaError_t launch_sample_rows(const SampleRowsArgs& a, bool f32, cudaStream_t s);
+
 struct MergeArgs {
   const void* partials;          // [B][partial_ld] RowAcc
   int partial_ld, count;
@@ -108,6 +133,7 @@ struct MergeArgs {
   float* zero_f32;               // [B, zero_len]
   uint16_t* zero_bf16;           // [B, zero_len]
   int zero_len;
+  SampleArgs smp;
 };
 cudaError_t launch_draft_merge(const MergeArgs& a, cudaStream_t s);
 
@@ -149,6 +175,9 @@ struct TcGemmArgs {
   int partial_ld;
   int* status;
   int debug_skip_producer;       // test hook: producer never fills (exercises the bounded waits)
+  // EPI_COMBINE at temperature 1: Gumbel-max keys (Philox4x64-10 under (seed, step))
+  int sample;
+  unsigned long long seed, step;
   // EPI_STORE, optional: the K splits of one output tile run on the CTAs of
   // one thread-block cluster (cluster_k CTAs, split = rank in the cluster);
   // the others send their accumulators to rank 0 through distributed shared
@@ -237,6 +266,7 @@ struct GatesTableArgs {
   float* h;                      // [B, H]
   uint16_t* h_bf16;              // [B, H]
   int* status;
+  SampleArgs smp;
 };
 cudaError_t launch_gru_gates_table(const GatesTableArgs& a, cudaStream_t s);
 cudaError_t launch_splitk_finish(const float* part, int S, int B, int O, const float* residual, int act,
@@ -251,7 +281,8 @@ cudaError_t launch_gemv_f32(const float* X, int ldx, const float* W, int B, int 
 cudaError_t launch_vocab_combine_f32(const float* feat, int K, const float* Wv, const void* longp, int long_f32,
                                      long long ld_long, const float* prior, float alpha, float beta, int B,
                                      int V, void* partials, int partial_ld, int nchunks, int* status,
-                                     cudaStream_t s);
+                                     cudaStream_t s,
+                                     const SampleArgs* smp = nullptr, int j = 0);
 
 // ---- host utilities ---------------------------------------------------------
 int device_sm_count();

@@ -119,10 +119,18 @@ __global__ void __launch_bounds__(kGatesThreads) k_gru_gates_table(GatesTableArg
     }
     x = rowacc_warp_reduce(x);
     if (lane == 0) {
-      s_tok = rowacc_valid(x) ? x.idx : -1;
-      if (blockIdx.y == 0) write_decode(x, (long long)b * a.n + a.jprev, a.tokens, a.out_lp, a.out_gap, a.status);
+      if (!a.smp.on) {
+        s_tok = rowacc_valid(x) ? x.idx : -1;
+        if (blockIdx.y == 0) write_decode(x, (long long)b * a.n + a.jprev, a.tokens, a.out_lp, a.out_gap, a.status);
+      } else if (blockIdx.y == 0) {
+        s_tok = decode_record(x, a.smp, b, a.n, a.jprev, a.tokens, a.out_lp, a.out_gap, a.status);
+      } else {
+        s_tok = rowacc_valid_sampled(x) ? x.idx : -1;
+      }
     }
   }
+  // temperature 1: keep r_{jprev} (not yet overwritten: the next products launch follows this one)
+  if (blockIdx.y == 0) keep_draft_input(a.smp, b, a.n, a.jprev);
   __syncthreads();
   if (!live) return;
   const int tok = s_tok;
@@ -292,7 +300,7 @@ __global__ void __launch_bounds__(256) k_vocab_combine_f32(const float* __restri
                                                            int long_f32, long long ld_long,
                                                            const float* __restrict__ prior, float alpha, float beta,
                                                            int V, void* partials, int partial_ld, int nchunks,
-                                                           int* status) {
+                                                           int* status, SampleArgs smp, int j) {
   if (threadIdx.x == 0) pdl_trigger();
   pdl_wait();
   const int chunk = blockIdx.x % nchunks, b = blockIdx.x / nchunks;
@@ -311,7 +319,9 @@ __global__ void __launch_bounds__(256) k_vocab_combine_f32(const float* __restri
     const float l = long_f32 ? static_cast<const float*>(longp)[(long long)b * ld_long + v]
                              : bf16_to_f(static_cast<const uint16_t*>(longp)[(long long)b * ld_long + v]);
     float f[1] = {fmaf(-beta, prior[v], fmaf(alpha, d, l))};
-    top2_push(f[0], v, best, second, idx);
+    // temperature 1: the top-2 over the keys f + g (see write_decode_sampled)
+    const float key = smp.on ? f[0] + gumbel_at(smp.seed, smp.step, b, j, kStreamDraft, v) : f[0];
+    top2_push(key, v, best, second, idx);
     lse_chunk<1>(f, best, m, s);
   }
   RowAcc r;
@@ -377,9 +387,11 @@ cudaError_t launch_gemv_f32(const float* X, int ldx, const float* W, int B, int 
 
 cudaError_t launch_vocab_combine_f32(const float* feat, int K, const float* Wv, const void* longp, int long_f32,
                                      long long ld_long, const float* prior, float alpha, float beta, int B, int V,
-                                     void* partials, int partial_ld, int nchunks, int* status, cudaStream_t s) {
+                                     void* partials, int partial_ld, int nchunks, int* status, cudaStream_t s,
+                                     const SampleArgs* smp, int j) {
+  const SampleArgs sm = smp ? *smp : SampleArgs{};
   return launch_pdl(k_vocab_combine_f32, dim3(B * nchunks), dim3(256), 0, s, feat, K, Wv, longp, long_f32, ld_long,
-                    prior, alpha, beta, V, partials, partial_ld, nchunks, status);
+                    prior, alpha, beta, V, partials, partial_ld, nchunks, status, sm, j);
 }
 
 }  // namespace dels

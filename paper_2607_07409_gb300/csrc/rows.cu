@@ -436,15 +436,14 @@ __global__ void __launch_bounds__(256) k_draft_merge(MergeArgs a) {
     x = rowacc_merge(x, ld_rowacc_cg(a.partials, (long long)b * a.partial_ld + k));
   x = rowacc_warp_reduce(x);
   if (lane == 0) red[warp] = x;
+  // temperature 1: keep this position's vocabulary-projection input before
+  // the gather below may overwrite it (the Markov head gathers into it)
+  keep_draft_input(a.smp, b, a.n, a.j);
   __syncthreads();
   if (warp == 0) {
     x = lane < (int)(blockDim.x >> 5) ? red[lane] : rowacc_init();
     x = rowacc_warp_reduce(x);
-    if (lane == 0) {
-      const long long o = (long long)b * a.n + a.j;
-      write_decode(x, o, a.tokens, a.out_lp, a.out_gap, a.status);
-      s_tok = rowacc_valid(x) ? x.idx : -1;
-    }
+    if (lane == 0) s_tok = decode_record(x, a.smp, b, a.n, a.j, a.tokens, a.out_lp, a.out_gap, a.status);
   }
   __syncthreads();
   if (a.table == nullptr) return;

@@ -316,10 +316,14 @@ __device__ __forceinline__ bool mma_run(const Ctx& c, const Phase& p, MmaState& 
 // then top-1/top-2 and the online log-sum-exp. `lrow` is this row's 128-byte
 // line of the logits box holding the chunk, `half` selects the chunk's
 // 64-byte half (bf16) and `ptile` the prior of the chunk's columns.
+// SAMPLE (temperature 1): the top-2 runs over the keys k = f + g, g the
+// drafting-stream Gumbel variates of (row b, position j, column), and the
+// sum over exp(f - k_max) (see write_decode_sampled).
+template <bool SAMPLE = false>
 __device__ __forceinline__ void combine_chunk(const float (&acc)[32], const uint8_t* lrow, int half, int swz,
                                               bool long_f32, const float* ptile, int cbase, int V, float alpha,
                                               float nbeta, float& best, float& second, int& idx, float& m,
-                                              float& ssum) {
+                                              float& ssum, const TcGemmArgs* sa = nullptr, int b = 0) {
   float f[32];
   if (!long_f32) {
 #pragma unroll
@@ -352,8 +356,19 @@ __device__ __forceinline__ void combine_chunk(const float (&acc)[32], const uint
     for (int i = 0; i < 32; ++i)
       if (cbase + i >= V) f[i] = -INFINITY;
   }
+  if (SAMPLE) {
+    // cbase is a multiple of 32: four Philox blocks of 8 columns
 #pragma unroll
-  for (int i = 0; i < 32; ++i) top2_push(f[i], cbase + i, best, second, idx);
+    for (int t = 0; t < 4; ++t) {
+      float g[8];
+      gumbel8(sa->seed, sa->step, b, sa->j, kStreamDraft, (cbase >> 3) + t, g);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) top2_push(f[t * 8 + i] + g[i], cbase + t * 8 + i, best, second, idx);
+    }
+  } else {
+#pragma unroll
+    for (int i = 0; i < 32; ++i) top2_push(f[i], cbase + i, best, second, idx);
+  }
   lse_chunk_ex2<32>(f, best, m, ssum);
 }
 
@@ -379,7 +394,7 @@ __device__ __forceinline__ void epi_stage_prior(const Ctx& c, const Phase& p, in
 // index under which combine partials are published.
 // COMB: the phase is a combine phase (EPI_COMBINE); a compile-time flag so
 // that a store-only kernel carries none of the combine's registers.
-template <bool COMB>
+template <bool COMB, bool SAMPLE = false>
 __device__ __forceinline__ bool epi_run(const Ctx& c, const Phase& p, EpiState& st, int warp, int lane, int cta) {
   const TcGemmArgs& a = *p.a;
   constexpr bool comb = COMB;
@@ -422,12 +437,12 @@ __device__ __forceinline__ bool epi_run(const Ctx& c, const Phase& p, EpiState& 
       auto run_chunk = [&](const float (&acc)[32], int cc) {
         if (!a.long_f32) {
           // bf16 boxes of 64 columns: chunk cc is half (cc & 1) of box (cc >> 1)
-          combine_chunk(acc, lbuf + (cc >> 1) * box_bytes + br * 128, cc & 1, swz, false, ptile + cc * 32,
-                        it.o0 + cc * 32, a.V, alpha, nbeta, best, second, idx, m, ssum);
+          combine_chunk<SAMPLE>(acc, lbuf + (cc >> 1) * box_bytes + br * 128, cc & 1, swz, false, ptile + cc * 32,
+                                it.o0 + cc * 32, a.V, alpha, nbeta, best, second, idx, m, ssum, &a, b);
         } else {
           // f32 boxes of 32 columns: chunk cc is box cc
-          combine_chunk(acc, lbuf + cc * box_bytes + br * 128, 0, swz, true, ptile + cc * 32, it.o0 + cc * 32, a.V,
-                        alpha, nbeta, best, second, idx, m, ssum);
+          combine_chunk<SAMPLE>(acc, lbuf + cc * box_bytes + br * 128, 0, swz, true, ptile + cc * 32,
+                                it.o0 + cc * 32, a.V, alpha, nbeta, best, second, idx, m, ssum, &a, b);
         }
       };
       if (c1 < nchunk) {

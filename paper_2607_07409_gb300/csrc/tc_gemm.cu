@@ -140,12 +140,12 @@ __device__ __forceinline__ void epi_cluster_finish(const Ctx& c, const TcGemmArg
   }
 }
 
-// COMB: combine launches (one CTA per SM, the combine epilogue's registers);
-// store launches are compiled separately with at most 2 x 352 threads' worth
-// of registers per SM, so that a store launch's CTAs can share an SM with the
-// small kernels around them.
-template <bool COMB>
-__global__ void __launch_bounds__(kThreads, COMB ? 1 : 2)
+// MODE 1 / 2: combine launches at temperature 0 / 1 (one CTA per SM, the
+// combine epilogue's registers); MODE 0: store launches, compiled separately
+// with at most 2 x 352 threads' worth of registers per SM, so that a store
+// launch's CTAs can share an SM with the small kernels around them.
+template <int MODE>
+__global__ void __launch_bounds__(kThreads, MODE != 0 ? 1 : 2)
     k_tc_gemm(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ CUtensorMap mB0,
               const __grid_constant__ CUtensorMap mA1, const __grid_constant__ CUtensorMap mB1,
               const __grid_constant__ CUtensorMap mL, const __grid_constant__ TcGemmArgs a0,
@@ -161,7 +161,7 @@ __global__ void __launch_bounds__(kThreads, COMB ? 1 : 2)
   const int ncta = second ? (int)gridDim.x - grid0 : grid0;
   const Smem lay = smem_layout(a);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  constexpr bool comb = COMB;
+  constexpr bool comb = MODE != 0;
 
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + lay.bar_off);
   Ctx c;
@@ -287,7 +287,7 @@ __global__ void __launch_bounds__(kThreads, COMB ? 1 : 2)
       if (p.count > 0) epi_cluster_send(c, a, smem_u32(smem + lay.clus_off), warp, lane, cluster_ctarank());
     } else {
       EpiState st;
-      epi_run<COMB>(c, p, st, warp, lane, cta);
+      epi_run<MODE != 0, MODE == 2>(c, p, st, warp, lane, cta);
     }
   }
 
@@ -324,16 +324,17 @@ cudaError_t launch_tc_gemm(const TcGemmArgs& a, const CUtensorMap* mA0, const CU
   // it once per device to the largest request seen.
   const bool comb = a.epi == EPI_COMBINE;
   if (two && (second->a->epi == EPI_COMBINE) != comb) return cudaErrorInvalidValue;
-  auto kern = comb ? k_tc_gemm<true> : k_tc_gemm<false>;
-  static int configured_bytes[2][64] = {{0}};
+  const int mode = comb ? (a.sample ? 2 : 1) : 0;
+  auto kern = mode == 2 ? k_tc_gemm<2> : mode == 1 ? k_tc_gemm<1> : k_tc_gemm<0>;
+  static int configured_bytes[3][64] = {{0}};
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
-  if ((int)smem_bytes > configured_bytes[comb][dev]) {
+  if ((int)smem_bytes > configured_bytes[mode][dev]) {
     e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_bytes);
     if (e != cudaSuccess) return e;
-    configured_bytes[comb][dev] = (int)smem_bytes;
+    configured_bytes[mode][dev] = (int)smem_bytes;
   }
   const uint64_t budget = a.debug_skip_producer ? 100000000ull : kWaitBudgetNs;
   const int g0 = std::max(grid, 0);

@@ -58,13 +58,14 @@ def check_rows(tok, lp, gap, ref_tok, ref_lp, ref_gap, lp_tol=LP_TOL_COMBINE, ex
     return dict(ties=int(ties.sum()), flips=int((~same).sum()), lp_err=float(err))
 
 
-def check_draft(tok, lp, gap, head, long, prior, alpha, beta, lp_tol):
+def check_draft(tok, lp, gap, head, long, prior, alpha, beta, lp_tol, sample=None):
     """Block drafting parity via the oracle's forced-prefix mode; also checks
     that the free-running oracle reproduces the device block exactly when no
-    position had a near-tie."""
+    position had a near-tie. ``sample=(seed, step)``: temperature 1 (the
+    token rule and the gap then refer to the Gumbel-max keys l + g)."""
     tok = np.asarray(tok)
     lp = np.asarray(lp)
-    ref = oracle.draft_block(head, long, prior, alpha, beta, forced=tok)
+    ref = oracle.draft_block(head, long, prior, alpha, beta, forced=tok, sample=sample)
     same = tok == ref.argmax
     ties = ref.gap < TIE_EPS
     bad = ~same & ~(ties & (ref.fused_at >= ref.fused_max - TIE_EPS))
@@ -79,4 +80,4 @@ def check_draft(tok, lp, gap, head, long, prior, alpha, beta, lp_tol):
     if not ties.any():
         # no near-tie anywhere: the device block is the oracle's own block
         assert same.all()
-    return dict(ties=int(ties.sum()), flips=int((~same).sum()), lp_err=err, gap_err=gerr)
+    return dict(ties=int(ties.sum()), flips=int((~same).sum()), lp_err=err, gap_err=gerr, ref=ref)

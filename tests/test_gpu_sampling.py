@@ -1,0 +1,79 @@
+"""GPU parity of temperature-1 drafting (Algorithm 1 with Decode = a draw from
+the softmax by the Gumbel-max rule) against the oracle.
+
+Both sides draw the same Philox4x64-10 uniforms, so a device token must be
+the oracle's argmax of the keys l + g at every position, except where the
+oracle's top-2 key gap is a near-tie (then within the tie tolerance of the
+maximum key); the drafted prefix is re-checked in the oracle's forced mode.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+import paper_2607_07409_gb300 as dels
+from parity import LP_TOL_BF16, LP_TOL_F32, LP_TOL_XFMR_BF16, check_draft
+from test_gpu_parity import DEV, SMALL, _oracle_head, _with_table, _learned_weights
+
+pytestmark = pytest.mark.gpu
+
+
+def _sampled(name, seed=17, step=3, weights="learned"):
+    w = synth.stress(SMALL[name])
+    d = synth.make_inputs(w, device=DEV, target=False)
+    if name == "gru_b64":
+        d = _with_table(w, d)
+    a, b = _learned_weights(w.n) if weights == "learned" else ([w.weight] * w.n, [w.weight] * w.n)
+    W = {k[5:]: v for k, v in d.items() if k.startswith("head.")}
+    prior = dels.dels_prior_from_counts(d["counts"]).to(DEV)
+    dr = dels.Drafter(w.head, W, w.B, w.n, w.V)
+    tok, lp, gap, state = dr.sample(d["long"], prior, a, b, seed, step)
+    torch.cuda.synchronize()
+    assert dr.status() == 0
+    W = {k: v for k, v in W.items() if k != "input_table"}
+    return w, d, W, a, b, tok.cpu().numpy(), lp.cpu().numpy(), gap.cpu().numpy(), state
+
+
+@pytest.mark.parametrize("name", ["gru", "gru_b64", "mlp2", "xfmr", "markov", "gru_f32", "tiny"])
+def test_sampled_draft_matches_oracle(name):
+    seed, step = 17, 3
+    w, d, W, a, b, tok, lp, gap, state = _sampled(name, seed, step)
+    tol = LP_TOL_F32 if w.head.wdtype == "f32" else (LP_TOL_XFMR_BF16 if name == "xfmr" else LP_TOL_BF16)
+    info = check_draft(tok, lp, gap, _oracle_head(w, W), d["long"].cpu(), oracle.log_prior(d["counts"]),
+                       np.array(a), np.array(b), tol, sample=(seed, step))
+    # the LSE of every fused row, kept for the verification
+    lse = state[: w.B * w.n * 4].view(torch.float32).view(w.B, w.n).cpu().numpy()
+    np.testing.assert_allclose(lse, info["ref"].lse, rtol=0, atol=tol * 4)
+    print(name, {k: v for k, v in info.items() if k != "ref"})
+
+
+def test_sampled_draft_depends_on_seed_and_step_only():
+    w, d, W, a, b, tok1, lp1, _, _ = _sampled("gru", 5, 9)
+    _, _, _, _, _, tok2, lp2, _, _ = _sampled("gru", 5, 9)
+    np.testing.assert_array_equal(tok1, tok2)
+    np.testing.assert_array_equal(lp1, lp2)
+    _, _, _, _, _, tok3, _, _, _ = _sampled("gru", 5, 10)
+    _, _, _, _, _, tok4, _, _, _ = _sampled("gru", 6, 9)
+    assert not np.array_equal(tok1, tok3) and not np.array_equal(tok1, tok4)
+
+
+def test_sampled_draft_first_token_frequencies_follow_the_softmax():
+    """x_0 over many steps: empirical frequencies against softmax(l_L^(0)) of a
+    small, flat row (every token has mass)."""
+    from scipy.stats import chisquare
+    V, B = 16, 64
+    w = synth.Workload("flat", B=B, n=1, V=V, logit_dtype="f32",
+                       head=synth.HeadSpec("markov", "f32", 0, 0, 16), weight=0.0, seed=3)
+    d = synth.make_inputs(w, device=DEV, target=False)
+    row = torch.linspace(-1.0, 1.0, V, device=DEV)
+    long = row.expand(B, 1, V).contiguous()
+    W = {k[5:]: v for k, v in d.items() if k.startswith("head.")}
+    dr = dels.Drafter(w.head, W, B, 1, V)
+    prior = torch.zeros(V, device=DEV)
+    counts = np.zeros(V)
+    for step in range(40):
+        tok, _, _, _ = dr.sample(long, prior, [0.0], [0.0], 99, step)
+        counts += np.bincount(tok.cpu().numpy().ravel(), minlength=V)
+    p = torch.softmax(row.double(), 0).cpu().numpy()
+    assert chisquare(counts, counts.sum() * p).pvalue > 1e-3
