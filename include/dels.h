@@ -285,6 +285,35 @@ int dels_draft_block_sampled(const dels_local_head* head, const void* long_logit
                              float* out_key_gap, void* draft_state, size_t state_bytes, void* workspace,
                              size_t workspace_bytes, dels_stream_t stream);
 
+/*
+ * Verification of a temperature-1 block by lossless speculative sampling
+ * (accept with probability min(1, p/q), resample the residual), so that the
+ * emitted tokens follow the target model's distribution:
+ * for j = 0..n-1, x_j is accepted when u_j < p_j(x_j) / q_j(x_j), with p_j =
+ * softmax(target row j), q_j the distribution x_j was drawn from
+ * (exp(draft_logprob)), u_j the acceptance uniform of (b, j) (stream 1,
+ * v = 0). At the first rejection a the bonus token is drawn from
+ * max(0, p_a - q_a) (normalised) and after n acceptances from p_n, both by
+ * the Gumbel-max rule with the residual stream (2) at position a (or n).
+ * q_a is rebuilt from draft_state: l = l_L[b, a] + alpha[a] W_vocab r_a -
+ * beta[a] l_P (l_L[b, 0] at a = 0) and its LSE.
+ *   head, long_logits, log_prior, alpha, beta, seed, step, B, n, V: those of
+ *        the dels_draft_block_sampled call that produced the block;
+ *   draft_tokens [device] [B, n] int32, draft_logprob [device] [B, n] float32,
+ *   draft_state [device]: that call's outputs;
+ *   target_logits [device] [B, n+1, V] of target_dtype;
+ *   out_accept_len [device] [B] int32 (0..n), out_bonus [device] [B] int32,
+ *   out_bonus_gap [device] [B] float32 key gap of the bonus draw, or NULL.
+ * Limits: 1 <= n <= 32; B <= 128 for bf16 heads.
+ */
+size_t dels_verify_sampled_workspace_bytes(const dels_local_head* head, int B, int n, int V, dels_dtype target_dtype);
+int dels_verify_block_sampled(const dels_local_head* head, const int32_t* draft_tokens, const float* draft_logprob,
+                              const void* draft_state, const void* long_logits, dels_dtype logit_dtype,
+                              const float* log_prior, const float* alpha, const float* beta,
+                              const void* target_logits, dels_dtype target_dtype, int B, int n, int V, uint64_t seed,
+                              uint64_t step, int32_t* out_accept_len, int32_t* out_bonus, float* out_bonus_gap,
+                              void* workspace, size_t workspace_bytes, dels_stream_t stream);
+
 /* ---- greedy verification (Algorithm 1, last two steps) ------------------ */
 
 size_t dels_verify_workspace_bytes(int B, int n, int V, dels_dtype dtype);

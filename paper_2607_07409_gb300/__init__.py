@@ -23,6 +23,7 @@ __all__ = [
     "DelsError", "LocalHead", "lib", "library_path", "exported_symbols",
     "dels_draft_workspace_bytes", "dels_draft_block", "dels_draft_block_weighted",
     "dels_draft_state_bytes", "dels_draft_block_sampled",
+    "dels_verify_sampled_workspace_bytes", "dels_verify_block_sampled",
     "dels_combine_workspace_bytes", "dels_combine_argmax", "dels_combine_argmax_noalloc",
     "dels_verify_workspace_bytes", "dels_verify_block",
     "dels_read_status", "dels_prior_from_counts", "dels_status_string", "dels_version",
@@ -72,6 +73,9 @@ _SIGS = {
     "dels_draft_state_bytes": (_sz, [ctypes.POINTER(LocalHead), _i, _i]),
     "dels_draft_block_sampled": (_i, [ctypes.POINTER(LocalHead), _vp, _i, _vp, _vp, _vp, _i, _i, _i, ctypes.c_uint64,
                                       ctypes.c_uint64, _vp, _vp, _vp, _vp, _sz, _vp, _sz, _vp]),
+    "dels_verify_sampled_workspace_bytes": (_sz, [ctypes.POINTER(LocalHead), _i, _i, _i, _i]),
+    "dels_verify_block_sampled": (_i, [ctypes.POINTER(LocalHead), _vp, _vp, _vp, _vp, _i, _vp, _vp, _vp, _vp, _i, _i,
+                                       _i, _i, ctypes.c_uint64, ctypes.c_uint64, _vp, _vp, _vp, _vp, _sz, _vp]),
     "dels_combine_workspace_bytes": (_sz, [_i, _i, _i]),
     "dels_combine_argmax": (_i, [_vp, _vp, _i, _vp, _f, _f, _i, _i, _vp, _vp, _vp, _vp, _sz, _vp]),
     "dels_combine_argmax_noalloc": (_i, [_vp, _vp, _i, _vp, _f, _f, _i, _i, _vp, _vp, _vp, _vp]),
@@ -253,6 +257,24 @@ def dels_draft_block_sampled(head: LocalHead, long_logits, logit_dtype: int, log
                                           B, n, V, int(seed), int(step), _ptr(out_tokens), _ptr(out_logprob),
                                           _ptr(out_key_gap), _ptr(draft_state), state_bytes, _ptr(workspace),
                                           workspace_bytes, _stream(stream))
+
+
+def dels_verify_sampled_workspace_bytes(head: LocalHead, B: int, n: int, V: int, target_dtype: int) -> int:
+    return lib().dels_verify_sampled_workspace_bytes(ctypes.byref(head), B, n, V, target_dtype)
+
+
+def dels_verify_block_sampled(head: LocalHead, draft_tokens, draft_logprob, draft_state, long_logits,
+                              logit_dtype: int, log_prior, alpha, beta, target_logits, target_dtype: int, B: int,
+                              n: int, V: int, seed: int, step: int, out_accept_len, out_bonus, out_bonus_gap,
+                              workspace, workspace_bytes: int, stream=None) -> int:
+    """Speculative-sampling verification of a temperature-1 block; ``alpha``/``beta`` host sequences of n."""
+    a, ap = _host_floats(alpha, n)
+    b, bp = _host_floats(beta, n)
+    return lib().dels_verify_block_sampled(ctypes.byref(head), _ptr(draft_tokens), _ptr(draft_logprob),
+                                           _ptr(draft_state), _ptr(long_logits), logit_dtype, _ptr(log_prior), ap, bp,
+                                           _ptr(target_logits), target_dtype, B, n, V, int(seed), int(step),
+                                           _ptr(out_accept_len), _ptr(out_bonus), _ptr(out_bonus_gap),
+                                           _ptr(workspace), workspace_bytes, _stream(stream))
 
 
 def dels_combine_workspace_bytes(rows: int, V: int, dtype: int) -> int:

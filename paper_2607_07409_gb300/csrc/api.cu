@@ -1602,6 +1602,152 @@ int dels_draft_block_sampled(const dels_local_head* head, const void* long_logit
                           out_logprob, out_key_gap, workspace, workspace_bytes, stream, &sm);
 }
 
+namespace {
+
+struct VerifySampledLayout {
+  RowsPlan t;                 // target-row records
+  int r_nchunks, r_chunk_cols;
+  size_t t_rec, acc, lse_t, rg, ls, r_rec, total;
+};
+
+VerifySampledLayout verify_sampled_layout(const dels_local_head* head, int B, int n, int V, dels_dtype tdt, int sms) {
+  VerifySampledLayout L{};
+  const int es_t = tdt == DELS_F32 ? 4 : 2;
+  const bool vec = (V % (16 / es_t)) == 0;
+  const int rows = B * (n + 1);
+  L.t = plan_rows(std::max(rows, 1), V, es_t, sms, vec, 1 << 20);
+  L.r_nchunks = std::max(1, std::min((V + 2047) / 2048, (4 * sms + std::max(B, 1) - 1) / std::max(B, 1)));
+  L.r_chunk_cols = (int)round_up((size_t)((V + L.r_nchunks - 1) / L.r_nchunks), 8);
+  L.r_nchunks = (V + L.r_chunk_cols - 1) / L.r_chunk_cols;
+  const size_t es_w = head->wdtype == DELS_BF16 ? 2 : 4;
+  size_t off = kHeaderBytes;
+  L.t_rec = off;
+  off = round_up(off + (size_t)rows * L.t.nchunks * 16, 256);
+  L.acc = off;
+  off = round_up(off + (size_t)B * 4, 256);
+  L.lse_t = off;
+  off = round_up(off + (size_t)B * 4, 256);
+  L.rg = off;
+  off = round_up(off + (size_t)B * head->d_rank * es_w, 256);
+  L.ls = off;
+  off = round_up(off + (size_t)B * V * 4, 256);
+  L.r_rec = off;
+  off = round_up(off + (size_t)B * L.r_nchunks * 32, 256);
+  L.total = off;
+  return L;
+}
+
+}  // namespace
+
+size_t dels_verify_sampled_workspace_bytes(const dels_local_head* head, int B, int n, int V, dels_dtype target_dtype) {
+  if (!head || B < 0 || n < 1 || n > kMaxSampledBlock || V < 1) return 0;
+  if (target_dtype != DELS_F32 && target_dtype != DELS_BF16) return 0;
+  const int sms = device_sm_count();
+  if (sms <= 0) return 0;
+  return verify_sampled_layout(head, B, n, V, target_dtype, sms).total;
+}
+
+int dels_verify_block_sampled(const dels_local_head* head, const int32_t* draft_tokens, const float* draft_logprob,
+                              const void* draft_state, const void* long_logits, dels_dtype logit_dtype,
+                              const float* log_prior, const float* alpha, const float* beta,
+                              const void* target_logits, dels_dtype target_dtype, int B, int n, int V, uint64_t seed,
+                              uint64_t step, int32_t* out_accept_len, int32_t* out_bonus, float* out_bonus_gap,
+                              void* workspace, size_t workspace_bytes, dels_stream_t stream) {
+  if (!head || !alpha || !beta) return DELS_ERR_NULL_POINTER;
+  if ((logit_dtype != DELS_F32 && logit_dtype != DELS_BF16) || (target_dtype != DELS_F32 && target_dtype != DELS_BF16))
+    return DELS_ERR_BAD_DTYPE;
+  if (B < 0 || n < 1 || n > kMaxSampledBlock || V < 1) return DELS_ERR_BAD_SHAPE;
+  if ((long long)B * (n + 1) > INT32_MAX) return DELS_ERR_BAD_SHAPE;
+  const bool bf = head->wdtype == DELS_BF16;
+  if (bf && B > kMaxBatchTile) return DELS_ERR_BAD_SHAPE;
+  for (int j = 0; j < n; ++j)
+    if (!std::isfinite(alpha[j]) || !std::isfinite(beta[j])) return DELS_ERR_BAD_SHAPE;
+  if (!workspace) return DELS_ERR_WORKSPACE;
+  if (B == 0) return DELS_OK;
+  if (!draft_tokens || !draft_logprob || !draft_state || !long_logits || !target_logits || !out_accept_len ||
+      !out_bonus || !head->w_vocab)
+    return DELS_ERR_NULL_POINTER;
+  const size_t es_w = bf ? 2 : 4;
+  if (((size_t)head->d_rank * es_w) % 16 != 0) return DELS_ERR_UNSUPPORTED;
+  if (!aligned16(workspace) || !aligned16(draft_state) || !aligned16(target_logits) || !aligned16(long_logits))
+    return DELS_ERR_ALIGNMENT;
+  const int sms = device_sm_count();
+  if (sms <= 0) return DELS_ERR_CUDA;
+  const VerifySampledLayout L = verify_sampled_layout(head, B, n, V, target_dtype, sms);
+  if (workspace_bytes < L.total) return DELS_ERR_WORKSPACE;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  int* status = at<int>(workspace, 0);
+  // 1. records of the target rows (their LSEs)
+  RowsArgs t{};
+  t.longp = target_logits;
+  t.rows = B * (n + 1);
+  t.V = V;
+  t.ld_long = V;
+  t.chunk_cols = L.t.chunk_cols;
+  t.nchunks = L.t.nchunks;
+  t.rows_per_cta = 1;
+  t.partials = at<void>(workspace, L.t_rec);
+  t.partial_ld = L.t.nchunks;
+  t.status = status;
+  const int es_t = target_dtype == DELS_F32 ? 4 : 2;
+  const bool vec = (V % (16 / es_t)) == 0;
+  { PROF(DELS_KCLASS_VERIFY); DELS_CUDA(launch_combine_rows(t, target_dtype, vec, false, s)); }
+  // 2. the acceptance tests and the rejected position's input
+  VerifySampledArgs a{};
+  a.B = B;
+  a.n = n;
+  a.V = V;
+  a.draft = draft_tokens;
+  a.draft_lp = draft_logprob;
+  a.state_lse = static_cast<const float*>(draft_state);
+  a.state_r = static_cast<const uint8_t*>(draft_state) + round_up((size_t)B * n * 4, 256);
+  a.R = head->d_rank;
+  a.r_bytes = (int)es_w;
+  a.target = target_logits;
+  a.target_f32 = target_dtype == DELS_F32;
+  a.longp = long_logits;
+  a.long_f32 = logit_dtype == DELS_F32;
+  a.prior = log_prior;
+  for (int j = 0; j < n; ++j) {
+    a.alpha[j] = alpha[j];
+    a.beta[j] = beta[j];
+  }
+  a.seed = seed;
+  a.step = step;
+  a.t_records = t.partials;
+  a.t_nchunks = L.t.nchunks;
+  a.t_ld = L.t.nchunks;
+  a.acc = at<int>(workspace, L.acc);
+  a.lse_t = at<float>(workspace, L.lse_t);
+  a.rg = at<void>(workspace, L.rg);
+  a.ls = at<float>(workspace, L.ls);
+  a.r_records = at<void>(workspace, L.r_rec);
+  a.r_nchunks = L.r_nchunks;
+  a.r_chunk_cols = L.r_chunk_cols;
+  a.out_accept = out_accept_len;
+  a.out_bonus = out_bonus;
+  a.out_bonus_gap = out_bonus_gap;
+  a.status = status;
+  { PROF(DELS_KCLASS_VERIFY); DELS_CUDA(launch_verify_accept(a, s)); }
+  // 3. l_S of the rejected positions: W_vocab r (rows with no head input are zero)
+  if (bf) {
+    Gemm g;
+    if (!plan_store(g, B, V, a.rg, head->w_vocab, head->d_rank, nullptr, nullptr, 0, 128, 1, 0, ACT_NONE,
+                    at<float>(workspace, L.ls), nullptr, 0, status, sms))
+      return DELS_ERR_CUDA;
+    { PROF(DELS_KCLASS_VERIFY); DELS_CUDA(run(g, s)); }
+  } else {
+    { PROF(DELS_KCLASS_VERIFY);
+      DELS_CUDA(launch_gemv_f32(static_cast<const float*>(a.rg), head->d_rank,
+                                static_cast<const float*>(head->w_vocab), B, V, head->d_rank, ACT_NONE,
+                                at<float>(workspace, L.ls), V, s)); }
+  }
+  // 4. the bonus draw: the residual at the rejection, or p_n after n acceptances
+  { PROF(DELS_KCLASS_VERIFY); DELS_CUDA(launch_residual_rows(a, s)); }
+  { PROF(DELS_KCLASS_VERIFY); DELS_CUDA(launch_residual_merge(a, s)); }
+  return DELS_OK;
+}
+
 int dels_draft_block_weighted(const dels_local_head* head, const void* long_logits, dels_dtype logit_dtype,
                               const float* log_prior, const float* alpha, const float* beta, int B, int n, int V,
                               int32_t* out_tokens, float* out_logprob, float* out_top2_gap, void* workspace,

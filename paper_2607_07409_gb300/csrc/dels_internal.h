@@ -116,6 +116,39 @@ struct SampleRowsArgs {
 };
 cudaError_t launch_sample_rows(const SampleRowsArgs& a, bool f32, cudaStream_t s);
 
+// Verification of a temperature-1 block by lossless speculative sampling.
+constexpr int kMaxSampledBlock = 32;
+struct VerifySampledArgs {
+  int B, n, V;
+  const int32_t* draft;          // [B, n]
+  const float* draft_lp;         // [B, n] log q_j(x_j)
+  const float* state_lse;        // [B, n] LSE of the fused rows
+  const void* state_r;           // [B][n][R] vocabulary-projection inputs (j >= 1)
+  int R, r_bytes;
+  const void* target;            // [B, n+1, V]
+  int target_f32;
+  const void* longp;             // [B, n, V]
+  int long_f32;
+  const float* prior;            // [V] or null
+  float alpha[kMaxSampledBlock], beta[kMaxSampledBlock];
+  unsigned long long seed, step;
+  const void* t_records;         // [B * (n+1)][t_ld] RowAcc of the target rows
+  int t_nchunks, t_ld;
+  int* acc;                      // [B] accepted length
+  float* lse_t;                  // [B] LSE of target row acc[b]
+  void* rg;                      // [B][R] the rejected position's input (zeros at j = 0 and n)
+  const float* ls;               // [B][V] W_vocab rg
+  void* r_records;               // [B][r_nchunks][2] RowAcc: residual keys, then target keys
+  int r_nchunks, r_chunk_cols;
+  int32_t* out_accept;
+  int32_t* out_bonus;
+  float* out_bonus_gap;          // or null
+  int* status;
+};
+cudaError_t launch_verify_accept(const VerifySampledArgs& a, cudaStream_t s);
+cudaError_t launch_residual_rows(const VerifySampledArgs& a, cudaStream_t s);
+cudaError_t launch_residual_merge(const VerifySampledArgs& a, cudaStream_t s);
+
 struct MergeArgs {
   const void* partials;          // [B][partial_ld] RowAcc
   int partial_ld, count;

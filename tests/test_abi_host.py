@@ -165,3 +165,48 @@ def test_prior_entry_points_reject_bad_arguments_before_enqueueing(dels):
     assert L.dels_prior_estimate(p, p, 10, V, 1.0, None, None, None, wsp, need, None) == -1
     assert L.dels_prior_estimate(p, p, 10, V, 1.0, p, p + 4, None, wsp, need, None) == -4
     assert L.dels_prior_estimate(p, p, 10, V, 1.0, p, None, None, wsp, 256 + 8 * V - 1, None) == -5
+
+
+def test_sampled_entry_points_reject_bad_arguments_before_enqueueing(dels):
+    L = dels.lib()
+    buf0 = ctypes.create_string_buffer(64)
+    head = dels.LocalHead()
+    head.kind, head.wdtype, head.d_model, head.d_hidden, head.d_rank = 0, 1, 64, 64, 64
+    head.w_vocab = (ctypes.addressof(buf0) + 15) // 16 * 16
+    buf = ctypes.create_string_buffer(1 << 16)
+    p = (ctypes.addressof(buf) + 15) // 16 * 16
+    w = (ctypes.c_float * 4)(0.5, 0.5, 0.5, 0.5)
+    bad = (ctypes.c_float * 4)(0.5, float("nan"), 0.5, 0.5)
+    hp = ctypes.byref(head)
+    assert dels.dels_draft_state_bytes(head, 2, 4) == 256 + 2 * 4 * 64 * 2
+    assert dels.dels_draft_state_bytes(head, 2, 0) == 0
+    # dels_draft_block_sampled(head, long, dt, prior, alpha, beta, B, n, V, seed, step, tok, lp, gap, state,
+    #                          state_bytes, ws, ws_bytes, stream)
+    args = [hp, p, 1, p, w, w, 2, 4, 1000, 1, 2, p, p, None, p, 1 << 12, p, 1 << 15, None]
+    def call(**kw):
+        a = list(args)
+        for k, v in kw.items():
+            a[int(k[1:])] = v
+        return L.dels_draft_block_sampled(*a)
+    assert call(_4=None) == -1                  # alpha missing
+    assert call(_5=bad) == -2                   # non-finite beta
+    assert call(_7=0) == -2 and call(_7=33) == -2
+    assert call(_12=None) == -1                 # the logprob output is required
+    assert call(_15=100) == -5                  # draft state too small
+    assert call(_14=p + 4) == -4                # draft state misaligned
+    # dels_verify_block_sampled(head, tok, lp, state, long, ldt, prior, alpha, beta, target, tdt, B, n, V,
+    #                           seed, step, acc, bonus, gap, ws, ws_bytes, stream)
+    vargs = [hp, p, p, p, p, 1, p, w, w, p, 1, 2, 4, 1000, 1, 2, p, p, None, p, 1 << 15, None]
+    def vcall(**kw):
+        a = list(vargs)
+        for k, v in kw.items():
+            a[int(k[1:])] = v
+        return L.dels_verify_block_sampled(*a)
+    assert vcall(_5=9) == -3 and vcall(_10=9) == -3
+    assert vcall(_12=0) == -2 and vcall(_12=40) == -2
+    assert vcall(_8=bad) == -2
+    assert vcall(_3=None) == -1                 # no draft state
+    assert vcall(_16=None) == -1
+    assert vcall(_19=None) == -5
+    assert vcall(_3=p + 8) == -4
+    assert vcall(_11=200) == -2                 # bf16 heads: B <= 128

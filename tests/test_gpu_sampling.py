@@ -77,3 +77,71 @@ def test_sampled_draft_first_token_frequencies_follow_the_softmax():
         counts += np.bincount(tok.cpu().numpy().ravel(), minlength=V)
     p = torch.softmax(row.double(), 0).cpu().numpy()
     assert chisquare(counts, counts.sum() * p).pvalue > 1e-3
+
+
+# ------------------------------------------------ speculative-sampling verification
+
+def _verify(w, d, W, a, b, tok, lp, state, target, seed, step):
+    head = dels.make_head(w.head, W)
+    tdt = dels.dtype_code(target)
+    nbytes = dels.dels_verify_sampled_workspace_bytes(head, w.B, w.n, w.V, tdt)
+    assert nbytes > 0
+    ws = torch.zeros(nbytes, dtype=torch.uint8, device=DEV)
+    acc = torch.full((w.B,), -5, dtype=torch.int32, device=DEV)
+    bonus = torch.full((w.B,), -5, dtype=torch.int32, device=DEV)
+    bgap = torch.empty(w.B, dtype=torch.float32, device=DEV)
+    prior = dels.dels_prior_from_counts(d["counts"]).to(DEV)
+    r = dels.dels_verify_block_sampled(head, torch.as_tensor(tok, device=DEV), torch.as_tensor(lp, device=DEV), state,
+                                       d["long"], dels.dtype_code(d["long"]), prior, a, b, target, tdt, w.B, w.n, w.V,
+                                       seed, step, acc, bonus, bgap, ws, nbytes)
+    assert r == 0, dels.dels_status_string(r)
+    torch.cuda.synchronize()
+    assert dels.dels_read_status(ws) == 0
+    return acc.cpu().numpy(), bonus.cpu().numpy(), bgap.cpu().numpy()
+
+
+def _check_verify(w, d, W, a, b, tok, acc, bonus, bgap, target, seed, step, lp_tol):
+    """Accepted lengths and bonus tokens against the oracle run on the device's
+    drafted tokens (the oracle rebuilds q from its own fused rows)."""
+    ref = oracle.draft_block(_oracle_head(w, W), d["long"].cpu(), oracle.log_prior(d["counts"]), np.array(a),
+                             np.array(b), forced=tok, sample=(seed, step), keep_fused=True)
+    r_acc, r_bonus, info = oracle.verify_sampled(tok, ref.fused, target.cpu(), seed, step)
+    # a test whose ratio p/q lies within the logprob tolerance of its uniform may go either way
+    close = info["margin"] < 8 * lp_tol
+    same_acc = acc == r_acc
+    assert np.all(same_acc | close), (acc, r_acc, info["margin"])
+    ok = same_acc & ~close
+    # the bonus draw: identical unless the oracle's key gap is a near-tie
+    tie = info["bonus_gap"] < 0.05
+    bad = ok & (bonus != r_bonus) & ~tie
+    assert not bad.any(), (bonus[bad], r_bonus[bad], info["bonus_gap"][bad])
+    fin = ok & (bonus == r_bonus) & np.isfinite(info["bonus_gap"])
+    return dict(requests=int(len(acc)), close=int(close.sum()), ties=int((ok & tie).sum()),
+                accept=acc.tolist(), gap_err=float(np.abs(bgap[fin] - info["bonus_gap"][fin]).max(initial=0)))
+
+
+@pytest.mark.parametrize("name", ["gru", "gru_b64", "mlp2", "xfmr", "markov", "gru_f32", "tiny"])
+def test_sampled_verify_matches_oracle(name):
+    seed, step = 23, 7
+    w, d, W, a, b, tok, lp, gap, state = _sampled(name, seed, step)
+    target = synth.make_target_logits(w, d["long"], device=DEV)
+    acc, bonus, bgap = _verify(w, d, W, a, b, tok, lp, state, target, seed, step)
+    tol = LP_TOL_F32 if w.head.wdtype == "f32" else (LP_TOL_XFMR_BF16 if name == "xfmr" else LP_TOL_BF16)
+    info = _check_verify(w, d, W, a, b, tok, acc, bonus, bgap, target, seed, step, tol)
+    print(name, info)
+    assert np.all((acc >= 0) & (acc <= w.n)) and np.all((bonus >= 0) & (bonus < w.V))
+
+
+@pytest.mark.parametrize("name", ["gru", "markov", "tiny"])
+def test_sampled_verify_rejection_at_position_zero(name):
+    """The target rules out every x_0 (p_0(x_0) = 0): every request rejects at
+    0 and its bonus comes from the residual of softmax(l_L^(0)), never x_0."""
+    seed, step = 31, 2
+    w, d, W, a, b, tok, lp, gap, state = _sampled(name, seed, step)
+    target = synth.make_target_logits(w, d["long"], device=DEV).clone()
+    for bb in range(w.B):
+        target[bb, 0, int(tok[bb, 0])] = float("-inf")
+    acc, bonus, bgap = _verify(w, d, W, a, b, tok, lp, state, target, seed, step)
+    assert np.all(acc == 0) and np.all(bonus != tok[:, 0])
+    tol = LP_TOL_F32 if w.head.wdtype == "f32" else LP_TOL_BF16
+    print(name, _check_verify(w, d, W, a, b, tok, acc, bonus, bgap, target, seed, step, tol))
