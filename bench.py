@@ -52,6 +52,9 @@ def parse_args():
     p.add_argument("--sweep", action="store_true",
                    help="instead of the drafting step: HBM GB/s of dels_combine_argmax and dels_verify_block over "
                         "the combine/verify sweep grid (one JSON line per point)")
+    p.add_argument("--temperature", type=int, choices=[0, 1], default=0,
+                   help="1: the temperature-1 step instead (Gumbel-max drafting + speculative-sampling "
+                        "verification), printed as its own JSON line")
     p.add_argument("--prior", action="store_true",
                    help="instead of the drafting step: device unigram-prior estimation (masked token histogram, "
                         "smoothing, log) over a 2^28-position synthetic chat corpus")
@@ -538,6 +541,111 @@ def run_sweep(args):
     return 0
 
 
+def run_sampled(args):
+    """Drafted tokens per second at temperature 1 on the same workload as the
+    default step: dels_draft_block_sampled (every position drawn by the
+    Gumbel-max rule inside the vocabulary projection's pass) followed by
+    dels_verify_block_sampled (acceptance tests, the rejected position's draft
+    distribution rebuilt, the residual or p_n bonus draw). A fresh `step`
+    every iteration, so every block draws new variates."""
+    import torch
+    import synth
+    import paper_2607_07409_gb300 as dels
+    from paper_2607_07409_gb300 import replicas
+    world, rank, local = dist_setup(args.gpus)
+    dev = torch.device(f"cuda:{local}")
+    torch.cuda.set_device(dev)
+    peak, peak_kind = measured_peaks()
+    w0 = synth.WORKLOADS[WORKLOAD]
+    w = synth.with_sizes(w0, seed=replicas.replica_seed(w0.seed, rank))
+    d = synth.make_inputs(w, device=dev)
+    W = {k[5:]: v for k, v in d.items() if k.startswith("head.")}
+    prior = dels.dels_prior_from_counts(d["counts"]).to(dev)
+    if not args.no_input_table:
+        W["input_table"] = dels.gru_input_table(w.head, W, w.V)
+    drafter = dels.Drafter(w.head, W, w.B, w.n, w.V)
+    a = [w.alpha] * w.n
+    b = [w.beta] * w.n
+    head = drafter.head
+    vbytes = dels.dels_verify_sampled_workspace_bytes(head, w.B, w.n, w.V, dels.DELS_BF16)
+    vws = torch.zeros(vbytes, dtype=torch.uint8, device=dev)
+    acc = torch.empty(w.B, dtype=torch.int32, device=dev)
+    bonus = torch.empty(w.B, dtype=torch.int32, device=dev)
+    stream = torch.cuda.current_stream()
+    seed = 1234 + rank
+
+    def draft(step):
+        return drafter.sample(d["long"], prior, a, b, seed, step, stream)
+
+    def verify(step, tok, lp, state):
+        r = dels.dels_verify_block_sampled(head, tok, lp, state, d["long"], dels.DELS_BF16, prior, a, b, d["target"],
+                                           dels.DELS_BF16, w.B, w.n, w.V, seed, step, acc, bonus, None, vws, vbytes,
+                                           stream)
+        if r != 0:
+            raise dels.DelsError(r, "dels_verify_block_sampled")
+
+    for i in range(max(3, args.warmup)):
+        tok, lp, _, state = draft(i)
+        verify(i, tok, lp, state)
+    torch.cuda.synchronize()
+    if drafter.status() != 0 or dels.dels_read_status(vws) != 0:
+        raise RuntimeError("device status set during warm-up")
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+    replicas.barrier()
+    torch.cuda.synchronize()
+    t_draft = t_ver = 0.0
+    lens = []
+    with ClockSampler(local) as clk:
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for i in range(args.steps):
+            tok, lp, _, state = draft(1000 + i)
+            verify(1000 + i, tok, lp, state)
+        e1.record(stream)
+        torch.cuda.synchronize()
+    ms = replicas.max_over_ranks(e0.elapsed_time(e1) / args.steps)
+    # the two halves, timed apart on a few more steps
+    for i in range(min(args.steps, 20)):
+        ev[0].record(stream)
+        tok, lp, _, state = draft(5000 + i)
+        ev[1].record(stream)
+        verify(5000 + i, tok, lp, state)
+        ev[2].record(stream)
+        torch.cuda.synchronize()
+        t_draft += ev[0].elapsed_time(ev[1])
+        t_ver += ev[1].elapsed_time(ev[2])
+        lens.append(acc.cpu().numpy().copy())
+    k = min(args.steps, 20)
+    # the sampled vocabulary kernel, event-timed by the library's profiler
+    dels.dels_profile_reset()
+    dels.dels_profile_enable(True)
+    for i in range(3):
+        draft(9000 + i)
+    torch.cuda.synchronize()
+    n_v, ms_v = dels.dels_profile_read(dels.KCLASS["vocab_combine"])
+    dels.dels_profile_enable(False)
+    us_v = 1e3 * ms_v / max(n_v, 1)
+    vbytes_alg = algorithmic_vocab_bytes(w)
+    import numpy as np
+    tau = float(np.mean(np.concatenate(lens)) + 1.0)
+    if rank == 0:
+        print(json.dumps({
+            "metric": "drafted tokens/sec at temperature 1 (Gumbel-max draft + speculative-sampling verify)",
+            "value": world * w.B * w.n / (ms * 1e-3), "unit": "drafted tokens/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16 weights/logits, f32 accumulate", "data": "synthetic",
+            "config": {"workload": f"{WORKLOAD} B={w.B} n={w.n} V={w.V} GRU 4096/1024/256, temperature 1",
+                       "l2": "inputs larger than L2"},
+            "draft_ms": t_draft / k, "verify_ms": t_ver / k, "tau": tau,
+            "roofline": {"bound": "hbm", "kernel": "k_tc_gemm<sample> (vocab projection + Gumbel-max)",
+                         "achieved": vbytes_alg / (us_v * 1e-6) / 1e9, "peak": peak, "unit": "GB/s",
+                         "frac": vbytes_alg / (us_v * 1e-6) / 1e9 / peak, "peak_source": peak_kind,
+                         "us_per_launch": us_v},
+            "clocks": clk.summary()}), flush=True)
+    replicas.barrier()
+    return 0
+
+
 def run_prior(args):
     """Corpus positions per second of dels_prior_estimate (zero the counts,
     count the loss-masked ids, write l_P) over the 2^28-position synthetic
@@ -638,6 +746,8 @@ def main():
         return run_sweep(args)
     if args.prior:
         return run_prior(args)
+    if args.temperature == 1:
+        return run_sampled(args)
     return run_ours(args)
 
 
