@@ -55,6 +55,9 @@ def parse_args():
     p.add_argument("--temperature", type=int, choices=[0, 1], default=0,
                    help="1: the temperature-1 step instead (Gumbel-max drafting + speculative-sampling "
                         "verification), printed as its own JSON line")
+    p.add_argument("--variant", choices=["gru", "wide"], default="gru",
+                   help="wide: the same step with a 4096-wide vocabulary projection (a Markov head over the "
+                        "4096-wide token state, W [V, 4096]) instead of the GRU head, printed as its own line")
     p.add_argument("--prior", action="store_true",
                    help="instead of the drafting step: device unigram-prior estimation (masked token histogram, "
                         "smoothing, log) over a 2^28-position synthetic chat corpus")
@@ -646,6 +649,83 @@ def run_sampled(args):
     return 0
 
 
+def run_wide(args):
+    """The wide-projection row: every position projects a 4096-wide state
+    (r = E[x_{j-1}], E [V, 4096]) onto the vocabulary through W [V, 4096]
+    (1.24 GB bf16 streamed per position, no recurrence), fused with the
+    combine; then the greedy verification. Same B, n, V and logits as the
+    default step."""
+    import torch
+    import synth
+    import paper_2607_07409_gb300 as dels
+    from paper_2607_07409_gb300 import replicas
+    world, rank, local = dist_setup(args.gpus)
+    dev = torch.device(f"cuda:{local}")
+    torch.cuda.set_device(dev)
+    peak, peak_kind = measured_peaks()
+    w0 = synth.WORKLOADS[WORKLOAD]
+    w = synth.Workload("qwen3_8b_wide", B=w0.B, n=w0.n, V=w0.V, logit_dtype=w0.logit_dtype,
+                       head=synth.HeadSpec("markov", "bf16", 0, 0, 4096), weight=w0.weight,
+                       seed=replicas.replica_seed(w0.seed, rank), zipf=w0.zipf, long_std=w0.long_std,
+                       target_noise=w0.target_noise)
+    d = synth.make_inputs(w, device=dev)
+    W = {k[5:]: v for k, v in d.items() if k.startswith("head.")}
+    prior = dels.dels_prior_from_counts(d["counts"]).to(dev)
+    drafter = dels.Drafter(w.head, W, w.B, w.n, w.V)
+    vbytes = dels.dels_verify_workspace_bytes(w.B, w.n, w.V, dels.DELS_BF16)
+    vws = torch.zeros(vbytes, dtype=torch.uint8, device=dev)
+    acc = torch.empty(w.B, dtype=torch.int32, device=dev)
+    bonus = torch.empty(w.B, dtype=torch.int32, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def step():
+        tok, lp, gap = drafter(d["long"], prior, w.alpha, w.beta, stream)
+        r = dels.dels_verify_block(tok, d["target"], dels.DELS_BF16, w.B, w.n, w.V, acc, bonus, None, vws, vbytes,
+                                   stream)
+        if r != 0:
+            raise dels.DelsError(r, "dels_verify_block")
+
+    for _ in range(max(3, args.warmup)):
+        step()
+    torch.cuda.synchronize()
+    if drafter.status() != 0:
+        raise RuntimeError("device status set during warm-up")
+    steps = max(1, min(args.steps, 30))
+    replicas.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(steps):
+            step()
+        e1.record(stream)
+        torch.cuda.synchronize()
+    ms = replicas.max_over_ranks(e0.elapsed_time(e1) / steps)
+    dels.dels_profile_reset()
+    dels.dels_profile_enable(True)
+    step()
+    torch.cuda.synchronize()
+    n_v, ms_v = dels.dels_profile_read(dels.KCLASS["vocab_combine"])
+    dels.dels_profile_enable(False)
+    us_v = 1e3 * ms_v / max(n_v, 1)
+    R = w.head.d_rank
+    vb = w.V * R * 2 + w.B * w.V * 2 + w.V * 4 + w.B * R * 2
+    if rank == 0:
+        print(json.dumps({
+            "metric": "drafted tokens/sec, wide vocabulary projection (W [V, 4096] per position) + verify",
+            "value": world * w.B * w.n / (ms * 1e-3), "unit": "drafted tokens/s", "n_gpus": world, "steps": steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": f"B={w.B} n={w.n} V={w.V}, 4096-wide state, W [V, 4096] bf16",
+                       "l2": "inputs larger than L2"},
+            "roofline": {"bound": "hbm", "kernel": "k_tc_gemm<1> (K = 4096)", "achieved": vb / (us_v * 1e-6) / 1e9,
+                         "peak": peak, "unit": "GB/s", "frac": vb / (us_v * 1e-6) / 1e9 / peak,
+                         "peak_source": peak_kind, "us_per_launch": us_v, "algorithmic_bytes": vb},
+            "clocks": clk.summary()}), flush=True)
+    replicas.barrier()
+    return 0
+
+
 def run_prior(args):
     """Corpus positions per second of dels_prior_estimate (zero the counts,
     count the loss-masked ids, write l_P) over the 2^28-position synthetic
@@ -748,6 +828,8 @@ def main():
         return run_prior(args)
     if args.temperature == 1:
         return run_sampled(args)
+    if args.variant == "wide":
+        return run_wide(args)
     return run_ours(args)
 
 

@@ -201,6 +201,9 @@ SMALL = {
                              head=synth.HeadSpec("markov", "bf16", 0, 0, 128), weight=0.5, seed=7),
     "markov_f32": synth.Workload("markov_f32", B=2, n=5, V=1000, logit_dtype="f32",
                                  head=synth.HeadSpec("markov", "f32", 0, 0, 64), weight=0.5, seed=8),
+    # the wide vocabulary projection: a 4096-wide state (no recurrence), K = 4096 streamed with W
+    "markov_wide": synth.Workload("markov_wide", B=40, n=4, V=1536, logit_dtype="bf16",
+                                  head=synth.HeadSpec("markov", "bf16", 0, 0, 4096), weight=0.5, seed=9),
     "gru_f32": synth.with_sizes(synth.WORKLOADS["qwen3_8b_batched"], B=3, n=5, V=1200, logit_dtype="f32",
                                 head_wdtype="f32", head_d_model=64, head_d_hidden=32, head_d_rank=16),
 }
