@@ -223,7 +223,7 @@ def sample_decode(l, g):
     return x, float(l[x] - z), gap, z
 
 
-def verify_sampled(draft, draft_logits, target, seed: int, step: int):
+def verify_sampled(draft, draft_logits, target, seed: int, step: int, request_ids=None):
     """Lossless speculative sampling (Leviathan et al. 2023; Chen et al. 2023)
     of a block drafted at temperature 1.
 
@@ -234,6 +234,9 @@ def verify_sampled(draft, draft_logits, target, seed: int, step: int):
     drawn from the residual max(0, p_j - q_j) (normalised) by the Gumbel-max
     rule with the residual stream at position j; when all n are accepted it
     is drawn from p_n the same way at position n.
+
+    ``request_ids``: the request index of each row for the random numbers
+    (default 0..B-1).
 
     Returns (accept [B], bonus [B], info) with info["margin"][b] the distance
     |u - p/q| of the deciding test (the smallest over the accepted positions
@@ -252,22 +255,23 @@ def verify_sampled(draft, draft_logits, target, seed: int, step: int):
     margin = np.full(B, np.inf)
     bonus_gap = np.zeros(B)
     for b in range(B):
+        rid = b if request_ids is None else int(request_ids[b])
         a = n
         for j in range(n):
             p = np.exp(T[b, j] - lse(T[b, j]))
             q = np.exp(Q[b, j] - lse(Q[b, j]))
             x = D[b, j]
-            u = float(uniforms(seed, step, b, j, STREAM_ACCEPT, np.array([0]))[0])
+            u = float(uniforms(seed, step, rid, j, STREAM_ACCEPT, np.array([0]))[0])
             ratio = p[x] / q[x]
             margin[b] = min(margin[b], abs(u - ratio))
             if not u < ratio:
                 a = j
                 w = np.maximum(p - q, 0.0)
                 with np.errstate(divide="ignore"):
-                    key = np.log(w) + gumbel(uniforms(seed, step, b, j, STREAM_RESIDUAL, vidx))
+                    key = np.log(w) + gumbel(uniforms(seed, step, rid, j, STREAM_RESIDUAL, vidx))
                 break
         if a == n:
-            key = T[b, n] + gumbel(uniforms(seed, step, b, n, STREAM_RESIDUAL, vidx))
+            key = T[b, n] + gumbel(uniforms(seed, step, rid, n, STREAM_RESIDUAL, vidx))
         accept[b] = a
         bonus[b] = int(np.argmax(key))
         rest = np.delete(key, bonus[b])

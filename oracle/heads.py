@@ -229,12 +229,15 @@ class DraftResult:
     fused: Optional[np.ndarray] = None      # [B, n, V] fused rows (temperature 1, keep_fused)
 
 
-def draft_block(head, long, prior, alpha, beta, forced=None, keep_short=(), sample=None, keep_fused=False):
+def draft_block(head, long, prior, alpha, beta, forced=None, keep_short=(), sample=None, keep_fused=False,
+                request_ids=None):
     """Algorithm 1 for one block of B independent rows, at temperature 0
     (``sample=None``: Decode = argmax) or temperature 1 (``sample=(seed,
     step)``: Decode draws x_j from softmax(l^(j)) by the Gumbel-max rule,
     x_j = argmax(l^(j) + g), g the drafting-stream Gumbel variates of (b, j);
     ``gap`` and the forced-mode values then refer to the keys l + g).
+    ``request_ids``: the request index of each row for the random numbers
+    (default 0..B-1), so that a subset of a batch draws its own variates.
 
     long [B, n, V] long-context logits; prior [V] log unigram prior.
     Position 0: x_0 = argmax l_L^(0) (no local head, no prior term).
@@ -275,7 +278,8 @@ def draft_block(head, long, prior, alpha, beta, forced=None, keep_short=(), samp
             x, lp, g = greedy_decode(f)
             key = f
         else:
-            gv = gumbel(uniforms(sample[0], sample[1], b, j, STREAM_DRAFT, vidx))
+            rid = b if request_ids is None else int(request_ids[b])
+            gv = gumbel(uniforms(sample[0], sample[1], rid, j, STREAM_DRAFT, vidx))
             x, lp, g, z = sample_decode(f, gv)
             key = f + gv
             lse_out[b, j] = z

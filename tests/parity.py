@@ -58,14 +58,15 @@ def check_rows(tok, lp, gap, ref_tok, ref_lp, ref_gap, lp_tol=LP_TOL_COMBINE, ex
     return dict(ties=int(ties.sum()), flips=int((~same).sum()), lp_err=float(err))
 
 
-def check_draft(tok, lp, gap, head, long, prior, alpha, beta, lp_tol, sample=None):
+def check_draft(tok, lp, gap, head, long, prior, alpha, beta, lp_tol, sample=None, request_ids=None):
     """Block drafting parity via the oracle's forced-prefix mode; also checks
     that the free-running oracle reproduces the device block exactly when no
     position had a near-tie. ``sample=(seed, step)``: temperature 1 (the
     token rule and the gap then refer to the Gumbel-max keys l + g)."""
     tok = np.asarray(tok)
     lp = np.asarray(lp)
-    ref = oracle.draft_block(head, long, prior, alpha, beta, forced=tok, sample=sample)
+    ref = oracle.draft_block(head, long, prior, alpha, beta, forced=tok, sample=sample, keep_fused=sample is not None,
+                             request_ids=request_ids)
     same = tok == ref.argmax
     ties = ref.gap < TIE_EPS
     bad = ~same & ~(ties & (ref.fused_at >= ref.fused_max - TIE_EPS))

@@ -80,3 +80,42 @@ def test_qwen3_0p6b_full_size():
 def test_qwen3_4b_full_size():
     w = synth.WORKLOADS["qwen3_4b"]
     print(_draft_and_verify(w, [0, 7]))
+
+
+def test_qwen3_8b_batched_full_size_temperature_one():
+    """Temperature 1 at full size (input-table path, the benchmark's launch
+    configuration): sampled rows drafted by the Gumbel-max rule and verified
+    by speculative sampling, against the oracle with the rows' own variates."""
+    w = synth.stress(synth.WORKLOADS["qwen3_8b_batched"])
+    seed, step = 77, 5
+    rows = [2, 45]
+    d = synth.make_inputs(w, device=DEV, target=True)
+    W = {k[5:]: v for k, v in d.items() if k.startswith("head.")}
+    W["input_table"] = dels.gru_input_table(w.head, W, w.V)
+    prior = dels.dels_prior_from_counts(d["counts"]).to(DEV)
+    a = [w.alpha] * w.n
+    b = [w.beta] * w.n
+    dr = dels.Drafter(w.head, W, w.B, w.n, w.V)
+    tok, lp, gap, state = dr.sample(d["long"], prior, a, b, seed, step)
+    head = dr.head
+    dt = dels.dtype_code(d["target"])
+    vb = dels.dels_verify_sampled_workspace_bytes(head, w.B, w.n, w.V, dt)
+    vws = torch.zeros(vb, dtype=torch.uint8, device=DEV)
+    acc = torch.empty(w.B, dtype=torch.int32, device=DEV)
+    bonus = torch.empty(w.B, dtype=torch.int32, device=DEV)
+    assert dels.dels_verify_block_sampled(head, tok, lp, state, d["long"], dels.dtype_code(d["long"]), prior, a, b,
+                                          d["target"], dt, w.B, w.n, w.V, seed, step, acc, bonus, None, vws, vb) == 0
+    torch.cuda.synchronize()
+    assert dr.status() == 0 and dels.dels_read_status(vws) == 0
+    tok, lp, gap = (t.cpu().numpy() for t in (tok, lp, gap))
+    ohead = _oracle_head(w, W)
+    info = check_draft(tok[rows], lp[rows], gap[rows], ohead, d["long"][rows].cpu(), oracle.log_prior(d["counts"]),
+                       np.array(a), np.array(b), LP_TOL_BF16, sample=(seed, step), request_ids=rows)
+    r_acc, r_bonus, vinfo = oracle.verify_sampled(tok[rows], info["ref"].fused, d["target"][rows].cpu(), seed, step,
+                                                  request_ids=rows)
+    acc, bonus = acc.cpu().numpy()[rows], bonus.cpu().numpy()[rows]
+    close = vinfo["margin"] < 8 * LP_TOL_BF16
+    assert np.all((acc == r_acc) | close), (acc, r_acc, vinfo["margin"])
+    ok = (acc == r_acc) & ~close
+    assert np.all((bonus == r_bonus) | ~ok | (vinfo["bonus_gap"] < 0.05)), (bonus, r_bonus, vinfo["bonus_gap"])
+    print({k: v for k, v in info.items() if k != "ref"}, "accept", acc.tolist(), r_acc.tolist())
