@@ -346,6 +346,70 @@ def test_draft_block_of_one_position():
     np.testing.assert_array_equal(tok[:, 0], np.argmax(L[:, 0], axis=1))
 
 
+@pytest.mark.parametrize("table", [False, True])
+def test_draft_largest_batch_tile(table):
+    """B = 128: every row of the tensor cores' M = 128 tile is a live request."""
+    w = synth.with_sizes(synth.stress(synth.WORKLOADS["qwen3_8b_batched"]), B=128, n=4, V=2048,
+                         head_d_model=128, head_d_hidden=64, head_d_rank=64)
+    d = synth.make_inputs(w, device=DEV, target=False)
+    if table:
+        d = _with_table(w, d)
+    tok, lp, gap, W, prior = _draft(w, d)
+    W = {k: v for k, v in W.items() if k != "input_table"}
+    print(check_draft(tok, lp, gap, _oracle_head(w, W), d["long"].cpu(), prior, w.alpha, w.beta, LP_TOL_BF16))
+
+
+def test_draft_and_sampled_calls_with_an_empty_batch():
+    w = synth.with_sizes(synth.WORKLOADS["qwen3_8b_batched"], B=2, n=4, V=1024,
+                         head_d_model=64, head_d_hidden=32, head_d_rank=32)
+    d = synth.make_inputs(w, device=DEV, target=True)
+    W = {k[5:]: v for k, v in d.items() if k.startswith("head.")}
+    head = dels.make_head(w.head, W)
+    prior = dels.dels_prior_from_counts(d["counts"]).to(DEV)
+    ws = _ws(dels.dels_draft_workspace_bytes(head, 2, w.n, w.V))
+    nb = ws.numel()
+    tok = torch.full((1,), -9, dtype=torch.int32, device=DEV)
+    lp = torch.zeros(1, device=DEV)
+    assert dels.dels_draft_block(head, d["long"], dels.DELS_BF16, prior, 0.3, 0.3, 0, w.n, w.V, tok, lp, None,
+                                 ws, nb) == 0
+    a = [0.3] * w.n
+    st = _ws(max(16, dels.dels_draft_state_bytes(head, 1, w.n)))
+    assert dels.dels_draft_block_sampled(head, d["long"], dels.DELS_BF16, prior, a, a, 0, w.n, w.V, 1, 2, tok, lp,
+                                         None, st, st.numel(), ws, nb) == 0
+    vb = dels.dels_verify_sampled_workspace_bytes(head, 1, w.n, w.V, dels.DELS_BF16)
+    vws = _ws(vb)
+    acc = torch.full((1,), -9, dtype=torch.int32, device=DEV)
+    assert dels.dels_verify_block_sampled(head, tok, lp, st, d["long"], dels.DELS_BF16, prior, a, a, d["target"],
+                                          dels.DELS_BF16, 0, w.n, w.V, 1, 2, acc, acc, None, vws, vb) == 0
+    torch.cuda.synchronize()
+    assert int(tok[0]) == -9 and int(acc[0]) == -9      # nothing was written
+    assert _status(ws) == 0 and _status(vws) == 0
+
+
+@pytest.mark.parametrize("table", [False, True])
+def test_draft_nonfinite_long_logits_flag_the_row(table):
+    """A NaN in request 1's DFlash logits at position 2: the status word flags
+    it, that position's token is -1, and the other requests are untouched."""
+    w = synth.with_sizes(synth.stress(synth.WORKLOADS["qwen3_8b_batched"]), B=4, n=5, V=2048,
+                         head_d_model=128, head_d_hidden=64, head_d_rank=64)
+    d = synth.make_inputs(w, device=DEV, target=False)
+    if table:
+        d = _with_table(w, d)
+    d["long"][1, 2, 77] = float("nan")
+    W = {k[5:]: v for k, v in d.items() if k.startswith("head.")}
+    prior = dels.dels_prior_from_counts(d["counts"]).to(DEV)
+    dr = dels.Drafter(w.head, W, w.B, w.n, w.V)
+    tok, lp, gap = dr(d["long"], prior, w.alpha, w.beta)
+    torch.cuda.synchronize()
+    assert dr.status() & dels.DELS_STATUS_NONFINITE
+    tok, lp, gap = tok.cpu().numpy(), lp.cpu().numpy(), gap.cpu().numpy()
+    assert tok[1, 2] == -1 and np.isnan(lp[1, 2])
+    rows = [0, 2, 3]
+    W = {k: v for k, v in W.items() if k != "input_table"}
+    check_draft(tok[rows], lp[rows], gap[rows], _oracle_head(w, W), d["long"][rows].cpu(),
+                oracle.log_prior(d["counts"]), w.alpha, w.beta, LP_TOL_BF16)
+
+
 # ------------------------------------------------------------ bounded waits
 
 def test_expired_wait_reports_timeout_and_context_survives():
