@@ -207,3 +207,27 @@ def test_hot_cold_pieces_on_top_of_earlier_counts():
     c_ref, n_in, _ = oracle.count_masked_tokens(tok.numpy(), mask.numpy(), V)
     np.testing.assert_array_equal(counts.cpu().numpy(), c_ref)
     assert tally.cpu().tolist() == [n_in, 0]
+
+
+def test_hot_path_hand_off_of_a_single_id():
+    """One id at every loss-masked position of a hot-path range: every CTA's
+    16-bit bin for it passes 2^15 twice and hands it to the global count."""
+    V, N = 151936, HOT_N
+    tok = torch.full((N,), 4242, dtype=torch.int32)
+    mask = torch.full((N,), 3, dtype=torch.uint8)
+    mask[::3] = 0
+    out, c, tally = _estimate(tok.to(DEV), mask.to(DEV), V)
+    expect = int((mask != 0).sum())
+    assert expect // torch.cuda.get_device_properties(0).multi_processor_count > 2 * 2 ** 15
+    assert c[4242] == expect and c.sum() == expect and tally.tolist() == [expect, 0]
+
+
+def test_hot_path_vocabulary_a_multiple_of_15_with_bad_ids():
+    """V = 15 * 10129: an id clamped to V falls on the remap table's zero
+    sentinel word, past the last word that holds vocabulary ids."""
+    V = 151935
+    tok, mask = _corpus(V, HOT_N, 11, bad=57)
+    c_ref, n_in, n_out = oracle.count_masked_tokens(tok.numpy(), mask.numpy(), V)
+    out, c, tally = _estimate(tok.to(DEV), mask.to(DEV), V)
+    np.testing.assert_array_equal(c, c_ref)
+    assert tally.tolist() == [n_in, n_out] and n_out == 57
