@@ -408,18 +408,15 @@ __global__ void __launch_bounds__(kThreads, 1) k_prior_hot(PriorHotArgs a) {
     for (int k = 0; k < 4; ++k) tk[k] = __ldcs(tv + w0 + 32 * k);
 #pragma unroll
     for (int k = 0; k < 4; ++k) mk[k] = __ldcs(mv + w0 + 32 * k);
-    uint32_t valid_bits = 0, bad_bits = 0;
 #pragma unroll
     for (int q = 0; q < 16; ++q) {
       const int id = int4_at(tk[q >> 2], q & 3);
       const bool masked = mask_byte(mk[q >> 2], q & 3) != 0u;
       const bool in_range = (unsigned)id < (unsigned)a.V;
-      valid_bits |= (masked && in_range) ? (1u << q) : 0u;
-      bad_bits |= (masked && !in_range) ? (1u << q) : 0u;
+      t.in += (masked && in_range) ? 1u : 0u;
+      t.out += (masked && !in_range) ? 1u : 0u;
       if (masked && in_range) count_one(id);
     }
-    t.in += __popc(valid_bits);
-    t.out += __popc(bad_bits);
   }
   const long long rest = r.n - r.nvec;
   for (long long j = worker * 32 + lane; j < rest; j += nworkers * 32) {
