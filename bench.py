@@ -52,6 +52,8 @@ def parse_args():
     p.add_argument("--sweep", action="store_true",
                    help="instead of the drafting step: HBM GB/s of dels_combine_argmax and dels_verify_block over "
                         "the combine/verify sweep grid (one JSON line per point)")
+    p.add_argument("--point", default=None, metavar="V,DTYPE,B,N",
+                   help="with --sweep: only this point of the grid, e.g. 151936,bf16,64,16")
     p.add_argument("--temperature", type=int, choices=[0, 1], default=0,
                    help="1: the temperature-1 step instead (Gumbel-max drafting + speculative-sampling "
                         "verification), printed as its own JSON line")
@@ -514,8 +516,12 @@ def run_sweep(args):
                 ts.append(a.elapsed_time(b) * 1e-3)
         return statistics.median(ts)
 
-    for pt in synth.sweep_points():
-        key = (pt["V"], pt["dtype"], pt["B"], pt["n"])
+    only = None
+    if args.point:
+        v_, d_, b_, n_ = args.point.split(",")
+        only = (int(v_), d_, int(b_), int(n_))
+    points = [only] if only else [(pt["V"], pt["dtype"], pt["B"], pt["n"]) for pt in synth.sweep_points()]
+    for key in points:
         if key in seen:
             continue
         seen.add(key)

@@ -133,17 +133,19 @@ __global__ void __launch_bounds__(kRowsThreads) k_combine_rows(RowsArgs a) {
   for (int r = 0; r < R; ++r) st[r].init();
 
   if constexpr (VEC) {
-    // Raw 16-byte words stay in registers until used, so bf16 rows keep as
-    // many bytes in flight per thread as f32 rows (8 loads per row for
-    // bf16, 4 for f32, when one row per CTA).
+    // Raw 16-byte words stay in registers until used: U groups of 8 values
+    // per row in flight (one row per CTA). U = 4 for both types: deeper
+    // unrolling of bf16 rows (8 loads) costs registers, and with two CTAs
+    // per SM instead of four the issue-heavy bf16 update stalls (measured
+    // 172 us against 126 us for 1024 rows of 151936).
     constexpr int WPV = sizeof(T) == 2 ? 1 : 2;            // 16-byte words per 8 values
-    constexpr int U = (R == 1) ? (sizeof(T) == 2 ? 8 : 4) : 1;
+    constexpr int U = (R == 1) ? 4 : 1;
     const int step = kRowsThreads * 8;
     for (int cb = c0 + threadIdx.x * 8; cb < c1; cb += step * U) {
       uint4 lw[U][R][WPV];
       uint4 sw[U][R][WPV];
       // f32: the prior goes out with the logits; bf16: it is read where it
-      // is used (keeps the bf16 kernel at two CTAs per SM)
+      // is used (fewer registers: four CTAs per SM)
       constexpr bool kPriorEarly = sizeof(T) == 4;
       float4 pw[kPriorEarly ? U : 1][2];
 #pragma unroll
@@ -302,7 +304,7 @@ __global__ void __launch_bounds__(kRowsThreads) k_verify_rows(RowsArgs a) {
     // holding the thread's maximum wins), and at the end the first element of
     // that vector equal to the maximum: the same lowest-index argmax as an
     // element-by-element scan, at a fraction of the instructions.
-    constexpr int U = 8;
+    constexpr int U = 4;   // 16-byte loads in flight per thread (8: 2.7% slower, same box)
     constexpr int E = 16 / sizeof(T);
     const int step = kRowsThreads * E;
     int bvec = -1;
