@@ -133,9 +133,18 @@ def lib():
 # ----------------------------------------------------------------------------- marshalling helpers
 
 def _ptr(x) -> Optional[int]:
+    """Device address of a CUDA tensor, or an integer address passed through.
+
+    Every pointer the library's entry points take through this helper is a
+    device pointer into a row-major layout, so a host tensor or a strided
+    view is refused here instead of reaching a kernel."""
     if x is None:
         return None
     if isinstance(x, torch.Tensor):
+        if not x.is_cuda:
+            raise ValueError("expected a CUDA tensor: the library's entry points take device pointers")
+        if not x.is_contiguous():
+            raise ValueError("expected a contiguous tensor: the library's layouts are dense row-major")
         return x.data_ptr()
     return int(x)
 

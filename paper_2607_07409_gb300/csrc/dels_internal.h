@@ -320,6 +320,10 @@ cudaError_t launch_vocab_combine_f32(const float* feat, int K, const float* Wv, 
 // ---- host utilities ---------------------------------------------------------
 int device_sm_count();
 int device_max_smem_optin();
+// Raises `kernel`'s dynamic shared-memory limit on the current device to at
+// least `bytes`, once per kernel, device and size (safe from several host
+// threads; the attribute is per device).
+cudaError_t ensure_dynamic_smem(const void* kernel, size_t bytes);
 bool encode_tmap_2d(CUtensorMap* m, const void* base, CUtensorMapDataType dt, int elem_bytes, uint64_t inner,
                     uint64_t outer, uint64_t row_pitch_bytes, uint32_t box_inner, uint32_t box_outer,
                     CUtensorMapSwizzle swz);

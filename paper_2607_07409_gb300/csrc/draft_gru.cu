@@ -459,16 +459,8 @@ size_t draft_gru_smem_bytes(const PersistGruArgs& P) { return smem_layout(P).tot
 
 cudaError_t launch_draft_gru(const PersistGruArgs& P, const CUtensorMap* maps, int grid, size_t smem,
                              cudaStream_t s) {
-  static int configured_bytes[64] = {0};
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
+  cudaError_t e = ensure_dynamic_smem(reinterpret_cast<const void*>(k_draft_gru), smem);
   if (e != cudaSuccess) return e;
-  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
-  if ((int)smem > configured_bytes[dev]) {
-    e = cudaFuncSetAttribute(k_draft_gru, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    configured_bytes[dev] = (int)smem;
-  }
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
   cfg.blockDim = dim3(kThreads);

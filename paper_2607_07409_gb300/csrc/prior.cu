@@ -514,26 +514,9 @@ __global__ void __launch_bounds__(kMapThreads) k_prior_log(PriorLogArgs a) {
   if (a.tally_out && blockIdx.x == 0 && threadIdx.x < 2) a.tally_out[threadIdx.x] = __ldcg(a.tally + threadIdx.x);
 }
 
-int max_smem_optin() {
-  static int v = -1;
-  if (v < 0) {
-    int dev = 0, x = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess ||
-        cudaDeviceGetAttribute(&x, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess)
-      x = 0;
-    v = x;
-  }
-  return v;
-}
-
 // CTAs per SM that one k_prior_slices launch can keep resident
 int slices_per_sm(size_t smem) {
-  static size_t set_for = 0;
-  if (set_for < smem) {
-    if (cudaFuncSetAttribute(k_prior_slices, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
-      return 0;
-    set_for = smem;
-  }
+  if (ensure_dynamic_smem(reinterpret_cast<const void*>(k_prior_slices), smem) != cudaSuccess) return 0;
   int v = 0;
   if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, k_prior_slices, kThreads, smem) != cudaSuccess) return 0;
   return v;
@@ -543,7 +526,7 @@ int slices_per_sm(size_t smem) {
 
 PriorPlan plan_prior(int V, long long N, int sms) {
   PriorPlan p{};
-  const int smem = max_smem_optin();
+  const int smem = device_max_smem_optin();
   if (smem <= 0 || sms <= 0 || V < 1) return p;
   // slices: the bins take all but a little of the shared memory
   const int bins_max = (smem - 2048) / 4;
@@ -582,13 +565,9 @@ cudaError_t launch_prior_select(const PriorSelectArgs& a, int ctas, cudaStream_t
 }
 
 cudaError_t launch_prior_hot(const PriorHotArgs& a, size_t smem, cudaStream_t s) {
-  static size_t set_for = 0;
-  if (set_for < smem) {
-    cudaError_t e = cudaFuncSetAttribute(k_prior_hot, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    set_for = smem;
-  }
-  cudaError_t e = launch_pdl(k_prior_hot, dim3((unsigned)a.ctas), dim3(kThreads), smem, s, a);
+  cudaError_t e = ensure_dynamic_smem(reinterpret_cast<const void*>(k_prior_hot), smem);
+  if (e != cudaSuccess) return e;
+  e = launch_pdl(k_prior_hot, dim3((unsigned)a.ctas), dim3(kThreads), smem, s, a);
   if (e != cudaSuccess) return e;
   const int kw = (a.K + 1) / 2;
   const int blocks = std::max(1, std::min(a.ctas * 4, (kw + kMapThreads - 1) / kMapThreads));

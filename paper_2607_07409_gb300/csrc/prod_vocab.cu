@@ -26,6 +26,7 @@
 // warp 1 MMA issuer / TMEM owner, warps 2..9 epilogue, warp 10 logits
 // producer. The ring is one FIFO across the two phases: the products' fills
 // come first, then the vocabulary's.
+#include <atomic>
 #include <climits>
 
 #include "tc_engine.cuh"
@@ -345,16 +346,12 @@ size_t prod_vocab_smem_bytes(const ProdVocabArgs& P) { return pv_layout(P).total
 
 cudaError_t launch_prod_vocab(const ProdVocabArgs& P, const CUtensorMap* maps, int grid, size_t smem,
                               cudaStream_t s) {
-  static int configured_bytes[64] = {0};
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
-  if ((int)smem > configured_bytes[dev]) {
-    e = cudaFuncSetAttribute(k_prod_vocab, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    configured_bytes[dev] = (int)smem;
-  }
+  e = ensure_dynamic_smem(reinterpret_cast<const void*>(k_prod_vocab), smem);
+  if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
   cfg.blockDim = dim3(kThreads);
@@ -374,18 +371,18 @@ cudaError_t launch_prod_vocab(const ProdVocabArgs& P, const CUtensorMap* maps, i
   cfg.attrs = attr;
   // programmatic serialization with a cooperative launch where the runtime
   // allows it; plain stream order otherwise (remembered per device)
-  static int coop_pdl[64] = {0};   // 0 unknown, 1 allowed, -1 refused
-  cfg.numAttrs = coop_pdl[dev] >= 0 ? 3 : 2;
+  static std::atomic<int> coop_pdl[64];   // 0 unknown, 1 allowed, -1 refused (zero-initialised: static)
+  cfg.numAttrs = coop_pdl[dev].load() >= 0 ? 3 : 2;
   e = cudaLaunchKernelEx(&cfg, k_prod_vocab, maps[0], maps[1], maps[2], maps[3], maps[4], maps[5], P,
                          (uint64_t)kWaitBudgetNs);
-  if (e != cudaSuccess && cfg.numAttrs == 3 && coop_pdl[dev] == 0) {
+  if (e != cudaSuccess && cfg.numAttrs == 3 && coop_pdl[dev].load() == 0) {
     (void)cudaGetLastError();
-    coop_pdl[dev] = -1;
+    coop_pdl[dev].store(-1);
     cfg.numAttrs = 2;
     e = cudaLaunchKernelEx(&cfg, k_prod_vocab, maps[0], maps[1], maps[2], maps[3], maps[4], maps[5], P,
                            (uint64_t)kWaitBudgetNs);
   } else if (e == cudaSuccess && cfg.numAttrs == 3) {
-    coop_pdl[dev] = 1;
+    coop_pdl[dev].store(1);
   }
   return e;
 }

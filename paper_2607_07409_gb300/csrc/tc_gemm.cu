@@ -326,16 +326,8 @@ cudaError_t launch_tc_gemm(const TcGemmArgs& a, const CUtensorMap* mA0, const CU
   if (two && (second->a->epi == EPI_COMBINE) != comb) return cudaErrorInvalidValue;
   const int mode = comb ? (a.sample ? 2 : 1) : 0;
   auto kern = mode == 2 ? k_tc_gemm<2> : mode == 1 ? k_tc_gemm<1> : k_tc_gemm<0>;
-  static int configured_bytes[3][64] = {{0}};
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
+  cudaError_t e = ensure_dynamic_smem(reinterpret_cast<const void*>(kern), smem_bytes);
   if (e != cudaSuccess) return e;
-  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
-  if ((int)smem_bytes > configured_bytes[mode][dev]) {
-    e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_bytes);
-    if (e != cudaSuccess) return e;
-    configured_bytes[mode][dev] = (int)smem_bytes;
-  }
   const uint64_t budget = a.debug_skip_producer ? 100000000ull : kWaitBudgetNs;
   const int g0 = std::max(grid, 0);
   // clusters (split-K through distributed shared memory) cover the whole grid:

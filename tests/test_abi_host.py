@@ -210,3 +210,30 @@ def test_sampled_entry_points_reject_bad_arguments_before_enqueueing(dels):
     assert vcall(_19=None) == -5
     assert vcall(_3=p + 8) == -4
     assert vcall(_11=200) == -2                 # bf16 heads: B <= 128
+
+
+def test_binding_refuses_host_and_strided_tensors(dels):
+    """Device entry points take device pointers into dense row-major layouts:
+    the binding raises before a host or strided tensor reaches the library."""
+    rows, V = 2, 16
+    x = torch.zeros(rows, V, dtype=torch.bfloat16)
+    tok = torch.zeros(rows, dtype=torch.int32)
+    f = torch.zeros(rows)
+    with pytest.raises(ValueError, match="CUDA tensor"):
+        dels.dels_combine_argmax(x, x, dels.DELS_BF16, None, 0.0, 0.0, rows, V, tok, f, None, None, 0)
+    with pytest.raises(ValueError, match="CUDA tensor"):
+        dels.dels_verify_block(tok.view(rows, 1), x, dels.DELS_BF16, rows, 1, V, tok, tok, None, None, 0)
+    with pytest.raises(ValueError, match="contiguous"):
+        dels._ptr(_FakeStrided())
+
+
+class _FakeStrided(torch.Tensor):
+    """A CUDA-looking, non-contiguous tensor (no GPU needed to build it)."""
+
+    @staticmethod
+    def __new__(cls):
+        return torch.Tensor._make_subclass(cls, torch.zeros(4, 4).t())
+
+    @property
+    def is_cuda(self):
+        return True
