@@ -119,3 +119,33 @@ def test_qwen3_8b_batched_full_size_temperature_one():
     ok = (acc == r_acc) & ~close
     assert np.all((bonus == r_bonus) | ~ok | (vinfo["bonus_gap"] < 0.05)), (bonus, r_bonus, vinfo["bonus_gap"])
     print({k: v for k, v in info.items() if k != "ref"}, "accept", acc.tolist(), r_acc.tolist())
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_combine_full_size_8b_shape(dtype):
+    """dels_combine_argmax over the 8B workload's B*n = 1024 rows of V = 151936
+    (three column chunks per row, the last CTA of each row merging them), in
+    the launch configuration the sweep times; rows are independent, so the
+    oracle on sampled rows is exact for them."""
+    w = synth.WORKLOADS["qwen3_8b_batched"]
+    rows_n, V = w.B * w.n, w.V
+    d = synth.make_combine_inputs(rows_n, V, dtype, seed=88, device=DEV)
+    prior = oracle.log_prior(d["counts"]).astype(np.float32)
+    dt = dels.dtype_code(d["long"])
+    nbytes = dels.dels_combine_workspace_bytes(rows_n, V, dt)
+    ws = torch.zeros(nbytes, dtype=torch.uint8, device=DEV)
+    tok = torch.full((rows_n,), -7, dtype=torch.int32, device=DEV)
+    lp = torch.empty(rows_n, dtype=torch.float32, device=DEV)
+    gap = torch.empty(rows_n, dtype=torch.float32, device=DEV)
+    a = b = 0.3
+    assert dels.dels_combine_argmax(d["long"], d["short"], dt, torch.from_numpy(prior).to(DEV), a, b, rows_n, V,
+                                    tok, lp, gap, ws, nbytes) == 0
+    torch.cuda.synchronize()
+    assert dels.dels_read_status(ws) == 0
+    rows = [0, 1, 337, 511, 512, 1000, 1023]
+    rt, rl, rg = oracle.combine_argmax(d["long"][rows].cpu(), d["short"][rows].cpu(), prior.astype(np.float64), a, b)
+    fused = oracle.fuse(oracle.to_f64(d["long"][rows].cpu()), oracle.to_f64(d["short"][rows].cpu()),
+                        prior.astype(np.float64), a, b)
+    from parity import check_rows
+    print(check_rows(tok.cpu().numpy()[rows], lp.cpu().numpy()[rows], gap.cpu().numpy()[rows], rt, rl, rg,
+                     fused=fused))
