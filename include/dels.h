@@ -11,8 +11,11 @@
  *
  * Each block position is decoded from softmax(l) and fed back to the local
  * head; the finished block is verified by the target model (Algorithm 1).
- * This library runs that loop at temperature 0 (Decode = argmax, lowest
- * vocabulary index on exact ties) as hand-written CUDA kernels.
+ * This library runs that loop as hand-written CUDA kernels at temperature 0
+ * (Decode = argmax, lowest vocabulary index on exact ties; greedy
+ * verification) and at temperature 1 (Decode = a Gumbel-max draw; lossless
+ * speculative-sampling verification), and estimates the unigram prior from a
+ * corpus on the device (Appendix A).
  *
  * Conventions shared by every entry point
  * ---------------------------------------
@@ -26,7 +29,9 @@
  *   *_workspace_bytes function returns for the same arguments on the current
  *   device. A workspace must be zero-filled once before its first use (for
  *   example with cudaMemset); every call leaves it ready for the next call.
- *   Calls that share a workspace must be ordered on one stream.
+ *   Calls that share a workspace must be ordered on one stream. Calls with
+ *   distinct workspaces may be issued from several host threads at once
+ *   (the profiler switches below excepted).
  * - Return value: DELS_OK (0) or a negative DELS_ERR_* code detected on the
  *   host, in which case nothing was enqueued. Errors detected on the device
  *   (non-finite logits, an out-of-range token, a timed-out wait) are OR-ed
