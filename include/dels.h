@@ -31,7 +31,8 @@
  *   example with cudaMemset); every call leaves it ready for the next call.
  *   Calls that share a workspace must be ordered on one stream. Calls with
  *   distinct workspaces may be issued from several host threads at once
- *   (the profiler switches below excepted).
+ *   (except the profiler switches, and dels_combine_argmax_noalloc, whose
+ *   calls share one scratch per device).
  * - Return value: DELS_OK (0) or a negative DELS_ERR_* code detected on the
  *   host, in which case nothing was enqueued. Errors detected on the device
  *   (non-finite logits, an out-of-range token, a timed-out wait) are OR-ed
