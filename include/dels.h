@@ -24,7 +24,9 @@
  *   and 16-byte aligned. Pointers marked [host] are ordinary host memory.
  * - Calls are asynchronous on the given stream (a cudaStream_t; NULL is the
  *   legacy default stream) and never synchronise, except dels_read_status.
- * - The library allocates no memory and keeps no state between calls. Every
+ * - The library allocates no memory and keeps no state between calls, with
+ *   one exception: dels_combine_argmax_noalloc keeps a fixed scratch array per
+ *   device and caches its address (see there). Every other
  *   call takes a caller-owned device workspace of at least the size its
  *   *_workspace_bytes function returns for the same arguments on the current
  *   device. A workspace must be zero-filled once before its first use (for
@@ -244,8 +246,10 @@ int dels_combine_argmax(const void* long_logits, const void* short_logits, dels_
  * 4 MiB returns DELS_ERR_TOO_LARGE and enqueues nothing; at V = 151936 that
  * is reached only beyond roughly 200,000 rows.
  * Set-up: the first call on a device, with that device current, looks up
- * the scratch's device address (cudaGetSymbolAddress); make that first call
- * before any stream capture.
+ * the scratch's device address (cudaGetSymbolAddress) and caches it for the
+ * rest of the process; make that first call before any stream capture. The
+ * cached address does not survive cudaDeviceReset: after a reset of the
+ * device, do not call this entry point again in the same process.
  * The call allocates nothing (no cudaMalloc, cudaFree or allocating library
  * routine). It clears the part of the scratch that must start at zero with
  * cudaMemsetAsync on `stream`. All calls on a device share the one scratch,

@@ -881,6 +881,20 @@ size_t dels_combine_workspace_bytes(int rows, int V, dels_dtype dtype) {
   return off;
 }
 
+}  // extern "C"
+
+namespace dels {
+int combine_check_inputs(const void* long_logits, const void* short_logits, const float* log_prior,
+                         const int32_t* out_token) {
+  if (!long_logits || !out_token) return DELS_ERR_NULL_POINTER;
+  if (!aligned16(long_logits) || (short_logits && !aligned16(short_logits)) || (log_prior && !aligned16(log_prior)))
+    return DELS_ERR_ALIGNMENT;
+  return DELS_OK;
+}
+}  // namespace dels
+
+extern "C" {
+
 int dels_combine_argmax(const void* long_logits, const void* short_logits, dels_dtype dtype, const float* log_prior,
                         float alpha, float beta, int rows, int V, int32_t* out_token, float* out_logprob,
                         float* out_top2_gap, void* workspace, size_t workspace_bytes, dels_stream_t stream) {
@@ -888,10 +902,9 @@ int dels_combine_argmax(const void* long_logits, const void* short_logits, dels_
   if (rows < 0 || V < 1) return DELS_ERR_BAD_SHAPE;
   if (!workspace) return DELS_ERR_WORKSPACE;
   if (rows == 0) return DELS_OK;
-  if (!long_logits || !out_token) return DELS_ERR_NULL_POINTER;
-  if (!aligned16(long_logits) || (short_logits && !aligned16(short_logits)) || (log_prior && !aligned16(log_prior)) ||
-      !aligned16(workspace))
-    return DELS_ERR_ALIGNMENT;
+  const int chk = combine_check_inputs(long_logits, short_logits, log_prior, out_token);
+  if (chk != DELS_OK) return chk;
+  if (!aligned16(workspace)) return DELS_ERR_ALIGNMENT;
   const size_t need = dels_combine_workspace_bytes(rows, V, dtype);
   if (need == 0) return DELS_ERR_CUDA;
   if (workspace_bytes < need) return DELS_ERR_WORKSPACE;

@@ -318,6 +318,11 @@ cudaError_t launch_vocab_combine_f32(const float* feat, int K, const float* Wv, 
                                      const SampleArgs* smp = nullptr, int j = 0);
 
 // ---- host utilities ---------------------------------------------------------
+// Host-side checks of dels_combine_argmax's input and output pointers (NULL,
+// 16-byte alignment), shared with the no-allocation variant so that both
+// reject the same calls before anything is enqueued.
+int combine_check_inputs(const void* long_logits, const void* short_logits, const float* log_prior,
+                         const int32_t* out_token);
 int device_sm_count();
 int device_max_smem_optin();
 // Raises `kernel`'s dynamic shared-memory limit on the current device to at

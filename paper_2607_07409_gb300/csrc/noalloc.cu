@@ -10,7 +10,10 @@
 // library holds it until the process exits. Host code cannot use the array's
 // name as a device address (in host code it is only a stand-in symbol), so
 // the first call on each device looks the address up with
-// cudaGetSymbolAddress while that device is current and caches it.
+// cudaGetSymbolAddress while that device is current and caches it. The cache
+// assumes the device is not reset while the process runs: after
+// cudaDeviceReset the cached address is stale and the entry point must not
+// be called again in that process.
 #include <mutex>
 
 #include "dels_internal.h"
@@ -54,6 +57,10 @@ extern "C" int dels_combine_argmax_noalloc(const void* long_logits, const void* 
   if (dtype != DELS_F32 && dtype != DELS_BF16) return DELS_ERR_BAD_DTYPE;
   if (rows < 0 || V < 1) return DELS_ERR_BAD_SHAPE;
   if (rows == 0) return DELS_OK;
+  // every host-side check of dels_combine_argmax runs before the scratch is
+  // touched, so a rejected call enqueues nothing (not even the clearing)
+  const int chk = combine_check_inputs(long_logits, short_logits, log_prior, out_token);
+  if (chk != DELS_OK) return chk;
   const size_t need = dels_combine_workspace_bytes(rows, V, dtype);
   if (need == 0) return DELS_ERR_CUDA;
   if (need > kNoAllocScratchBytes) return DELS_ERR_TOO_LARGE;

@@ -142,6 +142,10 @@ def test_combine_full_size_8b_shape(dtype):
                                     tok, lp, gap, ws, nbytes) == 0
     torch.cuda.synchronize()
     assert dels.dels_read_status(ws) == 0
+    # every row was written: a token in range, a finite log-probability <= 0
+    tok_all, lp_all = tok.cpu().numpy(), lp.cpu().numpy()
+    assert ((tok_all >= 0) & (tok_all < V)).all()
+    assert np.isfinite(lp_all).all() and (lp_all <= 0).all()
     rows = [0, 1, 337, 511, 512, 1000, 1023]
     rt, rl, rg = oracle.combine_argmax(d["long"][rows].cpu(), d["short"][rows].cpu(), prior.astype(np.float64), a, b)
     fused = oracle.fuse(oracle.to_f64(d["long"][rows].cpu()), oracle.to_f64(d["short"][rows].cpu()),

@@ -56,6 +56,47 @@ def test_no_alloc_combine_matches_workspace_combine_twice():
         assert np.abs(got[2].cpu().numpy() - ref[2].cpu().numpy()).max() <= 2 * LP_TOL_COMBINE
 
 
+def test_no_alloc_combine_many_rows_and_a_non_finite_row():
+    """The four-rows-per-CTA plan (rows >= 64 x SMs), where the cleared ticket
+    region has its largest size, and a row holding a NaN: the workspace status
+    word is not readable here, so the row must come back as token -1 with a
+    NaN log-probability while every other row matches the workspace combine."""
+    rows, V = 20000, 64
+    d = synth.make_combine_inputs(rows, V, "f32", seed=23, device=DEV)
+    long = d["long"].clone()
+    long[777, 5] = float("nan")
+    prior = dels.dels_prior_from_counts(d["counts"]).to(DEV)
+    got = _no_alloc(long, d["short"], prior, 0.5)
+    ref = _with_workspace(long, d["short"], prior, 0.5)
+    torch.cuda.synchronize()
+    tok, lp = got[0].cpu().numpy(), got[1].cpu().numpy()
+    assert tok[777] == -1 and np.isnan(lp[777])
+    np.testing.assert_array_equal(tok, ref[0].cpu().numpy())
+    keep = np.arange(rows) != 777
+    assert np.abs(lp[keep] - ref[1].cpu().numpy()[keep]).max() <= LP_TOL_COMBINE
+    assert ((tok[keep] >= 0) & (tok[keep] < V)).all()
+
+
+def test_no_alloc_combine_rejects_bad_pointers_before_touching_its_scratch():
+    """A rejected call enqueues nothing: a misaligned input is refused before
+    the scratch is cleared, and the next call still matches the workspace path."""
+    rows, V = 9, 4096
+    d = synth.make_combine_inputs(rows, V, "bf16", seed=24, device=DEV)
+    prior = dels.dels_prior_from_counts(d["counts"]).to(DEV)
+    flat = d["long"].reshape(-1)
+    out = [torch.empty(rows, dtype=torch.int32, device=DEV), torch.empty(rows, device=DEV), None]
+    r = dels.dels_combine_argmax_noalloc(flat[1:], d["short"], dels.dtype_code(flat), prior, 0.5, 0.5, rows, V - 1,
+                                         *out)
+    assert r == dels.DELS_ERR_ALIGNMENT
+    r = dels.dels_combine_argmax_noalloc(d["long"], d["short"], dels.dtype_code(flat), prior, 0.5, 0.5, rows, V,
+                                         None, None, None)
+    assert r == dels.DELS_ERR_NULL_POINTER
+    got = _no_alloc(d["long"], d["short"], prior, 0.5)
+    ref = _with_workspace(d["long"], d["short"], prior, 0.5)
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(got[0].cpu().numpy(), ref[0].cpu().numpy())
+
+
 def test_no_alloc_combine_rejects_problems_beyond_its_scratch():
     rows, V = 300000, 64
     big = torch.zeros(1, device=DEV)          # never read: the call must refuse before launching
