@@ -14,6 +14,13 @@ plus a Zipf(1.1) bias, target logits = DFlash + N(0, 1). Synthetic data; the
 paper's checkpoints and benchmark prompts are not used.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                  [--workload qwen3_8b_batched|qwen3_4b|qwen3_0p6b|tiny]
+
+--workload picks one of the other Qwen3-shaped drafting workloads (same
+step, their own head and logits): Qwen3-4B-shaped (B = 8, 1-layer causal
+transformer head, d 2560, FFN 10240, float32 logits), Qwen3-0.6B-shaped
+(B = 1, 2-layer window MLP head over the last 4 tokens, hidden 1024, float32
+logits) and the tiny case (B = 1, V = 1024, float32 MLP head).
 
 Prints one JSON line (rank 0). N > 1 runs one independent replica per GPU
 (launched by torchrun): the drafting path has no cross-request exchange.
@@ -37,7 +44,10 @@ sys.path.insert(0, ROOT)
 METRIC = "drafted tokens/sec on 1 GB300; combine/argmax HBM GB/s vs 8 TB/s; oracle match"
 UNIT = "drafted tokens/s"
 WORKLOAD = "qwen3_8b_batched"
+WORKLOADS = ("qwen3_8b_batched", "qwen3_4b", "qwen3_0p6b", "tiny")
 FALLBACK_HBM_GBS = 6800.0
+NOMINAL_HBM_GBS = 8000.0      # the "8 TB/s" of the metric (GB300 HBM3e nominal, rounded)
+L2_BYTES = 129e6
 
 
 def parse_args():
@@ -68,6 +78,11 @@ def parse_args():
     p.add_argument("--no-input-table", action="store_true",
                    help="recompute the GRU input product W_ih E[x] at every position instead of reading the "
                         "precomputed table G = E W_ih^T")
+    p.add_argument("--workload", choices=WORKLOADS, default=WORKLOAD,
+                   help="drafting workload of the step (default: the Qwen3-8B-shaped batched drafting)")
+    p.add_argument("--cpu-positions", type=int, default=0,
+                   help="block positions in the CPU-oracle sample (0: the workload's default)")
+    p.add_argument("--oracle-single-thread", action="store_true", help=argparse.SUPPRESS)
     return p.parse_args()
 
 
@@ -180,33 +195,91 @@ def _isnum(s):
         return False
 
 
+def _es(dtype):
+    return 4 if dtype == "f32" else 2
+
+
 def algorithmic_vocab_bytes(w):
     """Bytes one vocabulary-projection + combine launch must move: W_vocab once,
-    the DFlash logits of one position for every request, the prior, and r."""
+    the DFlash logits of one position for every request, the prior, and the
+    projection's input r."""
     h = w.head
-    return w.V * h.d_rank * 2 + w.B * w.V * 2 + w.V * 4 + w.B * h.d_rank * 2
+    esw, esl = _es(h.wdtype), _es(w.logit_dtype)
+    return w.V * h.d_rank * esw + w.B * w.V * esl + w.V * 4 + w.B * h.d_rank * esw
 
 
-def algorithmic_block_bytes(w):
-    """Bytes of one drafted block with every weight streamed once per position
-    (positions 1..n-1) plus the DFlash logits and prior."""
+def head_weight_bytes(w, table=False):
+    """Bytes of the local head's own weights streamed at one drafted position,
+    and of the inputs it gathers per position. table: the GRU's input product
+    is read as B rows of G = E W_ih^T (3 * d_hidden float32 each) instead of
+    streaming W_ih and gathering E rows."""
     h = w.head
-    per_pos = (w.V * h.d_rank * 2 + 3 * h.d_hidden * (h.d_model + h.d_hidden) * 2 + h.d_rank * h.d_hidden * 2
-               + w.B * w.V * 2 + w.V * 4 + w.B * h.d_model * 2)
-    return (w.n - 1) * per_pos + w.B * w.V * 2
+    esw = _es(h.wdtype)
+    if h.kind == "gru":
+        if table:
+            return (3 * h.d_hidden * h.d_hidden + h.d_rank * h.d_hidden) * esw, w.B * 3 * h.d_hidden * 4
+        return (3 * h.d_hidden * (h.d_model + h.d_hidden) + h.d_rank * h.d_hidden) * esw, w.B * h.d_model * esw
+    if h.kind == "mlp":
+        wb = h.d_hidden * h.window * h.d_model + (h.d_hidden * h.d_hidden if h.n_layers == 2 else 0)
+        return wb * esw, w.B * h.window * h.d_model * esw
+    if h.kind == "xfmr":
+        D, F = h.d_model, h.d_hidden
+        return (4 * D * D + 2 * D * F) * esw, w.B * D * esw
+    return 0, w.B * h.d_rank * esw                       # markov: one E_M row per request
 
 
-def input_table_block_bytes(w):
-    """Bytes of one drafted block on the input-table path: as above, but the
-    W_ih stream of every position is replaced by B gathered rows of G
-    (3 * d_hidden float32 each)."""
+def step_bytes(w, table=False):
+    """Algorithmic bytes of one step (drafted block + verification): every
+    weight once per drafted position j >= 1, W_vocab included, the DFlash
+    logits of every position, the prior, the gathered head inputs, and the
+    n + 1 target rows of every request. table=False is the streaming model
+    (every head weight, W_ih included); table=True what the GRU input-table
+    path reads."""
     h = w.head
-    per_pos = (w.V * h.d_rank * 2 + 3 * h.d_hidden * h.d_hidden * 2 + h.d_rank * h.d_hidden * 2
-               + w.B * w.V * 2 + w.V * 4 + w.B * 3 * h.d_hidden * 4)
-    return (w.n - 1) * per_pos + w.B * w.V * 2
+    esl = _es(w.logit_dtype)
+    hw, gather = head_weight_bytes(w, table)
+    per_pos = w.V * h.d_rank * _es(h.wdtype) + hw + w.B * w.V * esl + w.V * 4 + gather
+    return (w.n - 1) * per_pos + w.B * w.V * esl + w.B * (w.n + 1) * w.V * esl
 
 
 # ----------------------------------------------------------------------------- CPU oracle leg
+
+def default_cpu_positions(w):
+    """Block positions in the CPU-oracle sample: the oracle decodes W_vocab to
+    float64 at every position, which dominates for the wide heads."""
+    return {"qwen3_4b": 6, "qwen3_0p6b": 12}.get(w.name, w.n)
+
+
+def oracle_single_thread(args):
+    """Child process: the oracle sample on one host thread (BLAS pinned to one
+    thread by the parent's environment, torch's intra-op pool set to one);
+    inputs from the same generators on the host. Prints one JSON line."""
+    import torch
+    import synth
+    w = synth.WORKLOADS[args.workload]
+    d = synth.make_inputs(w, device="cpu")
+    torch.set_num_threads(1)
+    positions = args.cpu_positions or default_cpu_positions(w)
+    rows = min(args.cpu_rows, w.B)
+    ntok, dt, _, _ = oracle_sample(w, d, rows, positions)
+    print(json.dumps({"tokens": ntok, "seconds": dt, "rows": rows, "positions": positions}), flush=True)
+    return 0
+
+
+def single_thread_baseline(args, w):
+    """The oracle sample timed on one host thread in a child process (None on failure)."""
+    env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1")
+    cmd = [sys.executable, os.path.join(ROOT, "bench.py"), "--oracle-single-thread", "--workload", w.name,
+           "--cpu-rows", str(max(1, min(args.cpu_rows, 2))), "--cpu-positions", str(args.cpu_positions)]
+    try:
+        r = subprocess.run(cmd, env=env, capture_output=True, text=True, timeout=600)
+        out = json.loads(r.stdout.strip().splitlines()[-1])
+    except Exception:
+        return None
+    return {"value": out["tokens"] / out["seconds"], "unit": UNIT, "cores": 1,
+            "sample": f"{out['rows']} of {w.B} requests x positions 0..{out['positions'] - 1} of {w.name} "
+                      f"(inputs from the host generators)"}
+
 
 def oracle_sample(w, d, rows, positions, gpu_tokens=None):
     """Time the oracle on `rows` requests x `positions` positions of the block
@@ -248,9 +321,9 @@ def run_reference(args):
         return 0
     import torch
     import synth
-    w = synth.WORKLOADS[WORKLOAD]
+    w = synth.WORKLOADS[args.workload]
     d = synth.make_inputs(w, device="cpu")
-    rows, positions = 1, 4
+    rows, positions = 1, min(4, w.n)
     for _ in range(args.warmup):
         oracle_sample(w, d, rows, positions)
     times = []
@@ -261,12 +334,12 @@ def run_reference(args):
         times.append(dt)
     total = sum(times)
     value = tokens / total
-    sample = f"{rows} of {w.B} requests x positions 0..{positions - 1} of {WORKLOAD} per step"
+    sample = f"{rows} of {w.B} requests x positions 0..{positions - 1} of {w.name} per step"
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * total / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": WORKLOAD, "B": w.B, "n": w.n, "V": w.V, "head": "gru 4096/1024/256"},
+        "config": {"workload": w.name, "B": w.B, "n": w.n, "V": w.V, "head": head_desc(w)},
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle", "sample": sample},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
@@ -275,6 +348,17 @@ def run_reference(args):
 
 
 # ----------------------------------------------------------------------------- our arm
+
+def head_desc(w):
+    h = w.head
+    if h.kind == "gru":
+        return f"gru emb {h.d_model} / hidden {h.d_hidden} / rank {h.d_rank}, {h.wdtype}"
+    if h.kind == "mlp":
+        return f"{h.n_layers}-layer window-{h.window} mlp, d {h.d_model} / hidden {h.d_hidden}, {h.wdtype}"
+    if h.kind == "xfmr":
+        return f"1-layer causal transformer d {h.d_model} / {h.n_heads} heads / ffn {h.d_hidden}, {h.wdtype}"
+    return f"markov d {h.d_rank}, {h.wdtype}"
+
 
 def run_ours(args):
     import torch
@@ -288,14 +372,16 @@ def run_ours(args):
     dev = torch.device(f"cuda:{local}")
     torch.cuda.set_device(dev)
     # weak scaling: every replica drafts its own batch of the same shape
-    w0 = synth.WORKLOADS[WORKLOAD]
+    w0 = synth.WORKLOADS[args.workload]
     w = synth.with_sizes(w0, seed=replicas.replica_seed(w0.seed, rank))
     d = synth.make_inputs(w, device=dev)
     W = {k[5:]: v for k, v in d.items() if k.startswith("head.")}
     prior = dels.dels_prior_from_counts(d["counts"]).to(dev)
     long, target = d["long"], d["target"]
+    ldt, tdt = dels.dtype_code(long), dels.dtype_code(target)
     table_ms = None
-    if not args.no_input_table:
+    use_table = w.head.kind == "gru" and w.head.wdtype == "bf16" and not args.no_input_table
+    if use_table:
         # head preparation, once per set of weights (not part of a step)
         torch.cuda.synchronize()
         t0 = time.perf_counter()
@@ -303,16 +389,15 @@ def run_ours(args):
         torch.cuda.synchronize()
         table_ms = 1e3 * (time.perf_counter() - t0)
     drafter = dels.Drafter(w.head, W, w.B, w.n, w.V)
-    vbytes = dels.dels_verify_workspace_bytes(w.B, w.n, w.V, dels.DELS_BF16)
+    vbytes = dels.dels_verify_workspace_bytes(w.B, w.n, w.V, tdt)
     vws = torch.zeros(vbytes, dtype=torch.uint8, device=dev)
     acc = torch.empty(w.B, dtype=torch.int32, device=dev)
     bonus = torch.empty(w.B, dtype=torch.int32, device=dev)
     stream = torch.cuda.current_stream()
 
-    def step(long_in, target_in):
-        tok, lp, gap = drafter(long_in, prior, w.alpha, w.beta, stream)
-        r = dels.dels_verify_block(tok, target_in, dels.DELS_BF16, w.B, w.n, w.V, acc, bonus, None, vws, vbytes,
-                                   stream)
+    def step(long_in, target_in, st=stream):
+        tok, lp, gap = drafter(long_in, prior, w.alpha, w.beta, st)
+        r = dels.dels_verify_block(tok, target_in, tdt, w.B, w.n, w.V, acc, bonus, None, vws, vbytes, st)
         if r != 0:
             raise dels.DelsError(r, "dels_verify_block")
         return tok
@@ -323,8 +408,14 @@ def run_ours(args):
     if drafter.status() != 0 or dels.dels_read_status(vws) != 0:
         raise RuntimeError("device status set during warm-up")
 
-    # ---- timed region: device-resident inputs (long 311 MB + target 331 MB per step > L2)
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    moved = step_bytes(w, table=use_table)
+    survey = step_bytes(w, table=False)
+    # a step whose bytes fit in L2 is timed launch by launch with an L2 flush
+    # (a write larger than L2) between steps, outside the timed brackets
+    flush_l2 = moved < 2 * L2_BYTES
+    flush = torch.empty(int(2 * L2_BYTES), dtype=torch.uint8, device=dev) if flush_l2 else None
+
+    # ---- timed region: device-resident inputs
     gpu_id = local
     try:
         gpu_id = "GPU-" + str(torch.cuda.get_device_properties(dev).uuid)
@@ -341,26 +432,39 @@ def run_ours(args):
         cap.wait_stream(stream)
         graph = torch.cuda.CUDAGraph()
         with torch.cuda.graph(graph, stream=cap):
-            gr_tok = drafter(long, prior, w.alpha, w.beta, cap)[0]
-            r = dels.dels_verify_block(gr_tok, target, dels.DELS_BF16, w.B, w.n, w.V, acc, bonus, None, vws, vbytes,
-                                       cap)
-            if r != 0:
-                raise dels.DelsError(r, "dels_verify_block")
+            step(long, target, cap)
         stream.wait_stream(cap)
         for _ in range(3):
             graph.replay()
         torch.cuda.synchronize()
+
+    def one():
+        if graph is not None:
+            graph.replay()
+        else:
+            step(long, target)
+
     with ClockSampler(gpu_id) as clk:
-        e0.record(stream)
-        for _ in range(args.steps):
-            if graph is not None:
-                graph.replay()
-            else:
-                step(long, target)
-        e1.record(stream)
-        torch.cuda.synchronize()
+        if flush_l2:
+            evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                   for _ in range(args.steps)]
+            for i in range(args.steps):
+                flush.fill_(i & 0xFF)
+                evs[i][0].record(stream)
+                one()
+                evs[i][1].record(stream)
+            torch.cuda.synchronize()
+            ms_local = sum(a.elapsed_time(b) for a, b in evs)
+        else:
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            for _ in range(args.steps):
+                one()
+            e1.record(stream)
+            torch.cuda.synchronize()
+            ms_local = e0.elapsed_time(e1)
     replicas.barrier()
-    ms_max = replicas.max_over_ranks(e0.elapsed_time(e1), dev)
+    ms_max = replicas.max_over_ranks(ms_local, dev)
 
     # ---- second timed region, same steps, with the library's per-kernel CUDA
     # events on (they serialise the kernels, so the value above is taken without)
@@ -396,13 +500,11 @@ def run_ours(args):
         achieved = algorithmic_vocab_bytes(w) / per_launch_s / 1e9
         roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
                     "frac": round(achieved / peak, 4), "peak_source": peak_kind,
-                    "kernel": "k_tc_gemm (vocab projection + fused combine)",
+                    "frac_of_nominal_8tbs": round(achieved / NOMINAL_HBM_GBS, 4),
+                    "kernel": ("k_tc_gemm<1> (vocab projection + fused combine)" if w.head.wdtype == "bf16" else
+                               "k_vocab_combine_f32 (vocab projection + fused combine, CUDA cores)"),
                     "algorithmic_bytes_per_launch": algorithmic_vocab_bytes(w),
-                    "traffic": ncu_traffic(f"vocab_combine_{WORKLOAD}.md")}
-    # whole step = drafted block + verification of its n + 1 target rows
-    verify_bytes = w.B * (w.n + 1) * w.V * 2
-    block_bytes = algorithmic_block_bytes(w) + verify_bytes
-    moved = block_bytes if table_ms is None else input_table_block_bytes(w) + verify_bytes
+                    "traffic": ncu_traffic(f"vocab_combine_{w.name}.md")}
     step_s = ms_max / args.steps * 1e-3
 
     # ---- end to end through the public API with host buffers
@@ -441,34 +543,44 @@ def run_ours(args):
     match = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         gpu_tok = drafter.tokens.cpu().numpy()
-        ntok, dt, match, _ = oracle_sample(w, d, args.cpu_rows, w.n, gpu_tokens=gpu_tok)
+        rows = min(args.cpu_rows, w.B)
+        positions = args.cpu_positions or default_cpu_positions(w)
+        ntok, dt, match, _ = oracle_sample(w, d, rows, positions, gpu_tokens=gpu_tok)
         cpu = {"value": ntok / dt, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
-               "sample": f"{args.cpu_rows} of {w.B} requests x all {w.n} positions of {WORKLOAD} "
-                         f"(+ their verification), forced to the device's tokens"}
+               "sample": f"{rows} of {w.B} requests x positions 0..{positions - 1} of {w.name} "
+                         f"({'+ their verification, ' if positions == w.n else ''}forced to the device's tokens)",
+               "single_thread": single_thread_baseline(args, w)}
 
     if rank == 0:
+        esl = _es(w.logit_dtype)
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": max(3, args.warmup), "ms_per_step": ms_max / args.steps, "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-            "config": {"workload": WORKLOAD, "B": w.B, "n": w.n, "V": w.V,
-                       "head": "gru emb 4096 / hidden 1024 / rank 256, bf16", "alpha": w.alpha, "beta": w.beta,
+            "scaling": "weak", "vs_baseline": None, "dtype": w.head.wdtype, "data": "synthetic",
+            "config": {"workload": w.name, "B": w.B, "n": w.n, "V": w.V, "head": head_desc(w),
+                       "logits": f"{w.logit_dtype} DFlash and target logits",
+                       "alpha": w.alpha, "beta": w.beta,
                        "step": "dels_draft_block + dels_verify_block",
                        "launch": ("stream launches" if args.no_graph else
                                   "CUDA graph of the step (captured once, replayed)"),
-                       "gru_input": ("W_ih E[x] recomputed every position" if table_ms is None else
+                       "gru_input": (None if w.head.kind != "gru" else
+                                     "W_ih E[x] recomputed every position" if table_ms is None else
                                      f"table G = E W_ih^T ({w.V * 3 * w.head.d_hidden * 4 / 1e9:.2f} GB f32) "
                                      f"built once before timing in {table_ms:.1f} ms"),
-                       "l2": "inputs larger than L2 (long 311 MB + target 331 MB per step, not flushed)",
+                       "l2": ("L2 flushed (a 258 MB write) before every step; steps timed one by one"
+                              if flush_l2 else
+                              f"inputs larger than L2 (weights, DFlash logits {w.B * w.n * w.V * esl / 1e6:.0f} MB "
+                              f"and target logits {w.B * (w.n + 1) * w.V * esl / 1e6:.0f} MB per step, not flushed)"),
                        "parallelism": f"replicas x{world}"},
             "roofline": roofline,
-            "step_roofline": {"algorithmic_bytes": block_bytes,
-                              "hbm_gbs_equiv": round(block_bytes / step_s / 1e9, 1),
-                              "frac_equiv": round(block_bytes / step_s / 1e9 / peak, 4),
-                              "bytes_read": moved,
-                              "hbm_gbs_read": round(moved / step_s / 1e9, 1),
-                              "note": "algorithmic bytes stream every weight once per position (W_ih included) "
-                                      "plus the DFlash and target logits; bytes_read is what this path reads"},
+            "step_roofline": {"bytes_read": moved,
+                              "gbs_read": round(moved / step_s / 1e9, 1),
+                              "frac_read": round(moved / step_s / 1e9 / peak, 4),
+                              "frac_read_of_nominal_8tbs": round(moved / step_s / 1e9 / NOMINAL_HBM_GBS, 4),
+                              "streaming_model_bytes": survey,
+                              "note": "bytes_read: what this path must read per step (drafted block + verification); "
+                                      "streaming_model_bytes: every head weight streamed once per position "
+                                      "(W_ih included), for comparison only"},
             "kernels": kernels,
             "gpu_launches": launches,
             "e2e": {"value": e2e_val, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
@@ -851,6 +963,8 @@ def run_prior(args):
 
 def main():
     args = parse_args()
+    if args.oracle_single_thread:
+        return oracle_single_thread(args)
     if args.impl == "reference":
         return run_reference(args)
     if args.sweep:

@@ -112,7 +112,11 @@ typedef enum {
  *     l_S = W_M E_M[x_{j-1}].
  *
  * Activations that feed a bf16 product are rounded to bf16 (round to nearest
- * even); accumulation and the recurrent GRU state are float32.
+ * even); accumulation and the recurrent GRU state are float32. Exception: the
+ * transformer head's own products (W_q, W_k, W_v, W_o, W_1, W_2) take their
+ * activations at float32 precision, passed to the tensor cores as the exact
+ * three-term bf16 expansion hi + mid + lo of each value; its feature is
+ * rounded to bf16 for W_vocab like the other heads'.
  */
 typedef struct {
   dels_head_kind kind;

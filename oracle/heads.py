@@ -156,7 +156,11 @@ class XfmrHead(_Head):
         a = RMSNorm(t),  q, k, v = W_q a, W_k a, W_v a  (per head, scale 1/sqrt(d_head))
         u = t_{j-1} + W_o attn(q_{j-1}, k_{0..j-1}, v_{0..j-1})
         y = u + W_2 GELU(W_1 RMSNorm(u));  feature = RMSNorm(y)
-    RMSNorm has eps 1e-6 and unit gain; there are no biases."""
+    RMSNorm has eps 1e-6 and unit gain; there are no biases.
+
+    Precision: the head's own products take their activations unrounded
+    (fp64 here); only the feature, which feeds the bf16 W_vocab product, is
+    rounded to bf16 for bf16 heads (in short_logits)."""
 
     def __init__(self, weights, wdtype, n_heads):
         super().__init__(weights, wdtype)
@@ -175,7 +179,7 @@ class XfmrHead(_Head):
             toks = hist[b]
             j = len(toks)
             t = self.emb_rows("emb", toks) + to_f64(self._raw["pos"][:j])
-            a = self.act(_rmsnorm(t))
+            a = _rmsnorm(t)
             q = a[-1] @ self.w("wq").T
             k = a @ self.w("wk").T
             v = a @ self.w("wv").T
@@ -185,9 +189,9 @@ class XfmrHead(_Head):
                 s = (k[:, sl] @ q[sl]) / math.sqrt(dh)
                 p = np.exp(s - lse(s))
                 o[sl] = p @ v[:, sl]
-            u = t[-1] + self.act(o) @ self.w("wo").T
-            f = _gelu(self.act(_rmsnorm(u)) @ self.w("w1").T)
-            y = u + self.act(f) @ self.w("w2").T
+            u = t[-1] + o @ self.w("wo").T
+            f = _gelu(_rmsnorm(u) @ self.w("w1").T)
+            y = u + f @ self.w("w2").T
             feats[b] = _rmsnorm(y)
         return hist, feats
 

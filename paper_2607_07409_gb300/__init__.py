@@ -20,6 +20,8 @@ __all__ = [
     "DELS_OK", "DELS_F32", "DELS_BF16",
     "DELS_HEAD_GRU", "DELS_HEAD_MLP", "DELS_HEAD_XFMR", "DELS_HEAD_MARKOV",
     "DELS_STATUS_NONFINITE", "DELS_STATUS_TIMEOUT", "DELS_STATUS_BAD_TOKEN",
+    "DELS_ERR_NULL_POINTER", "DELS_ERR_BAD_SHAPE", "DELS_ERR_BAD_DTYPE", "DELS_ERR_ALIGNMENT",
+    "DELS_ERR_WORKSPACE", "DELS_ERR_UNSUPPORTED", "DELS_ERR_CUDA", "DELS_ERR_TOO_LARGE",
     "DelsError", "LocalHead", "lib", "library_path", "exported_symbols",
     "dels_draft_workspace_bytes", "dels_draft_block", "dels_draft_block_weighted",
     "dels_draft_state_bytes", "dels_draft_block_sampled",
@@ -38,7 +40,8 @@ DELS_OK = 0
 DELS_F32, DELS_BF16 = 0, 1
 DELS_HEAD_GRU, DELS_HEAD_MLP, DELS_HEAD_XFMR, DELS_HEAD_MARKOV = 0, 1, 2, 3
 DELS_STATUS_NONFINITE, DELS_STATUS_TIMEOUT, DELS_STATUS_BAD_TOKEN = 1, 2, 4
-DELS_ERR_TOO_LARGE = -8
+(DELS_ERR_NULL_POINTER, DELS_ERR_BAD_SHAPE, DELS_ERR_BAD_DTYPE, DELS_ERR_ALIGNMENT, DELS_ERR_WORKSPACE,
+ DELS_ERR_UNSUPPORTED, DELS_ERR_CUDA, DELS_ERR_TOO_LARGE) = -1, -2, -3, -4, -5, -6, -7, -8
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _LIB_PATH = os.path.join(_HERE, "libdels.so")

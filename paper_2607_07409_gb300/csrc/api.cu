@@ -320,7 +320,45 @@ bool persistent_enabled() {
   return e && e[0] == '1';
 }
 
+// A store product over `rows` activation rows that may exceed one 128-row
+// tile (the transformer head's three-term rows, 3B): ceil(rows / 128)
+// launches over consecutive row blocks, all writing one partial buffer
+// [S][rows][O].
+struct RowBlocks {
+  Gemm g[3];
+  int count = 0;
+};
+
+bool plan_store_rows(RowBlocks& rb, int rows, int O, const uint16_t* X, const void* W, int K, int splits,
+                     float* part, int* status, int sms) {
+  rb.count = 0;
+  for (int r0 = 0; r0 < rows; r0 += kMaxBatchTile) {
+    if (rb.count >= 3) return false;
+    const int m = std::min(kMaxBatchTile, rows - r0);
+    Gemm& g = rb.g[rb.count++];
+    if (!plan_store(g, m, O, X + (size_t)r0 * K, W, K, nullptr, nullptr, 0, 128, splits, 0, ACT_NONE,
+                    part + (size_t)r0 * O, nullptr, 0, status, sms))
+      return false;
+    g.a.out_split_stride = (long long)rows * O;
+  }
+  return rb.count > 0;
+}
+
+cudaError_t run_rows(const RowBlocks& rb, cudaStream_t s) {
+  for (int i = 0; i < rb.count; ++i) {
+    const cudaError_t e = run(rb.g[i], s);
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
 // ------------------------------------------------------------ draft layout
+
+// Transformer head: every activation that feeds one of the head's own bf16
+// products is passed as its exact three-term bf16 expansion (hi + mid + lo,
+// stacked as extra rows of the product), so those products equal float32
+// products; only the feature fed to W_vocab is rounded to bf16.
+constexpr int kXfmrTerms = 3;
 
 // Input-table GRU path: output tile widths of the rank product and of the
 // recurrent product (both split over K).
@@ -402,10 +440,12 @@ DraftLayout draft_layout(const dels_local_head* hd, int B, int n, int V) {
       break;
     }
     case DELS_HEAD_XFMR: {
-      const int D = hd->d_model, F = hd->d_hidden, P = hd->max_pos;
+      // the activations of the head's products are three-term bf16
+      // expansions (kXfmrTerms rows per request, see launch_splitk_finish)
+      const int D = hd->d_model, F = hd->d_hidden, P = hd->max_pos, T = kXfmrTerms;
       L.ex = c.take((size_t)B * D * 2);
       L.t = c.take((size_t)B * D * 4);
-      L.ab = c.take((size_t)B * D * 2);
+      L.ab = c.take((size_t)T * B * D * 2);
       L.q = c.take((size_t)B * D * 4);
       L.kc = c.take((size_t)B * P * D * 4);
       L.vc = c.take((size_t)B * P * D * 4);
@@ -414,11 +454,11 @@ DraftLayout draft_layout(const dels_local_head* hd, int B, int n, int V) {
       L.xs_1 = splits_for(F, 128, D, sms);
       L.xs_2 = splits_for(D, 128, F, sms);
       const int smax = std::max(std::max(L.xs_qkv, L.xs_o), std::max(L.xs_1, L.xs_2));
-      L.xpart = c.take((size_t)smax * B * std::max(D, F) * 4);
-      L.ob = c.take((size_t)B * D * 2);
+      L.xpart = c.take((size_t)smax * T * B * std::max(D, F) * 4);
+      L.ob = c.take((size_t)T * B * D * 2);
       L.uu = c.take((size_t)B * D * 4);
-      L.anb = c.take((size_t)B * D * 2);
-      L.fb = c.take((size_t)B * F * 2);
+      L.anb = c.take((size_t)T * B * D * 2);
+      L.fb = c.take((size_t)T * B * F * 2);
       L.y = c.take((size_t)B * D * 4);
       L.feat = c.take((size_t)B * D * 2);
       break;
@@ -1497,43 +1537,41 @@ int draft_block_impl(const dels_local_head* head, const void* long_logits, dels_
       mb.smp.src_r = feat;
       r = draft_position0(long_logits, logit_dtype, B, n, V, partials, L.partial_ld, status, mb, sms, s);
       if (r != DELS_OK || n == 1) return r;
-      Gemm gq, gk, gvv, go, g1, g2, gv;
-      bool ok = plan_store(gq, B, D, ab, head->w[1], D, nullptr, nullptr, 0, 128, L.xs_qkv, 0, ACT_NONE, xpart,
-                           nullptr, 0, status, sms) &&
-                plan_store(gk, B, D, ab, head->w[2], D, nullptr, nullptr, 0, 128, L.xs_qkv, 0, ACT_NONE, xpart,
-                           nullptr, 0, status, sms) &&
-                plan_store(gvv, B, D, ab, head->w[3], D, nullptr, nullptr, 0, 128, L.xs_qkv, 0, ACT_NONE, xpart,
-                           nullptr, 0, status, sms) &&
-                plan_store(go, B, D, ob, head->w[4], D, nullptr, nullptr, 0, 128, L.xs_o, 0, ACT_NONE, xpart,
-                           nullptr, 0, status, sms) &&
-                plan_store(g1, B, F, anb, head->w[5], D, nullptr, nullptr, 0, 128, L.xs_1, 0, ACT_NONE, xpart,
-                           nullptr, 0, status, sms) &&
-                plan_store(g2, B, D, fb, head->w[6], F, nullptr, nullptr, 0, 128, L.xs_2, 0, ACT_NONE, xpart,
-                           nullptr, 0, status, sms) &&
+      constexpr int T = kXfmrTerms;
+      RowBlocks gq, gk, gvv, go, g1, g2;
+      Gemm gv;
+      bool ok = plan_store_rows(gq, T * B, D, ab, head->w[1], D, L.xs_qkv, xpart, status, sms) &&
+                plan_store_rows(gk, T * B, D, ab, head->w[2], D, L.xs_qkv, xpart, status, sms) &&
+                plan_store_rows(gvv, T * B, D, ab, head->w[3], D, L.xs_qkv, xpart, status, sms) &&
+                plan_store_rows(go, T * B, D, ob, head->w[4], D, L.xs_o, xpart, status, sms) &&
+                plan_store_rows(g1, T * B, F, anb, head->w[5], D, L.xs_1, xpart, status, sms) &&
+                plan_store_rows(g2, T * B, D, fb, head->w[6], F, L.xs_2, xpart, status, sms) &&
                 plan_combine(gv, B, V, n, feat, D, head->w_vocab, long_logits, logit_dtype, log_prior, alpha, beta,
                              partials, L.partial_ld, status, sms);
       if (!ok) return DELS_ERR_CUDA;
+      const int Sq = gq.g[0].a.total_splits, Sk = gk.g[0].a.total_splits, Sv = gvv.g[0].a.total_splits;
+      const int So = go.g[0].a.total_splits, S1 = g1.g[0].a.total_splits, S2 = g2.g[0].a.total_splits;
       const uint16_t* pos = static_cast<const uint16_t*>(head->w[0]);
       for (int j = 1; j < n; ++j) {
         const int p = j - 1;   // position of the newest drafted token x_{j-1}
-        { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_xfmr_embed(ex, pos, p, B, D, t, ab, s)); }
-        { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run(gq, s)); }
-        { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_splitk_finish(xpart, gq.a.total_splits, B, D, nullptr, ACT_NONE, q, D, nullptr, 0, s)); }
-        { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run(gk, s)); }
-        { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_splitk_finish(xpart, gk.a.total_splits, B, D, nullptr, ACT_NONE, kc + (size_t)p * D, P * D,
-                                       nullptr, 0, s)); }
-        { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run(gvv, s)); }
-        { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_splitk_finish(xpart, gvv.a.total_splits, B, D, nullptr, ACT_NONE, vc + (size_t)p * D, P * D,
-                                       nullptr, 0, s)); }
-        { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_attention(q, kc, vc, B, D, NH, p + 1, P, ob, s)); }
-        { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run(go, s)); }
-        { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_splitk_finish(xpart, go.a.total_splits, B, D, t, ACT_NONE, uu, D, nullptr, 0, s)); }
-        { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_rmsnorm_bf16(uu, B, D, D, anb, s)); }
-        { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run(g1, s)); }
-        { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_splitk_finish(xpart, g1.a.total_splits, B, F, nullptr, ACT_GELU, nullptr, 0, fb, F, s)); }
-        { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run(g2, s)); }
-        { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_splitk_finish(xpart, g2.a.total_splits, B, D, uu, ACT_NONE, y, D, nullptr, 0, s)); }
-        { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_rmsnorm_bf16(y, B, D, D, feat, s)); }
+        { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_xfmr_embed(ex, pos, p, B, D, t, ab, s, T)); }
+        { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run_rows(gq, s)); }
+        { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_splitk_finish(xpart, Sq, B, D, nullptr, ACT_NONE, q, D, nullptr, 0, s, T)); }
+        { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run_rows(gk, s)); }
+        { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_splitk_finish(xpart, Sk, B, D, nullptr, ACT_NONE, kc + (size_t)p * D, P * D,
+                                       nullptr, 0, s, T)); }
+        { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run_rows(gvv, s)); }
+        { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_splitk_finish(xpart, Sv, B, D, nullptr, ACT_NONE, vc + (size_t)p * D, P * D,
+                                       nullptr, 0, s, T)); }
+        { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_attention(q, kc, vc, B, D, NH, p + 1, P, ob, s, T)); }
+        { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run_rows(go, s)); }
+        { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_splitk_finish(xpart, So, B, D, t, ACT_NONE, uu, D, nullptr, 0, s, T)); }
+        { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_rmsnorm_bf16(uu, B, D, D, anb, s, T)); }
+        { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run_rows(g1, s)); }
+        { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_splitk_finish(xpart, S1, B, F, nullptr, ACT_GELU, nullptr, 0, fb, F, s, T, T)); }
+        { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run_rows(g2, s)); }
+        { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_splitk_finish(xpart, S2, B, D, uu, ACT_NONE, y, D, nullptr, 0, s, T)); }
+        { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_rmsnorm_bf16(y, B, D, D, feat, s, 1)); }
         gv.a.j = j;
           gv.a.sample = sm.on;
           gv.a.seed = sm.seed;

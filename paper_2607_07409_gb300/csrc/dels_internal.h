@@ -302,13 +302,18 @@ struct GatesTableArgs {
   SampleArgs smp;
 };
 cudaError_t launch_gru_gates_table(const GatesTableArgs& a, cudaStream_t s);
+// bf16 activations of the head products are written as `terms` bf16 terms:
+// 1 = rounded to bf16; 3 = the exact three-term expansion hi + mid + lo in
+// rows [0, B), [B, 2B), [2B, 3B) of a [3B, ld] buffer (a product over the 3B
+// rows then writes partials [S][3B][O], summed back by in_terms = 3).
 cudaError_t launch_splitk_finish(const float* part, int S, int B, int O, const float* residual, int act,
-                                 float* out_f32, int ld_f32, uint16_t* out_bf16, int ld_bf16, cudaStream_t s);
-cudaError_t launch_rmsnorm_bf16(const float* x, int B, int D, int ld, uint16_t* out, cudaStream_t s);
+                                 float* out_f32, int ld_f32, uint16_t* out_bf16, int ld_bf16, cudaStream_t s,
+                                 int in_terms = 1, int out_terms = 1);
+cudaError_t launch_rmsnorm_bf16(const float* x, int B, int D, int ld, uint16_t* out, cudaStream_t s, int terms = 1);
 cudaError_t launch_xfmr_embed(const uint16_t* e_rows, const uint16_t* pos_table, int pos, int B, int D,
-                              float* t_out, uint16_t* a_bf16, cudaStream_t s);
+                              float* t_out, uint16_t* a_bf16, cudaStream_t s, int terms = 1);
 cudaError_t launch_attention(const float* q, const float* kcache, const float* vcache, int B, int D, int nh,
-                             int npos, int cache_ld_pos, uint16_t* o_bf16, cudaStream_t s);
+                             int npos, int cache_ld_pos, uint16_t* o_bf16, cudaStream_t s, int terms = 1);
 cudaError_t launch_gemv_f32(const float* X, int ldx, const float* W, int B, int O, int K, int act, float* Y,
                             int ldy, cudaStream_t s);
 cudaError_t launch_vocab_combine_f32(const float* feat, int K, const float* Wv, const void* longp, int long_f32,

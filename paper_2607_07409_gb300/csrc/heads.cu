@@ -20,6 +20,26 @@ __device__ __forceinline__ float act_f(int act, float x) {
 
 __device__ __forceinline__ float bf16_to_f(uint16_t u) { return __uint_as_float((uint32_t)u << 16); }
 
+// Stores v for a bf16 product. terms = 1: v rounded to bf16 (nearest even)
+// at row b of an [B, ld] buffer. terms = 3: the three-term expansion
+// v = hi + mid + lo, each term the bf16 rounding of what the terms before it
+// left (every difference is exact in float32, and the three terms hold all
+// 24 significand bits of v), at rows b, B + b and 2B + b of a [3B, ld]
+// buffer; a bf16 product over the three rows, accumulated in float32, then
+// equals the product of the float32 activation.
+__device__ __forceinline__ void store_bf16_terms(uint16_t* out, int terms, int B, int b, long long ld, long long o,
+                                                 float v) {
+  const uint16_t hi = f32_to_bf16_rne(v);
+  out[(long long)b * ld + o] = hi;
+  if (terms == 3) {
+    const float r1 = v - bf16_to_f(hi);
+    const uint16_t mid = f32_to_bf16_rne(r1);
+    const float r2 = r1 - bf16_to_f(mid);
+    out[(long long)(B + b) * ld + o] = mid;
+    out[(long long)(2 * B + b) * ld + o] = f32_to_bf16_rne(r2);
+  }
+}
+
 // GRU gates (PyTorch bias-free form; gate rows r, z, n):
 //   gi = sum of the S0 input-product partials, gh = sum of the S1 recurrent ones
 //   r = sigmoid(gi_r + gh_r), z = sigmoid(gi_z + gh_z)
@@ -159,23 +179,28 @@ __global__ void __launch_bounds__(kGatesThreads) k_gru_gates_table(GatesTableArg
   a.h_bf16[e] = f32_to_bf16_rne(hn);
 }
 
-// out[b, o] = act(sum_s part[s, b, o] (+ residual[b, o])); partials and the
-// residual are dense [.., B, O]; outputs have their own row pitch.
+// out[b, o] = act(sum_s sum_t part[s, t*B + b, o] (+ residual[b, o])):
+// partials [S][in_terms*B][O] (in_terms = 3 when the product's input rows were
+// a three-term expansion), the residual dense [B, O]; the f32 output has its
+// own row pitch, the bf16 output is written as out_terms terms (see
+// store_bf16_terms).
 __global__ void k_splitk_finish(const float* __restrict__ part, int S, int B, int O,
                                 const float* __restrict__ residual, int act, float* __restrict__ out_f32, int ld_f32,
-                                uint16_t* __restrict__ out_bf16, int ld_bf16) {
+                                uint16_t* __restrict__ out_bf16, int ld_bf16, int in_terms, int out_terms) {
   if (threadIdx.x == 0) pdl_trigger();
   pdl_wait();
   const long long total = (long long)B * O;
+  const long long split_stride = total * in_terms;
   for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < total;
        e += (long long)gridDim.x * blockDim.x) {
     const int b = (int)(e / O), o = (int)(e % O);
     float acc = 0.f;
-    for (int s = 0; s < S; ++s) acc += part[s * total + e];
+    for (int s = 0; s < S; ++s)
+      for (int t = in_terms - 1; t >= 0; --t) acc += part[s * split_stride + t * total + e];
     if (residual) acc += residual[e];
     acc = act_f(act, acc);
     if (out_f32) out_f32[(long long)b * ld_f32 + o] = acc;
-    if (out_bf16) out_bf16[(long long)b * ld_bf16 + o] = f32_to_bf16_rne(acc);
+    if (out_bf16) store_bf16_terms(out_bf16, out_terms, B, b, ld_bf16, o, acc);
   }
 }
 
@@ -198,8 +223,10 @@ __device__ __forceinline__ float block_sum(float v) {
   return red[0];
 }
 
-// out = bf16( x / sqrt(mean(x^2) + 1e-6) ), one CTA per row
-__global__ void k_rmsnorm_bf16(const float* __restrict__ x, int D, int ld, uint16_t* __restrict__ out) {
+// out = RMSNorm(x) = x / sqrt(mean(x^2) + 1e-6) as `terms` bf16 terms (rows
+// of pitch ld, see store_bf16_terms); one CTA per row.
+__global__ void k_rmsnorm_bf16(const float* __restrict__ x, int D, int ld, uint16_t* __restrict__ out, int terms,
+                               int B) {
   if (threadIdx.x == 0) pdl_trigger();
   pdl_wait();
   const float* row = x + (long long)blockIdx.x * ld;
@@ -207,12 +234,13 @@ __global__ void k_rmsnorm_bf16(const float* __restrict__ x, int D, int ld, uint1
   for (int i = threadIdx.x; i < D; i += blockDim.x) ss += row[i] * row[i];
   ss = block_sum(ss);
   const float inv = rsqrtf(ss / (float)D + 1e-6f);
-  for (int i = threadIdx.x; i < D; i += blockDim.x) out[(long long)blockIdx.x * ld + i] = f32_to_bf16_rne(row[i] * inv);
+  for (int i = threadIdx.x; i < D; i += blockDim.x) store_bf16_terms(out, terms, B, blockIdx.x, ld, i, row[i] * inv);
 }
 
-// t = E[x] + P[pos] (float32), a = bf16(RMSNorm(t)); one CTA per row
+// t = E[x] + P[pos] (float32), a = RMSNorm(t) as `terms` bf16 terms; one CTA
+// per row.
 __global__ void k_xfmr_embed(const uint16_t* __restrict__ e_rows, const uint16_t* __restrict__ pos_table, int pos,
-                             int D, float* __restrict__ t_out, uint16_t* __restrict__ a_bf16) {
+                             int D, float* __restrict__ t_out, uint16_t* __restrict__ a_bf16, int terms, int B) {
   if (threadIdx.x == 0) pdl_trigger();
   pdl_wait();
   const long long off = (long long)blockIdx.x * D;
@@ -224,13 +252,16 @@ __global__ void k_xfmr_embed(const uint16_t* __restrict__ e_rows, const uint16_t
   }
   ss = block_sum(ss);
   const float inv = rsqrtf(ss / (float)D + 1e-6f);
-  for (int i = threadIdx.x; i < D; i += blockDim.x) a_bf16[off + i] = f32_to_bf16_rne(t_out[off + i] * inv);
+  for (int i = threadIdx.x; i < D; i += blockDim.x)
+    store_bf16_terms(a_bf16, terms, B, blockIdx.x, D, i, t_out[off + i] * inv);
 }
 
 // Causal attention of the newest position over positions 0..npos-1 of the
-// block: one CTA per (row, head); o = softmax(q k^T / sqrt(dh)) v, stored bf16.
+// block: one CTA per (row, head); o = softmax(q k^T / sqrt(dh)) v, stored as
+// `terms` bf16 terms.
 __global__ void k_attention(const float* __restrict__ q, const float* __restrict__ kc, const float* __restrict__ vc,
-                            int D, int nh, int npos, int cache_ld_pos, uint16_t* __restrict__ o_bf16) {
+                            int D, int nh, int npos, int cache_ld_pos, uint16_t* __restrict__ o_bf16, int terms,
+                            int B) {
   if (threadIdx.x == 0) pdl_trigger();
   pdl_wait();
   const int b = blockIdx.x / nh, hd = blockIdx.x % nh;
@@ -257,7 +288,7 @@ __global__ void k_attention(const float* __restrict__ q, const float* __restrict
   for (int i = threadIdx.x; i < dh; i += blockDim.x) {
     float o = 0.f;
     for (int p = 0; p < npos; ++p) o += w[p] * vc[((long long)b * cache_ld_pos + p) * D + hd * dh + i];
-    o_bf16[(long long)b * D + hd * dh + i] = f32_to_bf16_rne(o);
+    store_bf16_terms(o_bf16, terms, B, b, D, hd * dh + i, o);
   }
 }
 
@@ -359,23 +390,25 @@ cudaError_t launch_gru_gates_table(const GatesTableArgs& a, cudaStream_t s) {
 }
 
 cudaError_t launch_splitk_finish(const float* part, int S, int B, int O, const float* residual, int act,
-                                 float* out_f32, int ld_f32, uint16_t* out_bf16, int ld_bf16, cudaStream_t s) {
+                                 float* out_f32, int ld_f32, uint16_t* out_bf16, int ld_bf16, cudaStream_t s,
+                                 int in_terms, int out_terms) {
   return launch_pdl(k_splitk_finish, dim3(grid_for((long long)B * O, 256)), dim3(256), 0, s, part, S, B, O, residual,
-                    act, out_f32, ld_f32, out_bf16, ld_bf16);
+                    act, out_f32, ld_f32, out_bf16, ld_bf16, in_terms, out_terms);
 }
 
-cudaError_t launch_rmsnorm_bf16(const float* x, int B, int D, int ld, uint16_t* out, cudaStream_t s) {
-  return launch_pdl(k_rmsnorm_bf16, dim3(B), dim3(256), 0, s, x, D, ld, out);
+cudaError_t launch_rmsnorm_bf16(const float* x, int B, int D, int ld, uint16_t* out, cudaStream_t s, int terms) {
+  return launch_pdl(k_rmsnorm_bf16, dim3(B), dim3(256), 0, s, x, D, ld, out, terms, B);
 }
 
 cudaError_t launch_xfmr_embed(const uint16_t* e_rows, const uint16_t* pos_table, int pos, int B, int D,
-                              float* t_out, uint16_t* a_bf16, cudaStream_t s) {
-  return launch_pdl(k_xfmr_embed, dim3(B), dim3(256), 0, s, e_rows, pos_table, pos, D, t_out, a_bf16);
+                              float* t_out, uint16_t* a_bf16, cudaStream_t s, int terms) {
+  return launch_pdl(k_xfmr_embed, dim3(B), dim3(256), 0, s, e_rows, pos_table, pos, D, t_out, a_bf16, terms, B);
 }
 
 cudaError_t launch_attention(const float* q, const float* kcache, const float* vcache, int B, int D, int nh,
-                             int npos, int cache_ld_pos, uint16_t* o_bf16, cudaStream_t s) {
-  return launch_pdl(k_attention, dim3(B * nh), dim3(128), 0, s, q, kcache, vcache, D, nh, npos, cache_ld_pos, o_bf16);
+                             int npos, int cache_ld_pos, uint16_t* o_bf16, cudaStream_t s, int terms) {
+  return launch_pdl(k_attention, dim3(B * nh), dim3(128), 0, s, q, kcache, vcache, D, nh, npos, cache_ld_pos, o_bf16,
+                    terms, B);
 }
 
 cudaError_t launch_gemv_f32(const float* X, int ldx, const float* W, int B, int O, int K, int act, float* Y, int ldy,

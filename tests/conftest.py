@@ -25,3 +25,19 @@ def pytest_collection_modifyitems(config, items):
     for item in items:
         if "gpu" in item.keywords:
             item.add_marker(skip)
+
+
+def pytest_terminal_summary(terminalreporter, exitstatus, config):
+    """Prints the tie and flip counts of the session's parity checks (the
+    tests record them in parity.PARITY_LOG)."""
+    try:
+        from parity import PARITY_LOG
+    except Exception:  # pragma: no cover
+        return
+    if not PARITY_LOG:
+        return
+    tr = terminalreporter
+    tr.write_sep("-", "parity checks: positions, oracle near-ties (gap < 1e-3), tie-rule flips, max |dlogprob|")
+    for name, info in PARITY_LOG:
+        tr.write_line(f"{name}: " + ", ".join(f"{k}={v:.3g}" if isinstance(v, float) else f"{k}={v}"
+                                               for k, v in info.items()))

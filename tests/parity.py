@@ -21,17 +21,21 @@ TIE_EPS = 1e-3
 LP_TOL_BF16 = 2e-3
 LP_TOL_F32 = 1e-5
 LP_TOL_COMBINE = 1e-5
-# The transformer head at d_model 2560 / FFN 10240 rounds three activations
-# to bf16 in sequence (attention input, FFN input and output, the feature).
-# Both sides round at the same points, but the value being rounded carries
-# the float32 summation error of the device's products (~3e-6 relative for
-# K = 2560), so about 0.2 % of the FFN outputs land on the other side of a
-# bf16 rounding boundary; each such flip moves y by one bf16 step of that
-# activation times W_2, and RMSNorm(y) then flips ~3 % of the feature's bf16
-# codes. Measured at full size: feature flips 3 %, logprob error up to 4.3e-3.
-# The bar for this head is therefore 1e-2 (derived; the fp32 and GRU/MLP
-# heads keep the bars above).
-LP_TOL_XFMR_BF16 = 1e-2
+# Tie-rule flips allowed in one parity check: at most this fraction of the
+# checked positions (and at least 2), so that a device path that lands on
+# near-ties far more often than the oracle's gaps predict still fails.
+MAX_FLIP_FRACTION = 0.01
+
+# Tie and flip counts of every parity check in the session, printed at the end
+# of the run by conftest.pytest_terminal_summary.
+PARITY_LOG = []
+
+
+def record(name, info):
+    """Adds one check's counts to the session summary and returns them."""
+    keep = {k: v for k, v in info.items() if k != "ref"}
+    PARITY_LOG.append((name, keep))
+    return keep
 
 
 def check_rows(tok, lp, gap, ref_tok, ref_lp, ref_gap, lp_tol=LP_TOL_COMBINE, exact_ties=False, fused=None):
@@ -55,7 +59,7 @@ def check_rows(tok, lp, gap, ref_tok, ref_lp, ref_gap, lp_tol=LP_TOL_COMBINE, ex
     fin = same & np.isfinite(ref_gap)
     gerr = np.abs(gap[fin] - ref_gap[fin]).max(initial=0.0)
     assert gerr <= max(2 * lp_tol, 1e-5), f"gap error {gerr}"
-    return dict(ties=int(ties.sum()), flips=int((~same).sum()), lp_err=float(err))
+    return dict(positions=int(tok.size), ties=int(ties.sum()), flips=int((~same).sum()), lp_err=float(err))
 
 
 def check_draft(tok, lp, gap, head, long, prior, alpha, beta, lp_tol, sample=None, request_ids=None):
@@ -81,4 +85,6 @@ def check_draft(tok, lp, gap, head, long, prior, alpha, beta, lp_tol, sample=Non
     if not ties.any():
         # no near-tie anywhere: the device block is the oracle's own block
         assert same.all()
-    return dict(ties=int(ties.sum()), flips=int((~same).sum()), lp_err=err, gap_err=gerr, ref=ref)
+    flips = int((~same).sum())
+    assert flips <= max(2, MAX_FLIP_FRACTION * tok.size), f"{flips} tie-rule flips in {tok.size} positions"
+    return dict(positions=int(tok.size), ties=int(ties.sum()), flips=flips, lp_err=err, gap_err=gerr, ref=ref)

@@ -42,6 +42,14 @@ def test_library_exports_every_declared_symbol(dels):
     assert sorted(dels.exported_symbols()) == declared
 
 
+def test_binding_codes_match_the_header(dels):
+    src = open(os.path.join(ROOT, "include", "dels.h")).read()
+    codes = dict((k, int(v)) for k, v in re.findall(r"\b(DELS_(?:ERR|STATUS)_[A-Z_]+)\s*=\s*(-?\d+)", src))
+    assert len(codes) >= 11
+    for name, value in codes.items():
+        assert getattr(dels, name) == value, name
+
+
 def test_version_and_status_strings(dels):
     assert dels.dels_version() >= 100
     assert dels.dels_status_string(0) == "ok"

@@ -1,10 +1,12 @@
 """Parity at the workloads' full sizes, in the launch configuration the
-benchmark times, on sampled requests.
+benchmark times, over every request of the batch.
 
-Requests are independent (Algorithm 1 touches no state across rows), so the
-oracle run on a subset of the batch is the exact reference for those rows;
-the device always drafts the whole batch. The oracle takes its own prior
-from the counts and re-checks each sampled row in forced-prefix mode.
+The oracle takes its own prior from the counts and re-checks each request in
+forced-prefix mode; the tie-rule flips and near-ties are counted, bounded
+(parity.MAX_FLIP_FRACTION) and listed in the session summary. The
+combine entry point at the 8B shape (1024 rows) is checked on sampled rows
+(rows are independent, so the oracle on a subset is exact for them) and every
+row for range and finiteness.
 """
 import numpy as np
 import pytest
@@ -13,7 +15,7 @@ import torch
 import oracle
 import synth
 import paper_2607_07409_gb300 as dels
-from parity import LP_TOL_BF16, LP_TOL_F32, LP_TOL_XFMR_BF16, check_draft
+from parity import LP_TOL_BF16, LP_TOL_F32, check_draft, record
 
 pytestmark = pytest.mark.gpu
 
@@ -29,7 +31,7 @@ def _oracle_head(w, W):
     return head
 
 
-def _draft_and_verify(w, rows, table=False):
+def _draft_and_verify(w, name, table=False):
     d = synth.make_inputs(w, device=DEV, target=True)
     W = {k[5:]: v for k, v in d.items() if k.startswith("head.")}
     if table:
@@ -48,38 +50,45 @@ def _draft_and_verify(w, rows, table=False):
     torch.cuda.synchronize()
     assert dr.status() == 0 and dels.dels_read_status(vws) == 0
     tok, lp, gap = (t.cpu().numpy() for t in (tok, lp, gap))
-    rows = list(rows)
+    rows = list(range(w.B))
     head = _oracle_head(w, W)
     prior64 = oracle.log_prior(d["counts"])
-    tol = LP_TOL_F32 if w.head.wdtype == "f32" else (LP_TOL_XFMR_BF16 if w.head.kind == "xfmr" else LP_TOL_BF16)
+    tol = LP_TOL_F32 if w.head.wdtype == "f32" else LP_TOL_BF16
     info = check_draft(tok[rows], lp[rows], gap[rows], head, d["long"][rows].cpu(), prior64, w.alpha, w.beta, tol)
     # verification of the same rows: bit-exact accept length, bonus and target argmax
     ref_acc, ref_bonus, ref_t = oracle.verify_greedy(tok[rows], d["target"][rows].cpu())
     np.testing.assert_array_equal(acc.cpu().numpy()[rows], ref_acc)
     np.testing.assert_array_equal(bonus.cpu().numpy()[rows], ref_bonus)
     np.testing.assert_array_equal(targ.cpu().numpy()[rows], ref_t)
-    return info
+    return record(name, info)
 
 
 @pytest.mark.parametrize("table", [True, False])
 def test_qwen3_8b_batched_full_size(table):
     w = synth.WORKLOADS["qwen3_8b_batched"]
-    print(_draft_and_verify(w, [0, 21, 63], table=table))
+    print(_draft_and_verify(w, f"qwen3_8b_batched full size, input table {table}", table=table))
 
 
 def test_qwen3_8b_batched_full_size_stress():
     w = synth.stress(synth.WORKLOADS["qwen3_8b_batched"])
-    print(_draft_and_verify(w, [5, 40], table=True))
+    print(_draft_and_verify(w, "qwen3_8b_batched full size, stress weights", table=True))
 
 
 def test_qwen3_0p6b_full_size():
     w = synth.WORKLOADS["qwen3_0p6b"]
-    print(_draft_and_verify(w, [0]))
+    print(_draft_and_verify(w, "qwen3_0p6b full size"))
 
 
 def test_qwen3_4b_full_size():
     w = synth.WORKLOADS["qwen3_4b"]
-    print(_draft_and_verify(w, [0, 7]))
+    print(_draft_and_verify(w, "qwen3_4b full size"))
+
+
+def test_qwen3_4b_full_size_stress():
+    """The transformer head with fan-in-scaled weights, where the short logits
+    are O(1) and move tokens: held to the same 2e-3 logprob bar."""
+    w = synth.stress(synth.WORKLOADS["qwen3_4b"])
+    print(_draft_and_verify(w, "qwen3_4b full size, stress weights"))
 
 
 def test_qwen3_8b_batched_full_size_temperature_one():
@@ -88,7 +97,7 @@ def test_qwen3_8b_batched_full_size_temperature_one():
     by speculative sampling, against the oracle with the rows' own variates."""
     w = synth.stress(synth.WORKLOADS["qwen3_8b_batched"])
     seed, step = 77, 5
-    rows = [2, 45]
+    rows = list(range(w.B))
     d = synth.make_inputs(w, device=DEV, target=True)
     W = {k[5:]: v for k, v in d.items() if k.startswith("head.")}
     W["input_table"] = dels.gru_input_table(w.head, W, w.V)
@@ -117,8 +126,14 @@ def test_qwen3_8b_batched_full_size_temperature_one():
     close = vinfo["margin"] < 8 * LP_TOL_BF16
     assert np.all((acc == r_acc) | close), (acc, r_acc, vinfo["margin"])
     ok = (acc == r_acc) & ~close
-    assert np.all((bonus == r_bonus) | ~ok | (vinfo["bonus_gap"] < 0.05)), (bonus, r_bonus, vinfo["bonus_gap"])
-    print({k: v for k, v in info.items() if k != "ref"}, "accept", acc.tolist(), r_acc.tolist())
+    near_bonus = vinfo["bonus_gap"] < 0.05
+    assert np.all((bonus == r_bonus) | ~ok | near_bonus), (bonus, r_bonus, vinfo["bonus_gap"])
+    # the exemptions stay a small share of the batch
+    assert close.sum() <= max(4, 0.15 * len(rows)), f"{close.sum()} rows with a near-threshold acceptance test"
+    assert near_bonus.sum() <= max(4, 0.15 * len(rows)), f"{near_bonus.sum()} rows with a near-tie bonus draw"
+    info = dict(info, accept_exempt=int(close.sum()), accept_differs=int((acc != r_acc).sum()),
+                bonus_exempt=int((near_bonus & ok).sum()), bonus_differs=int((ok & (bonus != r_bonus)).sum()))
+    print(record("qwen3_8b_batched full size, temperature 1", info))
 
 
 @pytest.mark.parametrize("dtype", ["bf16", "f32"])
@@ -151,5 +166,6 @@ def test_combine_full_size_8b_shape(dtype):
     fused = oracle.fuse(oracle.to_f64(d["long"][rows].cpu()), oracle.to_f64(d["short"][rows].cpu()),
                         prior.astype(np.float64), a, b)
     from parity import check_rows
-    print(check_rows(tok.cpu().numpy()[rows], lp.cpu().numpy()[rows], gap.cpu().numpy()[rows], rt, rl, rg,
-                     fused=fused))
+    print(record(f"combine 1024 x 151936 {dtype}, sampled rows",
+                 check_rows(tok.cpu().numpy()[rows], lp.cpu().numpy()[rows], gap.cpu().numpy()[rows], rt, rl, rg,
+                            fused=fused)))

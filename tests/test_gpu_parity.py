@@ -12,7 +12,7 @@ import torch
 import oracle
 import synth
 import paper_2607_07409_gb300 as dels
-from parity import LP_TOL_BF16, LP_TOL_F32, check_draft, check_rows
+from parity import LP_TOL_BF16, LP_TOL_F32, check_draft, check_rows, record
 
 pytestmark = pytest.mark.gpu
 
@@ -197,6 +197,10 @@ SMALL = {
     "xfmr": synth.with_sizes(synth.WORKLOADS["qwen3_4b"], B=2, n=5, V=1536,
                              head_d_model=256, head_d_hidden=512, head_d_rank=256, head_n_heads=4,
                              head_max_pos=8),
+    # 3B = 144 three-term rows: the head's products run as two row blocks (128 + 16)
+    "xfmr_b48": synth.with_sizes(synth.WORKLOADS["qwen3_4b"], B=48, n=4, V=1024,
+                                 head_d_model=128, head_d_hidden=256, head_d_rank=128, head_n_heads=4,
+                                 head_max_pos=4),
     "markov": synth.Workload("markov", B=4, n=6, V=2048, logit_dtype="bf16",
                              head=synth.HeadSpec("markov", "bf16", 0, 0, 128), weight=0.5, seed=7),
     "markov_f32": synth.Workload("markov_f32", B=2, n=5, V=1000, logit_dtype="f32",
@@ -219,7 +223,7 @@ def test_draft_small_matches_oracle(name, stress):
     tok, lp, gap, W, prior = _draft(w, d)
     tol = LP_TOL_F32 if w.head.wdtype == "f32" else LP_TOL_BF16
     info = check_draft(tok, lp, gap, _oracle_head(w, W), d["long"].cpu(), prior, w.alpha, w.beta, tol)
-    print(name, stress, info)
+    print(name, stress, record(f"draft {name}, stress {stress}", info))
 
 
 @pytest.mark.parametrize("stress", [False, True])

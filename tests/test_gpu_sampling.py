@@ -13,7 +13,7 @@ import torch
 import oracle
 import synth
 import paper_2607_07409_gb300 as dels
-from parity import LP_TOL_BF16, LP_TOL_F32, LP_TOL_XFMR_BF16, check_draft
+from parity import LP_TOL_BF16, LP_TOL_F32, check_draft, record
 from test_gpu_parity import DEV, SMALL, _oracle_head, _with_table, _learned_weights
 
 pytestmark = pytest.mark.gpu
@@ -39,13 +39,13 @@ def _sampled(name, seed=17, step=3, weights="learned"):
 def test_sampled_draft_matches_oracle(name):
     seed, step = 17, 3
     w, d, W, a, b, tok, lp, gap, state = _sampled(name, seed, step)
-    tol = LP_TOL_F32 if w.head.wdtype == "f32" else (LP_TOL_XFMR_BF16 if name == "xfmr" else LP_TOL_BF16)
+    tol = LP_TOL_F32 if w.head.wdtype == "f32" else LP_TOL_BF16
     info = check_draft(tok, lp, gap, _oracle_head(w, W), d["long"].cpu(), oracle.log_prior(d["counts"]),
                        np.array(a), np.array(b), tol, sample=(seed, step))
     # the LSE of every fused row, kept for the verification
     lse = state[: w.B * w.n * 4].view(torch.float32).view(w.B, w.n).cpu().numpy()
     np.testing.assert_allclose(lse, info["ref"].lse, rtol=0, atol=tol * 4)
-    print(name, {k: v for k, v in info.items() if k != "ref"})
+    print(name, record(f"sampled draft {name}", info))
 
 
 def test_sampled_draft_depends_on_seed_and_step_only():
@@ -126,7 +126,7 @@ def test_sampled_verify_matches_oracle(name):
     w, d, W, a, b, tok, lp, gap, state = _sampled(name, seed, step)
     target = synth.make_target_logits(w, d["long"], device=DEV)
     acc, bonus, bgap = _verify(w, d, W, a, b, tok, lp, state, target, seed, step)
-    tol = LP_TOL_F32 if w.head.wdtype == "f32" else (LP_TOL_XFMR_BF16 if name == "xfmr" else LP_TOL_BF16)
+    tol = LP_TOL_F32 if w.head.wdtype == "f32" else LP_TOL_BF16
     info = _check_verify(w, d, W, a, b, tok, acc, bonus, bgap, target, seed, step, tol)
     print(name, info)
     assert np.all((acc >= 0) & (acc <= w.n)) and np.all((bonus >= 0) & (bonus < w.V))

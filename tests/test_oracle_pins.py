@@ -368,6 +368,37 @@ def test_xfmr_head_matches_torch_causal_block():
             np.testing.assert_allclose(feat[b], ref.numpy(), rtol=1e-11, atol=1e-13)
 
 
+def test_xfmr_head_bf16_contract_rounds_only_the_feature():
+    """bf16 transformer head: the head's own products take unrounded
+    activations (the same features as the torch float64 block above), and only
+    the feature fed to W_vocab is rounded to bf16 (RNE)."""
+    w = synth.with_sizes(synth.stress(synth.WORKLOADS["qwen3_4b"]), V=40, B=2, n=6,
+                         head_d_model=16, head_d_hidden=32, head_d_rank=16, head_n_heads=4, head_max_pos=6)
+    d = synth.make_inputs(w, target=False)
+    W = {k[5:]: v for k, v in d.items() if k.startswith("head.")}
+    assert W["wq"].dtype == torch.bfloat16
+    Wd = {k: v.double() for k, v in W.items()}
+    head = oracle.XfmrHead(W, "bf16", 4)
+    st = head.init(2)
+    F = torch.nn.functional
+    seq = [[3, 39, 3, 0, 17], [8, 8, 8, 8, 8]]
+    for j in range(5):
+        st, feat = head.step(st, np.array([seq[0][j], seq[1][j]]))
+        for b in range(2):
+            toks = torch.as_tensor(seq[b][: j + 1])
+            t = Wd["emb"][toks] + Wd["pos"][: j + 1]
+            a = F.rms_norm(t, (16,), eps=1e-6)
+            q, k, v = (a @ Wd[n].T for n in ("wq", "wk", "wv"))
+            sh = lambda x: x.view(-1, 4, 4).transpose(0, 1)
+            o = F.scaled_dot_product_attention(sh(q), sh(k), sh(v), is_causal=True).transpose(0, 1).reshape(-1, 16)
+            u = t + o @ Wd["wo"].T
+            y = u + F.gelu(F.rms_norm(u, (16,), eps=1e-6) @ Wd["w1"].T) @ Wd["w2"].T
+            np.testing.assert_allclose(feat[b], F.rms_norm(y, (16,), eps=1e-6)[-1].numpy(), rtol=1e-11, atol=1e-13)
+        S = head.short_logits(feat)
+        r = torch.from_numpy(feat).float().bfloat16().double()
+        np.testing.assert_allclose(S, (r @ Wd["w_vocab"].T).numpy(), rtol=1e-12, atol=1e-13)
+
+
 def test_markov_head_is_embedding_times_vocab_matrix():
     w = synth.Workload("m", B=3, n=4, V=30, logit_dtype="f32",
                        head=synth.HeadSpec("markov", "f32", 0, 0, 6), weight=0.5, weight_std=None,
