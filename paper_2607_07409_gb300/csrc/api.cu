@@ -286,6 +286,14 @@ bool plan_combine(Gemm& g, int B, int V, int n, const void* X, int K, const void
   const int rpc = (B + 31) / 32 * 32;
   a.a_box_rows = rpc;
   a.a_copies = (rpc == 32) ? 4 : (rpc == 64 ? 2 : 1);
+  if (!a.a_resident && B <= 32) {
+    // Activations staged with every K chunk: load only the live rows, once.
+    // The copies (and a 32-row box for a handful of requests) would make
+    // every CTA fetch the same few L2 lines four times per stage, while a
+    // long K leaves the epilogue ample time for the rows of one quadrant.
+    a.a_box_rows = (B + 7) / 8 * 8;
+    a.a_copies = 1;
+  }
   if (!map_x(&g.mA0, X, B, K, a.a_box_rows) || !map_w(&g.mB0, Wv, V, K, n_tile)) return false;
   if (!encode_tmap_3d(&g.mL, longp, a.long_f32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16,
                       es, (uint64_t)V, (uint64_t)n, (uint64_t)B, (uint64_t)V * es, (uint64_t)n * V * es,
