@@ -195,8 +195,20 @@ __global__ void k_splitk_finish(const float* __restrict__ part, int S, int B, in
        e += (long long)gridDim.x * blockDim.x) {
     const int b = (int)(e / O), o = (int)(e % O);
     float acc = 0.f;
-    for (int s = 0; s < S; ++s)
-      for (int t = in_terms - 1; t >= 0; --t) acc += part[s * split_stride + t * total + e];
+    if (in_terms == 1) {
+      // eight partial loads in flight before they are added in split order
+      for (int s0 = 0; s0 < S; s0 += 8) {
+        float v[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) v[k] = s0 + k < S ? part[(s0 + k) * split_stride + e] : 0.f;
+#pragma unroll
+        for (int k = 0; k < 8; ++k)
+          if (s0 + k < S) acc += v[k];
+      }
+    } else {
+      for (int s = 0; s < S; ++s)
+        for (int t = in_terms - 1; t >= 0; --t) acc += part[s * split_stride + t * total + e];
+    }
     if (residual) acc += residual[e];
     acc = act_f(act, acc);
     if (out_f32) out_f32[(long long)b * ld_f32 + o] = acc;
