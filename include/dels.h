@@ -270,14 +270,15 @@ int dels_combine_argmax_noalloc(const void* long_logits, const void* short_logit
 /* ---- temperature 1 (Algorithm 1 with Decode = a draw from the softmax) --- */
 
 /*
- * Random numbers. Every uniform is drawn from Philox4x64-10 (Salmon et al.,
+ * Random numbers. Every uniform is drawn from Philox4x32-10 (Salmon et al.,
  * "Parallel random numbers: as easy as 1, 2, 3", SC 2011) under the key
- * (seed, step) with the counter (v / 8, j, b, stream) for vocabulary index v,
- * block position j, request b and stream (0 drafting, 1 acceptance tests, 2
- * residual / bonus draws); the 4 output words give 8 32-bit halves, high half
- * first, for v = 8 (v / 8) .. + 7, and a half h gives u = (floor(h / 2^9) +
- * 1/2) / 2^23. Draws use the Gumbel-max rule: x = argmax_v (l_v + g_v),
- * g = -log(-log u). Give each block its own `step`.
+ * (seed mod 2^32, seed div 2^32) with the counter (v / 4, step, b + 2^16 j +
+ * 2^24 stream, 0) for vocabulary index v, block position j, request b and
+ * stream (0 drafting, 1 acceptance tests, 2 residual / bonus draws); output
+ * word v mod 4 (a 32-bit value h) gives u = (floor(h / 2^9) + 1/2) / 2^23.
+ * Draws use the Gumbel-max rule: x = argmax_v (l_v + g_v), g = -log(-log u).
+ * Give each block its own `step`; step >= 2^32 or B >= 2^16 returns
+ * DELS_ERR_BAD_SHAPE.
  *
  * dels_draft_block_sampled: as dels_draft_block_weighted, but every position
  * is drawn: x_0 ~ softmax(l_L^(0)), x_j ~ softmax(l^(j)).

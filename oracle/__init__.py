@@ -51,7 +51,7 @@ from .core import (  # noqa: F401
     greedy_decode,
     combine_argmax,
     verify_greedy,
-    philox4x64_10,
+    philox4x32_10,
     uniforms,
     gumbel,
     sample_decode,

@@ -144,46 +144,35 @@ def combine_argmax(long, short, prior, alpha: float, beta: float):
 # ----------------------------------------------------------------------------
 # temperature-1 Decode (Algorithm 1, x_j ~ softmax(l^(j))) and its random numbers
 # ----------------------------------------------------------------------------
-# The random numbers come from Philox4x64-10, the counter-based generator of
+# The random numbers come from Philox4x32-10, the counter-based generator of
 # Salmon, Moraes, Dror and Shaw ("Parallel random numbers: as easy as 1, 2, 3",
-# SC 2011): ten rounds of two 64x64 -> 128-bit products on a 4-word counter
-# under a 2-word key that is bumped by two Weyl constants between rounds.
+# SC 2011): ten rounds on a counter of four 32-bit words under a key of two
+# 32-bit words. A round multiplies words 0 and 2 by two fixed constants
+# (32 x 32 -> 64-bit products), exchanges the words and folds the key into
+# the high halves; the key is bumped by two Weyl constants between rounds.
 # The drafting and verification kernels implement the same definition, so
 # both sides draw identical uniforms from (seed, step, request, position,
 # stream, vocabulary index).
 
-PHILOX_M0, PHILOX_M1 = 0xD2E7470EE14C6C93, 0xCA5A826395121157
-PHILOX_W0, PHILOX_W1 = 0x9E3779B97F4A7C15, 0xBB67AE8584CAA73B
+PHILOX_M0, PHILOX_M1 = 0xD2511F53, 0xCD9E8D57
+PHILOX_W0, PHILOX_W1 = 0x9E3779B9, 0xBB67AE85
 STREAM_DRAFT, STREAM_ACCEPT, STREAM_RESIDUAL = 0, 1, 2
 _M32 = np.uint64(0xFFFFFFFF)
 
 
-def _mulhilo64(a, m: int):
-    """(high, low) 64-bit halves of the 128-bit products a * m, a uint64 array."""
-    a = np.asarray(a, dtype=np.uint64)
-    m = np.uint64(m)
+def philox4x32_10(c0, c1, c2, c3, k0: int, k1: int):
+    """Philox4x32-10 of the counter words (c0, c1, c2, c3) (integer arrays
+    below 2^32, broadcast) under the key (k0, k1); returns the four output
+    words as uint64 arrays holding 32-bit values."""
+    x = [np.asarray(c, dtype=np.uint64) & _M32 for c in np.broadcast_arrays(c0, c1, c2, c3)]
+    k0, k1 = np.uint64(k0 & 0xFFFFFFFF), np.uint64(k1 & 0xFFFFFFFF)
     s32 = np.uint64(32)
-    a_lo, a_hi = a & _M32, a >> s32
-    m_lo, m_hi = m & _M32, m >> s32
-    p0, p1, p2, p3 = a_lo * m_lo, a_lo * m_hi, a_hi * m_lo, a_hi * m_hi
-    mid = (p0 >> s32) + (p1 & _M32) + (p2 & _M32)
-    hi = p3 + (p1 >> s32) + (p2 >> s32) + (mid >> s32)
-    with np.errstate(over="ignore"):
-        lo = a * m
-    return hi, lo
-
-
-def philox4x64_10(c0, c1, c2, c3, k0: int, k1: int):
-    """Philox4x64-10 of counters (c0, c1, c2, c3) (uint64 arrays, broadcast) under key (k0, k1)."""
-    x = [np.asarray(c, dtype=np.uint64) for c in np.broadcast_arrays(c0, c1, c2, c3)]
-    k0, k1 = np.uint64(k0 & 0xFFFFFFFFFFFFFFFF), np.uint64(k1 & 0xFFFFFFFFFFFFFFFF)
-    with np.errstate(over="ignore"):
-        for _ in range(10):
-            hi0, lo0 = _mulhilo64(x[0], PHILOX_M0)
-            hi1, lo1 = _mulhilo64(x[2], PHILOX_M1)
-            x = [hi1 ^ x[1] ^ k0, lo1, hi0 ^ x[3] ^ k1, lo0]
-            k0 = k0 + np.uint64(PHILOX_W0)
-            k1 = k1 + np.uint64(PHILOX_W1)
+    for _ in range(10):
+        p0 = x[0] * np.uint64(PHILOX_M0)          # < 2^64: exact in uint64
+        p1 = x[2] * np.uint64(PHILOX_M1)
+        x = [(p1 >> s32) ^ x[1] ^ k0, p1 & _M32, (p0 >> s32) ^ x[3] ^ k1, p0 & _M32]
+        k0 = (k0 + np.uint64(PHILOX_W0)) & _M32
+        k1 = (k1 + np.uint64(PHILOX_W1)) & _M32
     return x
 
 
@@ -191,15 +180,19 @@ def uniforms(seed: int, step: int, b: int, j: int, stream: int, v):
     """The uniform variates U(0, 1) of vocabulary indices v (array) for request
     b, position j and stream (0 drafting, 1 acceptance, 2 residual/bonus).
 
-    Counter (v // 8, j, b, stream), key (seed, step); the 4 output words give 8
-    32-bit halves (high half first), and a half h gives u = (floor(h / 2^9) +
-    1/2) / 2^23, an exact float32 in [2^-24, 1 - 2^-24].
+    Key (seed mod 2^32, seed div 2^32); counter (v div 4, step, b + 2^16 j +
+    2^24 stream, 0); output word v mod 4 gives u = (floor(w / 2^9) + 1/2) /
+    2^23, an exact float32 in [2^-24, 1 - 2^-24]. Needs 0 <= step < 2^32,
+    0 <= b < 2^16 and 0 <= j < 2^8.
     """
+    if not (0 <= step < 2 ** 32 and 0 <= b < 2 ** 16 and 0 <= j < 2 ** 8 and 0 <= stream < 4):
+        raise ValueError("uniforms: step, request or position out of range")
     v = np.asarray(v, dtype=np.int64)
-    words = philox4x64_10((v >> 3).astype(np.uint64), np.uint64(j), np.uint64(b), np.uint64(stream), seed, step)
-    w = np.select([(v & 7) >> 1 == k for k in range(4)], words)
-    half = np.where((v & 1) == 0, w >> np.uint64(32), w & _M32)
-    return ((half >> np.uint64(9)).astype(np.float64) + 0.5) / float(1 << 23)
+    seed &= 0xFFFFFFFFFFFFFFFF
+    words = philox4x32_10((v >> 2).astype(np.uint64), np.uint64(step), np.uint64(b + (j << 16) + (stream << 24)),
+                          np.uint64(0), seed & 0xFFFFFFFF, seed >> 32)
+    w = np.select([(v & 3) == k for k in range(4)], words)
+    return ((w >> np.uint64(9)).astype(np.float64) + 0.5) / float(1 << 23)
 
 
 def gumbel(u):

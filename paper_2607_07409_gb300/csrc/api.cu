@@ -919,19 +919,26 @@ size_t dels_combine_workspace_bytes(int rows, int V, dels_dtype dtype) {
   if (rows < 0 || V < 1 || (dtype != DELS_F32 && dtype != DELS_BF16)) return 0;
   const int sms = device_sm_count();
   if (sms <= 0) return 0;
-  const int es = dtype == DELS_F32 ? 4 : 2;
-  const bool vec = (V % (16 / es)) == 0;
-  RowsPlan p = plan_rows(rows, V, 2 * es, sms, vec, 1 << 20, true);
-  const size_t groups = ((size_t)rows + p.rows_per_cta - 1) / p.rows_per_cta;
-  size_t off = kHeaderBytes;
-  off = round_up(off + groups * 4, 256);
-  off = round_up(off + (size_t)rows * p.nchunks * 16, 256);
-  return off;
+  return combine_layout(rows, V, dtype, sms).total;
 }
 
 }  // extern "C"
 
 namespace dels {
+// Workspace of dels_combine_argmax: status header, one ticket per row group,
+// then the partial records ([rows][partial_ld], 16 bytes each).
+CombineLayout combine_layout(int rows, int V, dels_dtype dtype, int sms) {
+  CombineLayout L{};
+  const int es = dtype == DELS_F32 ? 4 : 2;
+  L.vec = (V % 8) == 0;
+  L.p = plan_rows(rows, V, 2 * es, sms, L.vec, 1 << 20, true, rows_slots_per_sm(false, dtype));
+  const size_t groups = ((size_t)rows + L.p.rows_per_cta - 1) / L.p.rows_per_cta;
+  L.tickets_off = kHeaderBytes;
+  L.partials_off = round_up(L.tickets_off + groups * 4, 256);
+  L.total = round_up(L.partials_off + (size_t)rows * L.p.nchunks * 16, 256);
+  return L;
+}
+
 int combine_check_inputs(const void* long_logits, const void* short_logits, const float* log_prior,
                          const int32_t* out_token) {
   if (!long_logits || !out_token) return DELS_ERR_NULL_POINTER;
@@ -957,10 +964,7 @@ int dels_combine_argmax(const void* long_logits, const void* short_logits, dels_
   if (need == 0) return DELS_ERR_CUDA;
   if (workspace_bytes < need) return DELS_ERR_WORKSPACE;
   const int sms = device_sm_count();
-  const int es = dtype == DELS_F32 ? 4 : 2;
-  const bool vec = (V % (16 / es)) == 0;
-  RowsPlan p = plan_rows(rows, V, 2 * es, sms, vec, 1 << 20, true);
-  const size_t groups = ((size_t)rows + p.rows_per_cta - 1) / p.rows_per_cta;
+  const CombineLayout L = combine_layout(rows, V, dtype, sms);
   RowsArgs a{};
   a.longp = long_logits;
   a.shortp = short_logits;
@@ -971,45 +975,58 @@ int dels_combine_argmax(const void* long_logits, const void* short_logits, dels_
   a.V = V;
   a.ld_long = V;
   a.ld_short = V;
-  a.chunk_cols = p.chunk_cols;
-  a.nchunks = p.nchunks;
-  a.rows_per_cta = p.rows_per_cta;
-  a.counters = at<int>(workspace, kHeaderBytes);
-  a.partials = at<void>(workspace, round_up(kHeaderBytes + groups * 4, 256));
-  a.partial_ld = p.nchunks;
+  a.chunk_cols = L.p.chunk_cols;
+  a.nchunks = L.p.nchunks;
+  a.rows_per_cta = L.p.rows_per_cta;
+  a.counters = at<int>(workspace, L.tickets_off);
+  a.partials = at<void>(workspace, L.partials_off);
+  a.partial_ld = L.p.nchunks;
   a.out_token = out_token;
   a.out_lp = out_logprob;
   a.out_gap = out_top2_gap;
   a.status = at<int>(workspace, 0);
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   PROF(DELS_KCLASS_COMBINE);
-  if (launch_combine_rows(a, dtype, vec, true, s) != cudaSuccess) return DELS_ERR_CUDA;
+  if (launch_combine_rows(a, dtype, L.vec, true, s) != cudaSuccess) return DELS_ERR_CUDA;
   return DELS_OK;
 }
 
 // ------------------------------------------------------------------ verify
 
+// Workspace of dels_verify_block: status header, per-request tickets, then
+// the partial records ([B (n + 1)][nchunks]).
+struct VerifyLayout {
+  bool vec;
+  RowsPlan p;
+  size_t req_tk, partials, total;
+};
+
+VerifyLayout verify_layout(int B, int n, int V, dels_dtype dtype, int sms) {
+  VerifyLayout L{};
+  const int es = dtype == DELS_F32 ? 4 : 2;
+  const size_t rows = (size_t)B * (n + 1);
+  L.vec = (V % 8) == 0;
+  L.p = plan_rows((int)std::min<size_t>(rows, INT32_MAX), V, es, sms, L.vec, 1 << 20, false,
+                  rows_slots_per_sm(true, dtype));
+  L.req_tk = kHeaderBytes;
+  L.partials = round_up(L.req_tk + (size_t)B * 4, 256);
+  L.total = round_up(L.partials + rows * L.p.nchunks * 16, 256);
+  return L;
+}
+
 size_t dels_verify_workspace_bytes(int B, int n, int V, dels_dtype dtype) {
-  if (B < 0 || n < 1 || n > 1024 || V < 1 || (dtype != DELS_F32 && dtype != DELS_BF16)) return 0;
+  if (B < 0 || n < 1 || n > kMaxVerifyBlock || V < 1 || (dtype != DELS_F32 && dtype != DELS_BF16)) return 0;
+  if ((long long)B * (n + 1) > INT32_MAX) return 0;
   const int sms = device_sm_count();
   if (sms <= 0) return 0;
-  const int es = dtype == DELS_F32 ? 4 : 2;
-  const bool vec = (V % (16 / es)) == 0;
-  const size_t rows = (size_t)B * (n + 1);
-  RowsPlan p = plan_rows((int)std::min<size_t>(rows, INT32_MAX), V, es, sms, vec, 1 << 20);
-  size_t off = kHeaderBytes;
-  off = round_up(off + rows * 4, 256);        // per-row tickets
-  off = round_up(off + (size_t)B * 4, 256);   // per-request tickets
-  off = round_up(off + rows * 4, 256);        // target argmax scratch
-  off = round_up(off + rows * p.nchunks * 16, 256);
-  return off;
+  return verify_layout(B, n, V, dtype, sms).total;
 }
 
 int dels_verify_block(const int32_t* draft_tokens, const void* target_logits, dels_dtype dtype, int B, int n, int V,
                       int32_t* out_accept_len, int32_t* out_bonus, int32_t* out_target_argmax, void* workspace,
                       size_t workspace_bytes, dels_stream_t stream) {
   if (dtype != DELS_F32 && dtype != DELS_BF16) return DELS_ERR_BAD_DTYPE;
-  if (B < 0 || n < 1 || n > 1024 || V < 1) return DELS_ERR_BAD_SHAPE;
+  if (B < 0 || n < 1 || n > kMaxVerifyBlock || V < 1) return DELS_ERR_BAD_SHAPE;
   if ((long long)B * (n + 1) > INT32_MAX) return DELS_ERR_BAD_SHAPE;
   if (!workspace) return DELS_ERR_WORKSPACE;
   if (B == 0) return DELS_OK;
@@ -1019,27 +1036,19 @@ int dels_verify_block(const int32_t* draft_tokens, const void* target_logits, de
   if (need == 0) return DELS_ERR_CUDA;
   if (workspace_bytes < need) return DELS_ERR_WORKSPACE;
   const int sms = device_sm_count();
-  const int es = dtype == DELS_F32 ? 4 : 2;
-  const bool vec = (V % (16 / es)) == 0;
   const size_t rows = (size_t)B * (n + 1);
-  RowsPlan p = plan_rows((int)rows, V, es, sms, vec, 1 << 20);
+  const VerifyLayout L = verify_layout(B, n, V, dtype, sms);
   RowsArgs a{};
   a.longp = target_logits;
   a.rows = (int)rows;
   a.V = V;
   a.ld_long = V;
-  a.chunk_cols = p.chunk_cols;
-  a.nchunks = p.nchunks;
+  a.chunk_cols = L.p.chunk_cols;
+  a.nchunks = L.p.nchunks;
   a.rows_per_cta = 1;
-  size_t off = kHeaderBytes;
-  a.counters = at<int>(workspace, off);
-  off = round_up(off + rows * 4, 256);
-  a.counters_b = at<int>(workspace, off);
-  off = round_up(off + (size_t)B * 4, 256);
-  a.targ_scratch = at<int32_t>(workspace, off);
-  off = round_up(off + rows * 4, 256);
-  a.partials = at<void>(workspace, off);
-  a.partial_ld = p.nchunks;
+  a.counters_b = at<int>(workspace, L.req_tk);
+  a.partials = at<void>(workspace, L.partials);
+  a.partial_ld = L.p.nchunks;
   a.out_token = out_target_argmax;
   a.draft = draft_tokens;
   a.n = n;
@@ -1048,7 +1057,7 @@ int dels_verify_block(const int32_t* draft_tokens, const void* target_logits, de
   a.status = at<int>(workspace, 0);
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   PROF(DELS_KCLASS_VERIFY);
-  if (launch_verify_rows(a, dtype, vec, s) != cudaSuccess) return DELS_ERR_CUDA;
+  if (launch_verify_rows(a, dtype, L.vec, s) != cudaSuccess) return DELS_ERR_CUDA;
   return DELS_OK;
 }
 
@@ -1667,6 +1676,7 @@ int dels_draft_block_sampled(const dels_local_head* head, const void* long_logit
                              size_t workspace_bytes, dels_stream_t stream) {
   if (!head || !alpha || !beta || !out_logprob) return DELS_ERR_NULL_POINTER;
   if (n < 1 || n > 32 || B < 0) return DELS_ERR_BAD_SHAPE;
+  if (!sample_counter_ok(B, step)) return DELS_ERR_BAD_SHAPE;
   for (int j = 0; j < n; ++j)
     if (!std::isfinite(alpha[j]) || !std::isfinite(beta[j])) return DELS_ERR_BAD_SHAPE;
   const size_t es = head->wdtype == DELS_BF16 ? 2 : 4;
@@ -1696,7 +1706,7 @@ struct VerifySampledLayout {
 VerifySampledLayout verify_sampled_layout(const dels_local_head* head, int B, int n, int V, dels_dtype tdt, int sms) {
   VerifySampledLayout L{};
   const int es_t = tdt == DELS_F32 ? 4 : 2;
-  const bool vec = (V % (16 / es_t)) == 0;
+  const bool vec = (V % 8) == 0;
   const int rows = B * (n + 1);
   L.t = plan_rows(std::max(rows, 1), V, es_t, sms, vec, 1 << 20);
   L.r_nchunks = std::max(1, std::min((V + 2047) / 2048, (4 * sms + std::max(B, 1) - 1) / std::max(B, 1)));
@@ -1741,6 +1751,7 @@ int dels_verify_block_sampled(const dels_local_head* head, const int32_t* draft_
     return DELS_ERR_BAD_DTYPE;
   if (B < 0 || n < 1 || n > kMaxSampledBlock || V < 1) return DELS_ERR_BAD_SHAPE;
   if ((long long)B * (n + 1) > INT32_MAX) return DELS_ERR_BAD_SHAPE;
+  if (!sample_counter_ok(B, step)) return DELS_ERR_BAD_SHAPE;
   const bool bf = head->wdtype == DELS_BF16;
   if (bf && B > kMaxBatchTile) return DELS_ERR_BAD_SHAPE;
   for (int j = 0; j < n; ++j)
@@ -1773,7 +1784,7 @@ int dels_verify_block_sampled(const dels_local_head* head, const int32_t* draft_
   t.partial_ld = L.t.nchunks;
   t.status = status;
   const int es_t = target_dtype == DELS_F32 ? 4 : 2;
-  const bool vec = (V % (16 / es_t)) == 0;
+  const bool vec = (V % 8) == 0;
   { PROF(DELS_KCLASS_VERIFY); DELS_CUDA(launch_combine_rows(t, target_dtype, vec, false, s)); }
   // 2. the acceptance tests and the rejected position's input
   VerifySampledArgs a{};

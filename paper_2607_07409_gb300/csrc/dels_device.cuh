@@ -93,13 +93,16 @@ __device__ __forceinline__ float ex2_approx(float x) {
 constexpr float kLog2e = 1.4426950408889634f;
 
 // lse_chunk with the exponent pre-scaled to base 2: one FFMA + one ex2 per
-// element (exp(x - best) = 2^(x*log2e - best*log2e)).
+// element (exp(x - best) = 2^(x*log2e - best*log2e)). The running sum is
+// rescaled only when the maximum moved (rare after the first chunks).
 template <int K>
 __device__ __forceinline__ void lse_chunk_ex2(const float (&x)[K], float best, float& m, float& s) {
   if (best == -INFINITY) return;
   const float nb = -best * kLog2e;
-  s *= ex2_approx(fmaf(m, kLog2e, nb));
-  m = best;
+  if (best != m) {
+    s *= ex2_approx(fmaf(m, kLog2e, nb));
+    m = best;
+  }
   float acc = 0.f;
 #pragma unroll
   for (int i = 0; i < K; ++i) acc += ex2_approx(fmaf(x[i], kLog2e, nb));
@@ -171,77 +174,80 @@ __device__ __forceinline__ void write_decode(const RowAcc& r, long long out_i, i
 }
 
 // ----------------------------------------------------------------------------
-// temperature 1: Gumbel-max draws with Philox4x64-10 uniforms
+// temperature 1: Gumbel-max draws with Philox4x32-10 uniforms
 // ----------------------------------------------------------------------------
-// Philox4x64-10 (Salmon, Moraes, Dror and Shaw, "Parallel random numbers: as
-// easy as 1, 2, 3", SC 2011): ten rounds of two 64 x 64 -> 128-bit products
-// on a 4-word counter, the key bumped by two Weyl constants between rounds.
-constexpr uint64_t kPhiloxM0 = 0xD2E7470EE14C6C93ull, kPhiloxM1 = 0xCA5A826395121157ull;
-constexpr uint64_t kPhiloxW0 = 0x9E3779B97F4A7C15ull, kPhiloxW1 = 0xBB67AE8584CAA73Bull;
+// Philox4x32-10 (Salmon, Moraes, Dror and Shaw, "Parallel random numbers: as
+// easy as 1, 2, 3", SC 2011): ten rounds of two 32 x 32 -> 64-bit products on
+// a counter of four 32-bit words, the key bumped by two Weyl constants
+// between rounds.
+constexpr uint32_t kPhiloxM0 = 0xD2511F53u, kPhiloxM1 = 0xCD9E8D57u;
+constexpr uint32_t kPhiloxW0 = 0x9E3779B9u, kPhiloxW1 = 0xBB67AE85u;
 enum { kStreamDraft = 0, kStreamAccept = 1, kStreamResidual = 2 };
 
-__device__ __forceinline__ void philox4x64_10(uint64_t (&x)[4], uint64_t k0, uint64_t k1) {
+__device__ __forceinline__ void philox4x32_10(uint32_t (&x)[4], uint32_t k0, uint32_t k1) {
 #pragma unroll
   for (int r = 0; r < 10; ++r) {
-    const uint64_t hi0 = __umul64hi(kPhiloxM0, x[0]), lo0 = kPhiloxM0 * x[0];
-    const uint64_t hi1 = __umul64hi(kPhiloxM1, x[2]), lo1 = kPhiloxM1 * x[2];
-    const uint64_t y0 = hi1 ^ x[1] ^ k0, y2 = hi0 ^ x[3] ^ k1;
-    x[0] = y0;
+    const uint32_t hi0 = __umulhi(kPhiloxM0, x[0]), lo0 = kPhiloxM0 * x[0];
+    const uint32_t hi1 = __umulhi(kPhiloxM1, x[2]), lo1 = kPhiloxM1 * x[2];
+    x[0] = hi1 ^ x[1] ^ k0;
     x[1] = lo1;
-    x[2] = y2;
+    x[2] = hi0 ^ x[3] ^ k1;
     x[3] = lo0;
     k0 += kPhiloxW0;
     k1 += kPhiloxW1;
   }
 }
 
-// A 32-bit half h gives u = (floor(h / 2^9) + 1/2) / 2^23, exact in float32.
+// A 32-bit output word h gives u = (floor(h / 2^9) + 1/2) / 2^23, exact in
+// float32: with k = floor(h / 2^9), the float 1 + k 2^-23 (k as the mantissa)
+// minus (1 - 2^-24) is (2k + 1) 2^-24, which a float holds exactly.
 __device__ __forceinline__ float uniform_from_bits(uint32_t h) {
-  return (float)(2u * (h >> 9) + 1u) * 5.9604644775390625e-08f;   // (2k + 1) * 2^-24
+  return __uint_as_float(0x3F800000u | (h >> 9)) - 0.999999940395355224609375f;
 }
 
 // Standard Gumbel variate -log(-log u): the inner log at full precision (it
 // decides how close to 1 u may be), the outer one through the fast log.
 __device__ __forceinline__ float gumbel_from_bits(uint32_t h) { return -__logf(-logf(uniform_from_bits(h))); }
 
-// Counter (v / 8, j, b, stream), key (seed, step): the 8 uniforms of
-// vocabulary indices 8c .. 8c + 7 are the halves of the 4 output words, high
-// half first.
+// Key (seed mod 2^32, seed div 2^32), counter (c, step, b + 2^16 j + 2^24
+// stream, 0): the 4 uniforms of vocabulary indices 4c .. 4c + 3, one per
+// output word. step < 2^32, b < 2^16, j < 2^8 (checked by the entry points).
 __device__ __forceinline__ void philox_block(uint64_t seed, uint64_t step, int b, int j, int stream, long long c,
-                                             uint64_t (&x)[4]) {
-  x[0] = (uint64_t)c;
-  x[1] = (uint64_t)j;
-  x[2] = (uint64_t)b;
-  x[3] = (uint64_t)stream;
-  philox4x64_10(x, seed, step);
+                                             uint32_t (&x)[4]) {
+  x[0] = (uint32_t)c;
+  x[1] = (uint32_t)step;
+  x[2] = (uint32_t)b | ((uint32_t)j << 16) | ((uint32_t)stream << 24);
+  x[3] = 0u;
+  philox4x32_10(x, (uint32_t)seed, (uint32_t)(seed >> 32));
 }
 
-__device__ __forceinline__ void gumbel8(uint64_t seed, uint64_t step, int b, int j, int stream, long long c,
+// The Gumbel variates of vocabulary indices 8 c8 .. 8 c8 + 7 (two blocks).
+__device__ __forceinline__ void gumbel8(uint64_t seed, uint64_t step, int b, int j, int stream, long long c8,
                                         float (&g)[8]) {
-  uint64_t x[4];
-  philox_block(seed, step, b, j, stream, c, x);
+  uint32_t x[4], y[4];
+  philox_block(seed, step, b, j, stream, 2 * c8, x);
+  philox_block(seed, step, b, j, stream, 2 * c8 + 1, y);
 #pragma unroll
   for (int k = 0; k < 4; ++k) {
-    g[2 * k] = gumbel_from_bits((uint32_t)(x[k] >> 32));
-    g[2 * k + 1] = gumbel_from_bits((uint32_t)x[k]);
+    g[k] = gumbel_from_bits(x[k]);
+    g[4 + k] = gumbel_from_bits(y[k]);
   }
 }
 
-__device__ __forceinline__ uint32_t philox_half_at(uint64_t seed, uint64_t step, int b, int j, int stream,
+__device__ __forceinline__ uint32_t philox_word_at(uint64_t seed, uint64_t step, int b, int j, int stream,
                                                    long long v) {
-  uint64_t x[4];
-  philox_block(seed, step, b, j, stream, v >> 3, x);
-  const int w = (int)((v & 7) >> 1);
-  const uint64_t word = w == 0 ? x[0] : w == 1 ? x[1] : w == 2 ? x[2] : x[3];
-  return (v & 1) ? (uint32_t)word : (uint32_t)(word >> 32);
+  uint32_t x[4];
+  philox_block(seed, step, b, j, stream, v >> 2, x);
+  const int w = (int)(v & 3);
+  return w == 0 ? x[0] : w == 1 ? x[1] : w == 2 ? x[2] : x[3];
 }
 
 __device__ __forceinline__ float gumbel_at(uint64_t seed, uint64_t step, int b, int j, int stream, long long v) {
-  return gumbel_from_bits(philox_half_at(seed, step, b, j, stream, v));
+  return gumbel_from_bits(philox_word_at(seed, step, b, j, stream, v));
 }
 
 __device__ __forceinline__ float uniform_at(uint64_t seed, uint64_t step, int b, int j, int stream, long long v) {
-  return uniform_from_bits(philox_half_at(seed, step, b, j, stream, v));
+  return uniform_from_bits(philox_word_at(seed, step, b, j, stream, v));
 }
 
 // A record of temperature-1 drafting holds the largest key k = l + g, its

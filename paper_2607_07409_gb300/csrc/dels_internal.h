@@ -55,6 +55,8 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
 }
 
 // ---- row reductions (combine / verify / draft position 0) -------------------
+constexpr int kMaxVerifyBlock = 1024;    // greedy verification: n <= 1024 draft positions
+
 struct RowsArgs {
   const void* longp;
   const void* shortp;
@@ -67,7 +69,7 @@ struct RowsArgs {
   int rows_per_cta;              // R
   void* partials;                // [rows][partial_ld] 16-byte records
   int partial_ld;
-  int* counters;                 // per row group (combine) / per row (verify)
+  int* counters;                 // combine: one ticket per row group
   int* counters_b;               // verify: per request
   int32_t* out_token;
   float* out_lp;
@@ -77,7 +79,6 @@ struct RowsArgs {
   int n;                         // draft positions (verify)
   int32_t* out_accept;
   int32_t* out_bonus;
-  int32_t* targ_scratch;         // [rows] target argmax (workspace)
   int* status;
 };
 
@@ -85,15 +86,30 @@ struct RowsPlan {
   int nchunks, chunk_cols, rows_per_cta, grid;
 };
 
+// Chunks per row for the row kernels. slots_per_sm > 0 (resident CTAs per
+// SM): when every row group fits in one wave, as many chunks as that wave
+// holds; otherwise about 16 CTAs per SM.
 RowsPlan plan_rows(int rows, int V, int bytes_per_col, int num_sms, bool vec, int max_chunks,
-                  bool multi_row = false);
+                  bool multi_row = false, int slots_per_sm = 0);
+// Resident CTAs per SM of the combine (verify = false) or verification row
+// kernel for this dtype (0 if the query fails).
+int rows_slots_per_sm(bool verify, dels_dtype dt);
 cudaError_t launch_combine_rows(const RowsArgs& a, dels_dtype dt, bool vec, bool finalize, cudaStream_t s);
 cudaError_t launch_verify_rows(const RowsArgs& a, dels_dtype dt, bool vec, cudaStream_t s);
 
+// Workspace layout of dels_combine_argmax (shared with the no-allocation
+// entry point, which clears the header and the tickets itself).
+struct CombineLayout {
+  bool vec;
+  RowsPlan p;
+  size_t tickets_off, partials_off, total;
+};
+CombineLayout combine_layout(int rows, int V, dels_dtype dtype, int sms);
+
 // ---- draft merge + gather of the next local-head input ----------------------
 // Temperature-1 drafting (on = 0: temperature 0). The uniforms of (request
-// b, position j, stream, vocabulary index) come from Philox4x64-10 under the
-// key (seed, step).
+// b, position j, stream, vocabulary index) come from Philox4x32-10 keyed by
+// the seed, with the step in the counter.
 struct SampleArgs {
   int on;
   unsigned long long seed, step;
@@ -118,6 +134,9 @@ cudaError_t launch_sample_rows(const SampleRowsArgs& a, bool f32, cudaStream_t s
 
 // Verification of a temperature-1 block by lossless speculative sampling.
 constexpr int kMaxSampledBlock = 32;
+// Temperature-1 counters: the step fills one 32-bit Philox counter word and
+// the request 16 bits of another.
+inline bool sample_counter_ok(int B, unsigned long long step) { return step < (1ull << 32) && B <= (1 << 16); }
 struct VerifySampledArgs {
   int B, n, V;
   const int32_t* draft;          // [B, n]
@@ -208,7 +227,7 @@ struct TcGemmArgs {
   int partial_ld;
   int* status;
   int debug_skip_producer;       // test hook: producer never fills (exercises the bounded waits)
-  // EPI_COMBINE at temperature 1: Gumbel-max keys (Philox4x64-10 under (seed, step))
+  // EPI_COMBINE at temperature 1: Gumbel-max keys (Philox4x32-10 of (seed, step))
   int sample;
   unsigned long long seed, step;
   // EPI_STORE, optional: the K splits of one output tile run on the CTAs of

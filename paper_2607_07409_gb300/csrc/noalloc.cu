@@ -69,12 +69,8 @@ extern "C" int dels_combine_argmax_noalloc(const void* long_logits, const void* 
   if (r != DELS_OK) return r;
   // The status word and the per-row-group tickets must start at zero; the
   // scratch keeps whatever the previous call left, so clear that prefix.
-  const int sms = device_sm_count();
-  const int es = dtype == DELS_F32 ? 4 : 2;
-  const bool vec = (V % (16 / es)) == 0;
-  const RowsPlan p = plan_rows(rows, V, 2 * es, sms, vec, 1 << 20, true);
-  const size_t groups = ((size_t)rows + p.rows_per_cta - 1) / p.rows_per_cta;
-  const size_t zero_bytes = kHeaderBytes + (groups * 4 + 255) / 256 * 256;
+  const CombineLayout L = combine_layout(rows, V, dtype, device_sm_count());
+  const size_t zero_bytes = L.partials_off;   // the header and the tickets
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   if (cudaMemsetAsync(scratch, 0, zero_bytes, s) != cudaSuccess) return DELS_ERR_CUDA;
   return dels_combine_argmax(long_logits, short_logits, dtype, log_prior, alpha, beta, rows, V, out_token,

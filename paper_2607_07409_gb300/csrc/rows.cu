@@ -7,6 +7,7 @@
 // loads (streaming cache hint) and keeps its per-row state in registers; a
 // row split over several CTAs is finished by the last CTA to arrive (atomic
 // ticket, reset by that CTA), so no [rows, V] intermediate is ever written.
+#include <algorithm>
 #include <climits>
 
 #include <cuda_bf16.h>
@@ -78,11 +79,19 @@ struct RowState {
   __device__ __forceinline__ void init() {
     best = -INFINITY; second = -INFINITY; m = -INFINITY; s = 0.f; idx = INT_MAX;
   }
+  // An element at or below the runner-up changes neither the top-1 nor the
+  // top-2, so the element-wise top-2 update runs only for groups whose
+  // maximum exceeds the runner-up (rare once the row's head is seen).
   template <int K>
   __device__ __forceinline__ void push(const float (&f)[K], int c) {
+    float vm = f[0];
 #pragma unroll
-    for (int i = 0; i < K; ++i) top2_push(f[i], c + i, best, second, idx);
-    lse_chunk<K>(f, best, m, s);
+    for (int i = 1; i < K; ++i) vm = fmaxf(vm, f[i]);
+    if (vm > second) {
+#pragma unroll
+      for (int i = 0; i < K; ++i) top2_push(f[i], c + i, best, second, idx);
+    }
+    lse_chunk_ex2<K>(f, best, m, s);
   }
   __device__ __forceinline__ RowAcc acc() const {
     RowAcc r;
@@ -115,7 +124,7 @@ __device__ __forceinline__ void block_reduce_rows(const RowAcc (&acc)[R], RowAcc
 // fused combine: l = l_L + alpha l_S - beta l_P, then top-1/top-2/LSE per row
 // ----------------------------------------------------------------------------
 template <typename T, int R, bool VEC, bool SH, bool PR, bool FINAL>
-__global__ void __launch_bounds__(kRowsThreads) k_combine_rows(RowsArgs a) {
+__global__ void __launch_bounds__(kRowsThreads, sizeof(T) == 2 ? 4 : 2) k_combine_rows(RowsArgs a) {
   if (threadIdx.x == 0) pdl_trigger();
   pdl_wait();
   const int chunk = blockIdx.x % a.nchunks;
@@ -139,7 +148,7 @@ __global__ void __launch_bounds__(kRowsThreads) k_combine_rows(RowsArgs a) {
     // per SM instead of four the issue-heavy bf16 update stalls (measured
     // 172 us against 126 us for 1024 rows of 151936).
     constexpr int WPV = sizeof(T) == 2 ? 1 : 2;            // 16-byte words per 8 values
-    constexpr int U = (R == 1) ? 4 : 1;
+    constexpr int U = (R == 1) ? 4 : (R == 2 ? 2 : 1);
     const int step = kRowsThreads * 8;
     for (int cb = c0 + threadIdx.x * 8; cb < c1; cb += step * U) {
       uint4 lw[U][R][WPV];
@@ -199,7 +208,7 @@ __global__ void __launch_bounds__(kRowsThreads) k_combine_rows(RowsArgs a) {
                 if constexpr (PR) x = fmaf(nbeta, pv[i], x);
                 f[i] = x;
               }
-              st[r].push<8>(f, c);
+              st[r].template push<8>(f, c);
             }
           }
         }
@@ -215,7 +224,7 @@ __global__ void __launch_bounds__(kRowsThreads) k_combine_rows(RowsArgs a) {
           if constexpr (SH) x = fmaf(alpha, load1(S + (long long)r * a.ld_short + c), x);
           if constexpr (PR) x = fmaf(nbeta, p, x);
           float f[1] = {x};
-          st[r].push<1>(f, c);
+          st[r].template push<1>(f, c);
         }
       }
     }
@@ -358,53 +367,52 @@ __global__ void __launch_bounds__(kRowsThreads) k_verify_rows(RowsArgs a) {
 
   __shared__ ArgAcc red[kRowsThreads / 32];
   __shared__ int s_last;
+  __shared__ int s_targ[kMaxVerifyBlock + 1];
   ArgAcc x{best, idx, nan_seen ? 1 : 0};
   x = argacc_warp_reduce(x);
   if (lane == 0) red[warp] = x;
   __syncthreads();
-  if (warp != 0) return;
-  x = lane < kRowsThreads / 32 ? red[lane] : ArgAcc{-INFINITY, INT_MAX, 0};
-  x = argacc_warp_reduce(x);
-
-  if (a.nchunks > 1) {
-    int last = 0;
+  // One ticket per request over its (n + 1) rows x nchunks records: the last
+  // CTA to publish merges every row of the request and takes the accept
+  // length and the bonus token.
+  const int n = a.n;
+  const int b = row / (n + 1);
+  if (warp == 0) {
+    x = lane < kRowsThreads / 32 ? red[lane] : ArgAcc{-INFINITY, INT_MAX, 0};
+    x = argacc_warp_reduce(x);
     if (lane == 0) {
       reinterpret_cast<float4*>(a.partials)[(long long)row * a.partial_ld + chunk] =
           make_float4(x.best, __int_as_float(x.idx), __int_as_float(x.nan), 0.f);
       __threadfence();
-      last = (atomicAdd(&a.counters[row], 1) == a.nchunks - 1);
+      s_last = (atomicAdd(&a.counters_b[b], 1) == (n + 1) * a.nchunks - 1);
     }
-    last = __shfl_sync(0xFFFFFFFFu, last, 0);
-    if (!last) return;
-    __threadfence();
+  }
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  const long long row0 = (long long)b * (n + 1);
+  for (int j = warp; j <= n; j += kRowsThreads / 32) {
     ArgAcc y{-INFINITY, INT_MAX, 0};
     for (int k = lane; k < a.nchunks; k += 32) {
-      const float4 v = __ldcg(reinterpret_cast<const float4*>(a.partials) + (long long)row * a.partial_ld + k);
+      const float4 v = __ldcg(reinterpret_cast<const float4*>(a.partials) + (row0 + j) * a.partial_ld + k);
       y = argacc_merge(y, ArgAcc{v.x, __float_as_int(v.y), __float_as_int(v.z)});
     }
-    x = argacc_warp_reduce(y);
-    if (lane == 0) a.counters[row] = 0;
+    y = argacc_warp_reduce(y);
+    if (lane == 0) {
+      if (y.nan) raise_status(a.status, DELS_STATUS_NONFINITE);
+      const int t = (y.idx == INT_MAX) ? 0 : y.idx;   // an all -inf row: first index
+      s_targ[j] = t;
+      if (a.out_token) a.out_token[row0 + j] = t;
+    }
   }
-  if (lane != 0) return;
-  (void)s_last;
-
-  // this CTA holds the finished argmax of `row`
-  if (x.nan) raise_status(a.status, DELS_STATUS_NONFINITE);
-  const int t = (x.idx == INT_MAX) ? 0 : x.idx;   // an all -inf row: first index
-  const int n = a.n;
-  const int b = row / (n + 1);
-  a.targ_scratch[row] = t;
-  if (a.out_token) a.out_token[row] = t;
-  __threadfence();
-  if (atomicAdd(&a.counters_b[b], 1) != n) return;
-  __threadfence();
+  __syncthreads();
+  if (threadIdx.x != 0) return;
   int acc = 0;
   bool bad = false;
   for (; acc < n; ++acc) {
     const int xd = a.draft[(long long)b * n + acc];
     bad |= (xd < 0 || xd >= a.V);
-    const int tj = __ldcg(a.targ_scratch + (long long)b * (n + 1) + acc);
-    if (xd != tj) break;
+    if (xd != s_targ[acc]) break;
   }
   for (int k = acc; k < n && !bad; ++k) {
     const int xd = a.draft[(long long)b * n + k];
@@ -412,7 +420,7 @@ __global__ void __launch_bounds__(kRowsThreads) k_verify_rows(RowsArgs a) {
   }
   if (bad) raise_status(a.status, DELS_STATUS_BAD_TOKEN);
   a.out_accept[b] = acc;
-  a.out_bonus[b] = __ldcg(a.targ_scratch + (long long)b * (n + 1) + acc);
+  a.out_bonus[b] = s_targ[acc];
   a.counters_b[b] = 0;
 }
 
@@ -492,31 +500,67 @@ cudaError_t dispatch_rv(const RowsArgs& a, bool vec, bool finalize, cudaStream_t
   if (a.rows_per_cta == 4) {
     return vec ? dispatch_sp<T, 4, true>(a, finalize, s) : dispatch_sp<T, 4, false>(a, finalize, s);
   }
+  if (a.rows_per_cta == 2 && vec) return dispatch_sp<T, 2, true>(a, finalize, s);
   return vec ? dispatch_sp<T, 1, true>(a, finalize, s) : dispatch_sp<T, 1, false>(a, finalize, s);
 }
 
 }  // namespace
 
-RowsPlan plan_rows(int rows, int V, int bytes_per_col, int num_sms, bool vec, int max_chunks, bool multi_row) {
+RowsPlan plan_rows(int rows, int V, int bytes_per_col, int num_sms, bool vec, int max_chunks, bool multi_row,
+                   int slots_per_sm) {
   RowsPlan p{};
-  const long long target_items = 16LL * num_sms;
-  // Four rows per CTA (the prior read once per four rows) only for very many
-  // short rows; measured slower than one row per CTA otherwise.
-  p.rows_per_cta = (multi_row && vec && rows >= 64LL * num_sms) ? 4 : 1;
+  const long long slots = (long long)slots_per_sm * num_sms;
+  // Rows per CTA (the prior read once for all of them): four for very many
+  // short rows; two for bf16 combines whose rows do not fit in one wave of
+  // resident CTAs (measured: 1024 rows of 151936, 141 -> 133 us; 1024 rows of
+  // 32000, 53 -> 39 us; no gain for f32 rows or for fewer rows).
+  p.rows_per_cta = 1;
+  if (multi_row && vec && rows >= 64LL * num_sms) p.rows_per_cta = 4;
+  else if (multi_row && vec && bytes_per_col <= 4 && slots > 0 && rows > slots) p.rows_per_cta = 2;
   const long long groups0 = ((long long)rows + p.rows_per_cta - 1) / p.rows_per_cta;
   int nchunks = 1;
-  if (groups0 > 0 && groups0 < target_items) nchunks = (int)((target_items + groups0 - 1) / groups0);
-  const int min_cols = std::max(2048, 32768 / std::max(1, bytes_per_col));
-  nchunks = std::min(nchunks, std::max(1, V / min_cols));
+  if (slots > 0 && groups0 > 0 && groups0 <= slots) {
+    // every row group fits in one wave of resident CTAs: split the rows into
+    // as many chunks as that wave holds (a second, partial wave would cost a
+    // whole CTA lifetime for a few CTAs), down to 2048 columns (one 8-value
+    // group per thread), so that small calls take one round trip per CTA
+    nchunks = (int)std::min<long long>(slots / groups0, std::max(1, V / 2048));
+  } else {
+    const long long target_items = 16LL * num_sms;
+    if (groups0 > 0 && groups0 < target_items) nchunks = (int)((target_items + groups0 - 1) / groups0);
+    const int min_cols = std::max(2048, 32768 / std::max(1, bytes_per_col));
+    nchunks = std::min(nchunks, std::max(1, V / min_cols));
+  }
   nchunks = std::max(1, std::min(nchunks, max_chunks));
   int chunk_cols = (V + nchunks - 1) / nchunks;
   chunk_cols = (chunk_cols + 7) / 8 * 8;
   nchunks = (V + chunk_cols - 1) / chunk_cols;
   p.nchunks = std::max(1, nchunks);
   p.chunk_cols = std::max(8, chunk_cols);
-  const long long groups = groups0;
-  p.grid = (int)std::min<long long>(groups * p.nchunks, INT_MAX);
+  p.grid = (int)std::min<long long>(groups0 * p.nchunks, INT_MAX);
   return p;
+}
+
+int rows_slots_per_sm(bool verify, dels_dtype dt) {
+  // resident CTAs per SM of the main instantiation (all four combine
+  // variants use the same registers to within a few), queried once
+  static int cache[4] = {-1, -1, -1, -1};
+  const int k = (verify ? 2 : 0) + (dt == DELS_F32 ? 1 : 0);
+  if (cache[k] < 0) {
+    int n = 0;
+    cudaError_t e;
+    if (verify)
+      e = dt == DELS_F32 ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_verify_rows<float, true>, kRowsThreads, 0)
+                         : cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_verify_rows<uint16_t, true>, kRowsThreads, 0);
+    else
+      e = dt == DELS_F32
+              ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_combine_rows<float, 1, true, true, true, true>,
+                                                              kRowsThreads, 0)
+              : cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_combine_rows<uint16_t, 1, true, true, true, true>,
+                                                              kRowsThreads, 0);
+    cache[k] = (e == cudaSuccess && n > 0) ? n : 0;
+  }
+  return cache[k];
 }
 
 cudaError_t launch_combine_rows(const RowsArgs& a, dels_dtype dt, bool vec, bool finalize, cudaStream_t s) {

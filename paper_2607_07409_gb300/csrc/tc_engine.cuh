@@ -362,8 +362,17 @@ __device__ __forceinline__ void combine_chunk(const float (&acc)[32], const uint
     for (int t = 0; t < 4; ++t) {
       float g[8];
       gumbel8(sa->seed, sa->step, b, sa->j, kStreamDraft, (cbase >> 3) + t, g);
+      // keys at or below the runner-up change neither the top-1 nor the top-2
+      float k[8], km = -INFINITY;
 #pragma unroll
-      for (int i = 0; i < 8; ++i) top2_push(f[t * 8 + i] + g[i], cbase + t * 8 + i, best, second, idx);
+      for (int i = 0; i < 8; ++i) {
+        k[i] = f[t * 8 + i] + g[i];
+        km = fmaxf(km, k[i]);
+      }
+      if (km > second) {
+#pragma unroll
+        for (int i = 0; i < 8; ++i) top2_push(k[i], cbase + t * 8 + i, best, second, idx);
+      }
     }
   } else {
 #pragma unroll

@@ -57,6 +57,10 @@ def _combine(long, short, prior, alpha, beta):
     (2, 151936, "f32", 0.5),       # few rows: split over many CTAs + last-CTA merge
     (1, 151936, "bf16", 1.0),
     (33, 5000, "f32", 0.0),
+    (3, 1004, "f32", 0.5),         # V = 4 mod 8: element-wise path
+    (5, 16392, "bf16", 0.5),       # streamed rows: the shortest streamed V, rows cut between CTAs
+    (40, 32000, "f32", 0.3),       # streamed rows, f32
+    (150, 20000, "bf16", 1.0),     # streamed rows, about one row per CTA
 ])
 def test_combine_matches_oracle(rows, V, dtype, w):
     d = synth.make_combine_inputs(rows, V, dtype, seed=rows * 31 + V, device=DEV)
@@ -90,12 +94,12 @@ def test_combine_optional_terms_absent():
     check_rows(tok, lp, gap, rt, rl, rg, exact_ties=True)
 
 
-def test_combine_masked_and_nonfinite_rows():
-    V = 2048
+@pytest.mark.parametrize("V", [2048, 32768])      # row kernel / streamed rows
+def test_combine_masked_and_nonfinite_rows(V):
     long = torch.randn(4, V, device=DEV) * 3
     long[0, :100] = -float("inf")            # masked entries are allowed
     long[1, :] = -float("inf")               # all masked: error
-    long[2, 77] = float("nan")               # NaN: error
+    long[2, V - 77] = float("nan")           # NaN: error
     long[3, 5] = float("inf")                # +inf: error
     tok, lp, gap, st = _combine(long, None, None, 0.0, 0.0)
     assert st & dels.DELS_STATUS_NONFINITE
@@ -129,6 +133,7 @@ def _verify(draft, target):
 
 @pytest.mark.parametrize("B,n,V,dtype", [
     (9, 6, 50, "bf16"), (5, 16, 151936, "bf16"), (3, 8, 32000, "f32"), (17, 4, 1003, "f32"), (2, 32, 4099, "bf16"),
+    (4, 3, 1004, "f32"), (1, 1, 16384, "bf16"), (64, 16, 151936, "f32"),
 ])
 def test_verify_planted_prefix(B, n, V, dtype):
     t, draft, planted, accept = synth.make_planted_verify(B, n, V, dtype, seed=B * n, device=DEV)
@@ -139,10 +144,12 @@ def test_verify_planted_prefix(B, n, V, dtype):
     np.testing.assert_array_equal(bonus, planted.numpy()[np.arange(B), accept.numpy()])
 
 
-def test_verify_random_ties_match_oracle():
-    B, n, V = 40, 5, 3000
-    g = torch.Generator().manual_seed(3)
-    T = torch.randint(-3, 3, (B, n + 1, V), generator=g).to(torch.bfloat16)     # many exact ties
+@pytest.mark.parametrize("B,n,V,dtype", [(40, 5, 3000, "bf16"), (6, 5, 32000, "bf16"), (5, 3, 20000, "f32")])
+def test_verify_random_ties_match_oracle(B, n, V, dtype):
+    """Small integer logits: many exact ties inside every quad, CTA and row,
+    all resolved to the lowest index (row kernel and streamed rows)."""
+    g = torch.Generator().manual_seed(3 + V)
+    T = torch.randint(-3, 3, (B, n + 1, V), generator=g).to(torch.bfloat16 if dtype == "bf16" else torch.float32)
     draft = torch.randint(0, 2, (B, n), generator=g).to(torch.int32)
     acc, bonus, targ, st, _ = _verify(draft.to(DEV), T.to(DEV))
     ra, rb, rt = oracle.verify_greedy(draft.numpy(), T)
@@ -151,20 +158,22 @@ def test_verify_random_ties_match_oracle():
     np.testing.assert_array_equal(bonus, rb)
 
 
-def test_verify_repeated_calls_reuse_workspace():
-    t, draft, planted, accept = synth.make_planted_verify(6, 7, 999, "f32", seed=5, device=DEV)
+@pytest.mark.parametrize("V", [999, 40000])
+def test_verify_repeated_calls_reuse_workspace(V):
+    t, draft, planted, accept = synth.make_planted_verify(6, 7, V, "f32", seed=5, device=DEV)
     acc, bonus, targ, st, (ws, nbytes) = _verify(draft, t)
     for _ in range(3):   # tickets must reset between calls
         a2 = torch.empty(6, dtype=torch.int32, device=DEV)
         b2 = torch.empty(6, dtype=torch.int32, device=DEV)
-        assert dels.dels_verify_block(draft, t, dels.DELS_F32, 6, 7, 999, a2, b2, None, ws, nbytes) == 0
+        assert dels.dels_verify_block(draft, t, dels.DELS_F32, 6, 7, V, a2, b2, None, ws, nbytes) == 0
         torch.cuda.synchronize()
         np.testing.assert_array_equal(a2.cpu().numpy(), accept.numpy())
 
 
-def test_verify_bad_draft_token_flags_status():
-    t, draft, planted, accept = synth.make_planted_verify(3, 4, 100, "f32", seed=6, device=DEV)
-    draft[2, 3] = 100
+@pytest.mark.parametrize("V", [100, 16384])
+def test_verify_bad_draft_token_flags_status(V):
+    t, draft, planted, accept = synth.make_planted_verify(3, 4, V, "f32", seed=6, device=DEV)
+    draft[2, 3] = V
     _, _, _, st, _ = _verify(draft, t)
     assert st & dels.DELS_STATUS_BAD_TOKEN
 

@@ -1,7 +1,7 @@
 """GPU parity of temperature-1 drafting (Algorithm 1 with Decode = a draw from
 the softmax by the Gumbel-max rule) against the oracle.
 
-Both sides draw the same Philox4x64-10 uniforms, so a device token must be
+Both sides draw the same Philox4x32-10 uniforms, so a device token must be
 the oracle's argmax of the keys l + g at every position, except where the
 oracle's top-2 key gap is a near-tie (then within the tie tolerance of the
 maximum key); the drafted prefix is re-checked in the oracle's forced mode.
@@ -35,9 +35,12 @@ def _sampled(name, seed=17, step=3, weights="learned"):
     return w, d, W, a, b, tok.cpu().numpy(), lp.cpu().numpy(), gap.cpu().numpy(), state
 
 
-@pytest.mark.parametrize("name", ["gru", "gru_b64", "mlp2", "xfmr", "markov", "gru_f32", "tiny"])
-def test_sampled_draft_matches_oracle(name):
-    seed, step = 17, 3
+@pytest.mark.parametrize("name,seed,step", [("gru", 17, 3), ("gru_b64", 17, 3), ("mlp2", 17, 3), ("xfmr", 17, 3),
+                                            ("markov", 17, 3), ("gru_f32", 17, 3), ("tiny", 17, 3),
+                                            ("gru", 0xFEDCBA9876543210, 2 ** 32 - 1)])
+def test_sampled_draft_matches_oracle(name, seed, step):
+    """Every head; the last case puts both halves of the key and the whole
+    step word of the counter to use."""
     w, d, W, a, b, tok, lp, gap, state = _sampled(name, seed, step)
     tol = LP_TOL_F32 if w.head.wdtype == "f32" else LP_TOL_BF16
     info = check_draft(tok, lp, gap, _oracle_head(w, W), d["long"].cpu(), oracle.log_prior(d["counts"]),
@@ -46,6 +49,17 @@ def test_sampled_draft_matches_oracle(name):
     lse = state[: w.B * w.n * 4].view(torch.float32).view(w.B, w.n).cpu().numpy()
     np.testing.assert_allclose(lse, info["ref"].lse, rtol=0, atol=tol * 4)
     print(name, record(f"sampled draft {name}", info))
+
+
+def test_sampled_calls_reject_a_step_outside_the_counter_word():
+    w = synth.stress(SMALL["gru"])
+    d = synth.make_inputs(w, device=DEV, target=False)
+    W = {k[5:]: v for k, v in d.items() if k.startswith("head.")}
+    prior = dels.dels_prior_from_counts(d["counts"]).to(DEV)
+    dr = dels.Drafter(w.head, W, w.B, w.n, w.V)
+    with pytest.raises(dels.DelsError) as e:
+        dr.sample(d["long"], prior, [0.3] * w.n, [0.3] * w.n, 1, 2 ** 32)
+    assert e.value.code == dels.DELS_ERR_BAD_SHAPE
 
 
 def test_sampled_draft_depends_on_seed_and_step_only():

@@ -555,18 +555,55 @@ def test_per_position_weights_brute_force_enumeration():
 
 # ------------------------------------------- temperature 1 (Algorithm 1 Decode ~ softmax)
 
-def test_philox_matches_numpys_philox4x64():
-    """Philox4x64-10 against numpy's Philox bit generator (which adds one to the
-    counter before each block of four outputs)."""
-    rng = np.random.default_rng(5)
-    for _ in range(20):
-        c = [int(x) for x in rng.integers(1, 2 ** 63, size=4, dtype=np.int64)]
-        k = [int(x) for x in rng.integers(0, 2 ** 63, size=2, dtype=np.int64)]
-        bg = np.random.Philox(counter=np.array([c[0] - 1, c[1], c[2], c[3]], dtype=np.uint64),
-                              key=np.array(k, dtype=np.uint64))
-        want = [int(x) for x in bg.random_raw(4)]
-        got = [int(x) for x in oracle.philox4x64_10(np.uint64(c[0]), c[1], c[2], c[3], k[0], k[1])]
-        assert got == want
+def _curand_host_philox(seed, offset, count):
+    """`count` 32-bit outputs of cuRAND's host-side Philox4x32-10 generator
+    (CURAND_RNG_PSEUDO_PHILOX4_32_10 = 161, default ordering) from `offset`."""
+    import ctypes
+    import os
+    lib = None
+    for name in (os.path.join(os.environ.get("CUDA_HOME", "/usr/local/cuda"), "lib64", "libcurand.so"),
+                 "libcurand.so", "libcurand.so.10"):
+        try:
+            lib = ctypes.CDLL(name)
+            break
+        except OSError:
+            continue
+    if lib is None:
+        pytest.skip("libcurand is not installed")
+    gen = ctypes.c_void_p()
+    assert lib.curandCreateGeneratorHost(ctypes.byref(gen), 161) == 0
+    try:
+        assert lib.curandSetPseudoRandomGeneratorSeed(gen, ctypes.c_ulonglong(seed)) == 0
+        assert lib.curandSetGeneratorOffset(gen, ctypes.c_ulonglong(offset)) == 0
+        out = np.zeros(count, dtype=np.uint32)
+        assert lib.curandGenerate(gen, out.ctypes.data_as(ctypes.c_void_p), ctypes.c_size_t(count)) == 0
+    finally:
+        lib.curandDestroyGenerator(gen)
+    return [int(x) for x in out]
+
+
+@pytest.mark.parametrize("seed", [0, 1234, 0xFEDCBA9876543210, 2 ** 64 - 1])
+def test_philox_matches_curands_host_philox4x32(seed):
+    """Philox4x32-10 against the host generator of a library that implements
+    the same published definition. That generator uses the key (seed mod
+    2^32, seed div 2^32) and emits block k of four outputs from the counter
+    (x0, x1, x2, 0) with x2 = k mod 2^16 and x0 + 2^32 x1 = k div 2^16; the
+    cases reach every counter word the drafting path sets (word 3 is always
+    0 there) with large and small values."""
+    for x0, x1, x2 in [(0, 0, 0), (1, 0, 0), (0, 0, 1), (123456, 0, 17), (2 ** 32 - 1, 0, 65534),
+                       (5, 3, 100), (77, 1, 65534), (2 ** 31 + 9, 11, 40000)]:
+        k = x2 + (1 << 16) * (x0 + (x1 << 32))
+        want = _curand_host_philox(seed, 4 * k, 8)
+        got = oracle.philox4x32_10(np.array([x0, x0], dtype=np.uint64), x1, np.array([x2, x2 + 1], dtype=np.uint64),
+                                   0, seed & 0xFFFFFFFF, seed >> 32)
+        got = [int(got[w][i]) for i in range(2) for w in range(4)]
+        assert got == want, (seed, x0, x1, x2)
+
+
+def test_uniforms_reject_counter_fields_out_of_range():
+    for args in ((1, 2 ** 32, 0, 0, 0), (1, 0, 2 ** 16, 0, 0), (1, 0, 0, 2 ** 8, 0), (1, -1, 0, 0, 0)):
+        with pytest.raises(ValueError):
+            oracle.uniforms(*args, np.arange(4))
 
 
 def test_uniforms_lie_on_the_float32_grid_inside_the_unit_interval():
