@@ -16,7 +16,7 @@ Speculative Drafting"):
   softmax of the fused logits; the block is then verified by the target.
   Decode at temperature 0 is the argmax (lowest vocabulary index on ties);
   at temperature 1 it is a draw from the softmax by the Gumbel-max rule, with
-  Philox4x64-10 uniforms, and the block is verified by lossless speculative
+  Philox4x32-10 uniforms, and the block is verified by lossless speculative
   sampling (accept with probability min(1, p/q), resample the residual).
 * Appendix A, local heads: the RNN head (target embedding -> one bias-free GRU
   layer -> SiLU(W_rank h) -> W_vocab r) and the Markov head
