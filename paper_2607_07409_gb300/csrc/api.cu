@@ -398,7 +398,8 @@ struct DraftLayout {
   size_t u = 0, mpart = 0, h1 = 0, h2 = 0;
   int mlp_s1 = 0, mlp_s2 = 0;
   // XFMR
-  size_t ex = 0, t = 0, ab = 0, q = 0, kc = 0, vc = 0, xpart = 0, ob = 0, uu = 0, anb = 0, fb = 0, y = 0, feat = 0;
+  size_t ex = 0, t = 0, ab = 0, q = 0, kc = 0, vc = 0, xpart = 0, xpk = 0, xpv = 0, ob = 0, uu = 0, anb = 0, fb = 0,
+         y = 0, feat = 0;
   int xs_qkv = 0, xs_o = 0, xs_1 = 0, xs_2 = 0;
   // MARKOV
   size_t mk = 0;
@@ -463,6 +464,10 @@ DraftLayout draft_layout(const dels_local_head* hd, int B, int n, int V) {
       L.xs_2 = splits_for(D, 128, F, sms);
       const int smax = std::max(std::max(L.xs_qkv, L.xs_o), std::max(L.xs_1, L.xs_2));
       L.xpart = c.take((size_t)smax * T * B * std::max(D, F) * 4);
+      // the k and v products of a position have their own partials, so that
+      // the q, k and v products run back to back before one reduction
+      L.xpk = c.take((size_t)L.xs_qkv * T * B * D * 4);
+      L.xpv = c.take((size_t)L.xs_qkv * T * B * D * 4);
       L.ob = c.take((size_t)T * B * D * 2);
       L.uu = c.take((size_t)B * D * 4);
       L.anb = c.take((size_t)T * B * D * 2);
@@ -1543,6 +1548,8 @@ int draft_block_impl(const dels_local_head* head, const void* long_logits, dels_
       float* kc = at<float>(workspace, L.kc);
       float* vc = at<float>(workspace, L.vc);
       float* xpart = at<float>(workspace, L.xpart);
+      float* xpk = at<float>(workspace, L.xpk);
+      float* xpv = at<float>(workspace, L.xpv);
       uint16_t* ob = at<uint16_t>(workspace, L.ob);
       float* uu = at<float>(workspace, L.uu);
       uint16_t* anb = at<uint16_t>(workspace, L.anb);
@@ -1558,8 +1565,8 @@ int draft_block_impl(const dels_local_head* head, const void* long_logits, dels_
       RowBlocks gq, gk, gvv, go, g1, g2;
       Gemm gv;
       bool ok = plan_store_rows(gq, T * B, D, ab, head->w[1], D, L.xs_qkv, xpart, status, sms) &&
-                plan_store_rows(gk, T * B, D, ab, head->w[2], D, L.xs_qkv, xpart, status, sms) &&
-                plan_store_rows(gvv, T * B, D, ab, head->w[3], D, L.xs_qkv, xpart, status, sms) &&
+                plan_store_rows(gk, T * B, D, ab, head->w[2], D, L.xs_qkv, xpk, status, sms) &&
+                plan_store_rows(gvv, T * B, D, ab, head->w[3], D, L.xs_qkv, xpv, status, sms) &&
                 plan_store_rows(go, T * B, D, ob, head->w[4], D, L.xs_o, xpart, status, sms) &&
                 plan_store_rows(g1, T * B, F, anb, head->w[5], D, L.xs_1, xpart, status, sms) &&
                 plan_store_rows(g2, T * B, D, fb, head->w[6], F, L.xs_2, xpart, status, sms) &&
@@ -1573,22 +1580,23 @@ int draft_block_impl(const dels_local_head* head, const void* long_logits, dels_
         const int p = j - 1;   // position of the newest drafted token x_{j-1}
         { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_xfmr_embed(ex, pos, p, B, D, t, ab, s, T)); }
         { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run_rows(gq, s)); }
-        { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_splitk_finish(xpart, Sq, B, D, nullptr, ACT_NONE, q, D, nullptr, 0, s, T)); }
         { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run_rows(gk, s)); }
-        { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_splitk_finish(xpart, Sk, B, D, nullptr, ACT_NONE, kc + (size_t)p * D, P * D,
-                                       nullptr, 0, s, T)); }
         { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run_rows(gvv, s)); }
-        { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_splitk_finish(xpart, Sv, B, D, nullptr, ACT_NONE, vc + (size_t)p * D, P * D,
-                                       nullptr, 0, s, T)); }
+        {
+          SplitkJobs3 jq{};
+          jq.j[0] = SplitkJob{xpart, Sq, q, (long long)D};
+          jq.j[1] = SplitkJob{xpk, Sk, kc + (size_t)p * D, (long long)P * D};
+          jq.j[2] = SplitkJob{xpv, Sv, vc + (size_t)p * D, (long long)P * D};
+          PROF(DELS_KCLASS_HEAD_MISC);
+          DELS_CUDA(launch_splitk_finish3(jq, 3, B, D, T, s));
+        }
         { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_attention(q, kc, vc, B, D, NH, p + 1, P, ob, s, T)); }
         { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run_rows(go, s)); }
-        { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_splitk_finish(xpart, So, B, D, t, ACT_NONE, uu, D, nullptr, 0, s, T)); }
-        { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_rmsnorm_bf16(uu, B, D, D, anb, s, T)); }
+        { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_finish_rmsnorm(xpart, So, T, B, D, t, uu, anb, T, s)); }
         { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run_rows(g1, s)); }
         { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_splitk_finish(xpart, S1, B, F, nullptr, ACT_GELU, nullptr, 0, fb, F, s, T, T)); }
         { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run_rows(g2, s)); }
-        { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_splitk_finish(xpart, S2, B, D, uu, ACT_NONE, y, D, nullptr, 0, s, T)); }
-        { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_rmsnorm_bf16(y, B, D, D, feat, s, 1)); }
+        { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_finish_rmsnorm(xpart, S2, T, B, D, uu, y, feat, 1, s)); }
         gv.a.j = j;
           gv.a.sample = sm.on;
           gv.a.seed = sm.seed;

@@ -4,6 +4,8 @@
 // are float32. The large matrix products of bf16 heads run in tc_gemm.cu.
 #include <climits>
 
+#include <algorithm>
+
 #include "dels_device.cuh"
 
 namespace dels {
@@ -216,6 +218,26 @@ __global__ void k_splitk_finish(const float* __restrict__ part, int S, int B, in
   }
 }
 
+// Up to three split-K reductions in one launch (blockIdx.y = job): the same
+// sum as k_splitk_finish with in_terms-term partials, no residual, no
+// activation, float32 output with its own row pitch (the transformer head's
+// q, k and v of the newest position).
+__global__ void k_splitk_finish3(SplitkJobs3 jobs, int B, int O, int in_terms) {
+  if (threadIdx.x == 0) pdl_trigger();
+  pdl_wait();
+  const SplitkJob& jb = jobs.j[blockIdx.y];
+  const long long total = (long long)B * O;
+  const long long split_stride = total * in_terms;
+  for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < total;
+       e += (long long)gridDim.x * blockDim.x) {
+    const int b = (int)(e / O), o = (int)(e % O);
+    float acc = 0.f;
+    for (int s = 0; s < jb.S; ++s)
+      for (int t = in_terms - 1; t >= 0; --t) acc += jb.part[s * split_stride + t * total + e];
+    jb.out[(long long)b * jb.ld + o] = acc;
+  }
+}
+
 __device__ __forceinline__ float block_sum(float v) {
   __shared__ float red[32];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -247,6 +269,72 @@ __global__ void k_rmsnorm_bf16(const float* __restrict__ x, int D, int ld, uint1
   ss = block_sum(ss);
   const float inv = rsqrtf(ss / (float)D + 1e-6f);
   for (int i = threadIdx.x; i < D; i += blockDim.x) store_bf16_terms(out, terms, B, blockIdx.x, ld, i, row[i] * inv);
+}
+
+// Split-K reduction + residual followed by RMSNorm, for one row per
+// thread-block cluster of kNormCluster CTAs: each CTA reduces a slice of the
+// row (as k_splitk_finish: sum over splits, terms last to first, then the
+// residual), writes the float32 sum, and adds its slice's sum of squares into
+// every CTA of the cluster (distributed shared memory, between two cluster
+// barriers: all CTAs running, all sums written); each CTA then normalises its
+// slice and writes it as `terms` bf16 terms.
+__global__ void k_finish_rmsnorm(const float* __restrict__ part, int S, int in_terms, int B, int D,
+                                 const float* __restrict__ residual, float* __restrict__ out_f32,
+                                 uint16_t* __restrict__ norm_bf16, int terms) {
+  __shared__ float ssq[kNormCluster];
+  __shared__ float red[32];
+  if (threadIdx.x == 0) pdl_trigger();
+  pdl_wait();
+  const uint32_t rank = cluster_ctarank();
+  const int b = blockIdx.x / kNormCluster;
+  const int per = (D + kNormCluster - 1) / kNormCluster;
+  const int o0 = (int)rank * per, o1 = min(D, o0 + per);
+  const long long total = (long long)B * D;
+  const long long split_stride = total * in_terms;
+  constexpr int kMaxPer = 4;     // row elements per thread (D <= kNormCluster * 4 * blockDim.x)
+  float v[kMaxPer];
+  float ss = 0.f;
+#pragma unroll
+  for (int k = 0; k < kMaxPer; ++k) {
+    const int o = o0 + (int)threadIdx.x + k * (int)blockDim.x;
+    v[k] = 0.f;
+    if (o < o1) {
+      const long long e = (long long)b * D + o;
+      float acc = 0.f;
+      for (int s = 0; s < S; ++s)
+        for (int t = in_terms - 1; t >= 0; --t) acc += part[s * split_stride + t * total + e];
+      if (residual) acc += residual[e];
+      out_f32[e] = acc;
+      v[k] = acc;
+      ss += acc * acc;
+    }
+  }
+  // slice sum of squares (block), then into slot `rank` of every CTA of the cluster
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int d = 16; d > 0; d >>= 1) ss += __shfl_down_sync(0xFFFFFFFFu, ss, d);
+  if (lane == 0) red[warp] = ss;
+  __syncthreads();
+  if (warp == 0) {
+    const int nw = (blockDim.x + 31) >> 5;
+    ss = lane < nw ? red[lane] : 0.f;
+#pragma unroll
+    for (int d = 16; d > 0; d >>= 1) ss += __shfl_down_sync(0xFFFFFFFFu, ss, d);
+    ss = __shfl_sync(0xFFFFFFFFu, ss, 0);
+  }
+  // every CTA of the cluster is running before its shared memory is written
+  cluster_sync_all();
+  if (warp == 0 && lane < kNormCluster) st_cluster_f32(cluster_map(smem_u32(&ssq[rank]), (uint32_t)lane), ss);
+  cluster_sync_all();
+  float tot = 0.f;
+#pragma unroll
+  for (int r = 0; r < kNormCluster; ++r) tot += ssq[r];
+  const float inv = rsqrtf(tot / (float)D + 1e-6f);
+#pragma unroll
+  for (int k = 0; k < kMaxPer; ++k) {
+    const int o = o0 + (int)threadIdx.x + k * (int)blockDim.x;
+    if (o < o1) store_bf16_terms(norm_bf16, terms, B, b, D, o, v[k] * inv);
+  }
 }
 
 // t = E[x] + P[pos] (float32), a = RMSNorm(t) as `terms` bf16 terms; one CTA
@@ -406,6 +494,21 @@ cudaError_t launch_splitk_finish(const float* part, int S, int B, int O, const f
                                  int in_terms, int out_terms) {
   return launch_pdl(k_splitk_finish, dim3(grid_for((long long)B * O, 256)), dim3(256), 0, s, part, S, B, O, residual,
                     act, out_f32, ld_f32, out_bf16, ld_bf16, in_terms, out_terms);
+}
+
+cudaError_t launch_splitk_finish3(const SplitkJobs3& jobs, int njobs, int B, int O, int in_terms, cudaStream_t s) {
+  if (njobs < 1 || njobs > 3) return cudaErrorInvalidValue;
+  return launch_pdl(k_splitk_finish3, dim3(grid_for((long long)B * O, 256), njobs), dim3(256), 0, s, jobs, B, O,
+                    in_terms);
+}
+
+cudaError_t launch_finish_rmsnorm(const float* part, int S, int in_terms, int B, int D, const float* residual,
+                                  float* out_f32, uint16_t* norm_bf16, int terms, cudaStream_t s) {
+  const int per = (D + kNormCluster - 1) / kNormCluster;
+  const int threads = std::min(1024, (per + 31) / 32 * 32);
+  if ((long long)threads * 4 < per) return cudaErrorInvalidValue;   // kMaxPer elements per thread
+  return launch_pdl_cluster(k_finish_rmsnorm, dim3(B * kNormCluster), dim3(threads), 0, s, kNormCluster, part, S,
+                            in_terms, B, D, residual, out_f32, norm_bf16, terms);
 }
 
 cudaError_t launch_rmsnorm_bf16(const float* x, int B, int D, int ld, uint16_t* out, cudaStream_t s, int terms) {
