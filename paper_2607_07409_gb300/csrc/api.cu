@@ -217,10 +217,10 @@ bool plan_store(Gemm& g, int B, int O, const void* X0, const void* W0, int K0, c
   a.out_bf16 = out_bf16;
   a.ldo_bf16 = ldo_bf16;
   a.status = status;
-  a.stages = pick_stages(a, 128 * 128 + n_tile * 128, (out_f32 && !out_bf16) ? kStoreTransposeBytes : 0);
   // only the B real rows are loaded; the tile's other rows feed unused outputs
   a.a_box_rows = std::min(128, (B + 7) / 8 * 8);
   a.a_copies = 1;
+  a.stages = pick_stages(a, 128 * 128 + n_tile * 128, (out_f32 && !out_bf16) ? kStoreTransposeBytes : 0);
   if (!map_x(&g.mA0, X0, B, K0, a.a_box_rows) || !map_w(&g.mB0, W0, O, K0, n_tile)) return false;
   if (K1 > 0) {
     if (!map_x(&g.mA1, X1, B, K1, a.a_box_rows) || !map_w(&g.mB1, W1, O, K1, n_tile)) return false;
@@ -274,11 +274,6 @@ bool plan_combine(Gemm& g, int B, int V, int n, const void* X, int K, const void
   a.max_items_per_cta = (a.num_o_tiles + grid - 1) / grid;
   const int l_fixed = 2 * a.l_boxes * a.l_box_rows * 128 + a.max_items_per_cta * n_tile * 4;
   a.a_resident = (a.seg_chunks[0] <= 4) ? 1 : 0;
-  if (a.a_resident) {
-    a.stages = pick_stages(a, n_tile * 128, a.seg_chunks[0] * 128 * 128 + l_fixed);
-  } else {
-    a.stages = pick_stages(a, 128 * 128 + n_tile * 128, l_fixed);
-  }
   const int es = a.long_f32 ? 4 : 2;
   // Rows of the A tile: the B requests rounded up to whole TMEM lane
   // quadrants; when that is 32 or 64 rows, 4 or 2 copies fill the tile so
@@ -293,6 +288,11 @@ bool plan_combine(Gemm& g, int B, int V, int n, const void* X, int K, const void
     // long K leaves the epilogue ample time for the rows of one quadrant.
     a.a_box_rows = (B + 7) / 8 * 8;
     a.a_copies = 1;
+  }
+  if (a.a_resident) {
+    a.stages = pick_stages(a, n_tile * 128, a.seg_chunks[0] * 128 * 128 + l_fixed);
+  } else {
+    a.stages = pick_stages(a, 128 * 128 + n_tile * 128, l_fixed);
   }
   if (!map_x(&g.mA0, X, B, K, a.a_box_rows) || !map_w(&g.mB0, Wv, V, K, n_tile)) return false;
   if (!encode_tmap_3d(&g.mL, longp, a.long_f32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16,
@@ -1494,14 +1494,27 @@ int draft_block_impl(const dels_local_head* head, const void* long_logits, dels_
         if (!plan_combine(gv, B, V, n, feat, Hd, head->w_vocab, long_logits, logit_dtype, log_prior, alpha, beta,
                           partials, L.partial_ld, status, sms))
           return DELS_ERR_CUDA;
+        // a few requests: each layer is one CUDA-core launch (product, GELU and
+        // bf16 rounding together) instead of a split-K product plus its reduction
+        const bool gemv = gemv_bf16_ok(B, K1) && gemv_bf16_ok(B, Hd);
         for (int j = 1; j < n; ++j) {
-          { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run(g1, s)); }
-          { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_splitk_finish(mpart, g1.a.total_splits, B, Hd, nullptr, ACT_GELU, nullptr, 0,
-                                         static_cast<uint16_t*>(h1), Hd, s)); }
-          if (head->n_layers == 2) {
-            { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run(g2, s)); }
-            { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_splitk_finish(mpart, g2.a.total_splits, B, Hd, nullptr, ACT_GELU, nullptr, 0,
-                                           static_cast<uint16_t*>(h2), Hd, s)); }
+          if (gemv) {
+            { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(launch_gemv_bf16(static_cast<const uint16_t*>(u), K1,
+                                             static_cast<const uint16_t*>(head->w[0]), B, Hd, K1, ACT_GELU,
+                                             static_cast<uint16_t*>(h1), Hd, s)); }
+            if (head->n_layers == 2)
+              { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(launch_gemv_bf16(static_cast<const uint16_t*>(h1), Hd,
+                                               static_cast<const uint16_t*>(head->w[1]), B, Hd, Hd, ACT_GELU,
+                                               static_cast<uint16_t*>(h2), Hd, s)); }
+          } else {
+            { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run(g1, s)); }
+            { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_splitk_finish(mpart, g1.a.total_splits, B, Hd, nullptr, ACT_GELU, nullptr, 0,
+                                           static_cast<uint16_t*>(h1), Hd, s)); }
+            if (head->n_layers == 2) {
+              { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run(g2, s)); }
+              { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_splitk_finish(mpart, g2.a.total_splits, B, Hd, nullptr, ACT_GELU, nullptr, 0,
+                                             static_cast<uint16_t*>(h2), Hd, s)); }
+            }
           }
           gv.a.j = j;
           gv.a.sample = sm.on;

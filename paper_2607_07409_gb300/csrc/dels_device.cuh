@@ -174,6 +174,51 @@ __device__ __forceinline__ void write_decode(const RowAcc& r, long long out_i, i
 }
 
 // ----------------------------------------------------------------------------
+// bf16 activations of the heads' products, block sums
+// ----------------------------------------------------------------------------
+__device__ __forceinline__ float bf16_to_f(uint16_t u) { return __uint_as_float((uint32_t)u << 16); }
+
+// Stores v for a bf16 product. terms = 1: v rounded to bf16 (nearest even)
+// at row b of an [B, ld] buffer. terms = 3: the three-term expansion
+// v = hi + mid + lo, each term the bf16 rounding of what the terms before it
+// left (every difference is exact in float32, and the three terms hold all
+// 24 significand bits of v), at rows b, B + b and 2B + b of a [3B, ld]
+// buffer; a bf16 product over the three rows, accumulated in float32, then
+// equals the product of the float32 activation.
+__device__ __forceinline__ void store_bf16_terms(uint16_t* out, int terms, int B, int b, long long ld, long long o,
+                                                 float v) {
+  const uint16_t hi = f32_to_bf16_rne(v);
+  out[(long long)b * ld + o] = hi;
+  if (terms == 3) {
+    const float r1 = v - bf16_to_f(hi);
+    const uint16_t mid = f32_to_bf16_rne(r1);
+    const float r2 = r1 - bf16_to_f(mid);
+    out[(long long)(B + b) * ld + o] = mid;
+    out[(long long)(2 * B + b) * ld + o] = f32_to_bf16_rne(r2);
+  }
+}
+
+// Sum of v over the CTA (every thread gets the result).
+__device__ __forceinline__ float block_sum(float v) {
+  __shared__ float red[32];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int d = 16; d > 0; d >>= 1) v += __shfl_down_sync(0xFFFFFFFFu, v, d);
+  __syncthreads();
+  if (lane == 0) red[warp] = v;
+  __syncthreads();
+  const int nw = (blockDim.x + 31) >> 5;
+  v = (threadIdx.x < nw) ? red[threadIdx.x] : 0.f;
+  if (warp == 0) {
+#pragma unroll
+    for (int d = 16; d > 0; d >>= 1) v += __shfl_down_sync(0xFFFFFFFFu, v, d);
+    if (lane == 0) red[0] = v;
+  }
+  __syncthreads();
+  return red[0];
+}
+
+// ----------------------------------------------------------------------------
 // temperature 1: Gumbel-max draws with Philox4x32-10 uniforms
 // ----------------------------------------------------------------------------
 // Philox4x32-10 (Salmon, Moraes, Dror and Shaw, "Parallel random numbers: as

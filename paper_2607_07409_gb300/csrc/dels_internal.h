@@ -351,6 +351,14 @@ cudaError_t launch_attention(const float* q, const float* kcache, const float* v
                              int npos, int cache_ld_pos, uint16_t* o_bf16, cudaStream_t s, int terms = 1);
 cudaError_t launch_gemv_f32(const float* X, int ldx, const float* W, int B, int O, int K, int act, float* Y,
                             int ldy, cudaStream_t s);
+// bf16 weights and activations, bf16 output after the activation, B <= kGemvBf16MaxRows.
+constexpr int kGemvBf16MaxRows = 4;
+// the X rows are staged in (at most 48 KB of) shared memory
+inline bool gemv_bf16_ok(int B, int K) {
+  return B >= 1 && B <= kGemvBf16MaxRows && K % 8 == 0 && (long long)B * K * 2 <= 48 * 1024;
+}
+cudaError_t launch_gemv_bf16(const uint16_t* X, int ldx, const uint16_t* W, int B, int O, int K, int act,
+                             uint16_t* Y, int ldy, cudaStream_t s);
 cudaError_t launch_vocab_combine_f32(const float* feat, int K, const float* Wv, const void* longp, int long_f32,
                                      long long ld_long, const float* prior, float alpha, float beta, int B,
                                      int V, void* partials, int partial_ld, int nchunks, int* status,

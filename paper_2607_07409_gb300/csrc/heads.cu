@@ -20,28 +20,6 @@ __device__ __forceinline__ float act_f(int act, float x) {
   return x;
 }
 
-__device__ __forceinline__ float bf16_to_f(uint16_t u) { return __uint_as_float((uint32_t)u << 16); }
-
-// Stores v for a bf16 product. terms = 1: v rounded to bf16 (nearest even)
-// at row b of an [B, ld] buffer. terms = 3: the three-term expansion
-// v = hi + mid + lo, each term the bf16 rounding of what the terms before it
-// left (every difference is exact in float32, and the three terms hold all
-// 24 significand bits of v), at rows b, B + b and 2B + b of a [3B, ld]
-// buffer; a bf16 product over the three rows, accumulated in float32, then
-// equals the product of the float32 activation.
-__device__ __forceinline__ void store_bf16_terms(uint16_t* out, int terms, int B, int b, long long ld, long long o,
-                                                 float v) {
-  const uint16_t hi = f32_to_bf16_rne(v);
-  out[(long long)b * ld + o] = hi;
-  if (terms == 3) {
-    const float r1 = v - bf16_to_f(hi);
-    const uint16_t mid = f32_to_bf16_rne(r1);
-    const float r2 = r1 - bf16_to_f(mid);
-    out[(long long)(B + b) * ld + o] = mid;
-    out[(long long)(2 * B + b) * ld + o] = f32_to_bf16_rne(r2);
-  }
-}
-
 // GRU gates (PyTorch bias-free form; gate rows r, z, n):
 //   gi = sum of the S0 input-product partials, gh = sum of the S1 recurrent ones
 //   r = sigmoid(gi_r + gh_r), z = sigmoid(gi_z + gh_z)
@@ -181,6 +159,32 @@ __global__ void __launch_bounds__(kGatesThreads) k_gru_gates_table(GatesTableArg
   a.h_bf16[e] = f32_to_bf16_rne(hn);
 }
 
+// sum_s sum_t part[s * split_stride + t * total + e] over S splits and
+// in_terms terms (terms last to first within a split), eight loads in flight
+// before they are added in that order.
+__device__ __forceinline__ float splitk_sum(const float* __restrict__ part, int S, int in_terms, long long total,
+                                           long long e) {
+  const long long split_stride = total * in_terms;
+  const int n = S * in_terms;
+  float acc = 0.f;
+  int s = 0, t = in_terms - 1;
+  for (int k0 = 0; k0 < n; k0 += 8) {
+    float v[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      v[k] = k0 + k < n ? part[s * split_stride + t * total + e] : 0.f;
+      if (--t < 0) {
+        t = in_terms - 1;
+        ++s;
+      }
+    }
+#pragma unroll
+    for (int k = 0; k < 8; ++k)
+      if (k0 + k < n) acc += v[k];
+  }
+  return acc;
+}
+
 // out[b, o] = act(sum_s sum_t part[s, t*B + b, o] (+ residual[b, o])):
 // partials [S][in_terms*B][O] (in_terms = 3 when the product's input rows were
 // a three-term expansion), the residual dense [B, O]; the f32 output has its
@@ -208,8 +212,7 @@ __global__ void k_splitk_finish(const float* __restrict__ part, int S, int B, in
           if (s0 + k < S) acc += v[k];
       }
     } else {
-      for (int s = 0; s < S; ++s)
-        for (int t = in_terms - 1; t >= 0; --t) acc += part[s * split_stride + t * total + e];
+      acc = splitk_sum(part, S, in_terms, total, e);
     }
     if (residual) acc += residual[e];
     acc = act_f(act, acc);
@@ -227,34 +230,11 @@ __global__ void k_splitk_finish3(SplitkJobs3 jobs, int B, int O, int in_terms) {
   pdl_wait();
   const SplitkJob& jb = jobs.j[blockIdx.y];
   const long long total = (long long)B * O;
-  const long long split_stride = total * in_terms;
   for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < total;
        e += (long long)gridDim.x * blockDim.x) {
     const int b = (int)(e / O), o = (int)(e % O);
-    float acc = 0.f;
-    for (int s = 0; s < jb.S; ++s)
-      for (int t = in_terms - 1; t >= 0; --t) acc += jb.part[s * split_stride + t * total + e];
-    jb.out[(long long)b * jb.ld + o] = acc;
+    jb.out[(long long)b * jb.ld + o] = splitk_sum(jb.part, jb.S, in_terms, total, e);
   }
-}
-
-__device__ __forceinline__ float block_sum(float v) {
-  __shared__ float red[32];
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-#pragma unroll
-  for (int d = 16; d > 0; d >>= 1) v += __shfl_down_sync(0xFFFFFFFFu, v, d);
-  __syncthreads();
-  if (lane == 0) red[warp] = v;
-  __syncthreads();
-  const int nw = (blockDim.x + 31) >> 5;
-  v = (threadIdx.x < nw) ? red[threadIdx.x] : 0.f;
-  if (warp == 0) {
-#pragma unroll
-    for (int d = 16; d > 0; d >>= 1) v += __shfl_down_sync(0xFFFFFFFFu, v, d);
-    if (lane == 0) red[0] = v;
-  }
-  __syncthreads();
-  return red[0];
 }
 
 // out = RMSNorm(x) = x / sqrt(mean(x^2) + 1e-6) as `terms` bf16 terms (rows
@@ -290,7 +270,6 @@ __global__ void k_finish_rmsnorm(const float* __restrict__ part, int S, int in_t
   const int per = (D + kNormCluster - 1) / kNormCluster;
   const int o0 = (int)rank * per, o1 = min(D, o0 + per);
   const long long total = (long long)B * D;
-  const long long split_stride = total * in_terms;
   constexpr int kMaxPer = 4;     // row elements per thread (D <= kNormCluster * 4 * blockDim.x)
   float v[kMaxPer];
   float ss = 0.f;
@@ -300,9 +279,7 @@ __global__ void k_finish_rmsnorm(const float* __restrict__ part, int S, int in_t
     v[k] = 0.f;
     if (o < o1) {
       const long long e = (long long)b * D + o;
-      float acc = 0.f;
-      for (int s = 0; s < S; ++s)
-        for (int t = in_terms - 1; t >= 0; --t) acc += part[s * split_stride + t * total + e];
+      float acc = splitk_sum(part, S, in_terms, total, e);
       if (residual) acc += residual[e];
       out_f32[e] = acc;
       v[k] = acc;
@@ -389,6 +366,80 @@ __global__ void k_attention(const float* __restrict__ q, const float* __restrict
     float o = 0.f;
     for (int p = 0; p < npos; ++p) o += w[p] * vc[((long long)b * cache_ld_pos + p) * D + hd * dh + i];
     store_bf16_terms(o_bf16, terms, B, b, D, hd * dh + i, o);
+  }
+}
+
+// bf16 skinny product on CUDA cores for a few rows, with the activation and
+// the bf16 rounding of the output fused: Y[b, o] = bf16(act(sum_k X[b, k]
+// W[o, k])) for B <= BMAX, float32 accumulation. One warp per output row o;
+// each lane keeps up to 16 weight loads of 16 bytes (8 values) in flight, the
+// first ones issued before waiting for the predecessor (the weights are not
+// its output); the X rows are staged in shared memory once per CTA. K is a
+// multiple of 8 and the rows are 16-byte aligned.
+template <int BMAX>
+__global__ void k_gemv_bf16(const uint16_t* __restrict__ X, int ldx, const uint16_t* __restrict__ W, int B, int O,
+                            int K, int act, uint16_t* __restrict__ Y, int ldy) {
+  extern __shared__ __align__(16) uint16_t sx[];   // [B][K]
+  constexpr int U = 16;   // weight vectors per lane in flight
+  if (threadIdx.x == 0) pdl_trigger();
+  const int lane = threadIdx.x & 31;
+  const int o = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  const bool live = o < O;
+  const int nv = K / 8;
+  const uint4* w = reinterpret_cast<const uint4*>(W + (long long)(live ? o : 0) * K);
+  uint4 wv[U];
+#pragma unroll
+  for (int u = 0; u < U; ++u) {
+    const int v = lane + u * 32;
+    wv[u] = (live && v < nv) ? __ldg(w + v) : make_uint4(0, 0, 0, 0);
+  }
+  pdl_wait();
+  uint4* sx4 = reinterpret_cast<uint4*>(sx);
+  for (int i = threadIdx.x; i < B * nv; i += blockDim.x) {
+    const int b = i / nv, v = i - b * nv;
+    sx4[i] = __ldg(reinterpret_cast<const uint4*>(X + (long long)b * ldx) + v);
+  }
+  __syncthreads();
+  if (!live) return;
+  float acc[BMAX];
+#pragma unroll
+  for (int i = 0; i < BMAX; ++i) acc[i] = 0.f;
+  for (int v0 = 0; v0 < nv; v0 += 32 * U) {
+    if (v0 > 0) {
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const int v = v0 + lane + u * 32;
+        wv[u] = v < nv ? __ldg(w + v) : make_uint4(0, 0, 0, 0);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int v = v0 + lane + u * 32;
+      if (v >= nv) continue;
+      const float w8[8] = {bf16lo(wv[u].x), bf16hi(wv[u].x), bf16lo(wv[u].y), bf16hi(wv[u].y),
+                           bf16lo(wv[u].z), bf16hi(wv[u].z), bf16lo(wv[u].w), bf16hi(wv[u].w)};
+#pragma unroll
+      for (int i = 0; i < BMAX; ++i) {
+        if (i < B) {
+          const uint4 xv = sx4[i * nv + v];
+          acc[i] = fmaf(w8[0], bf16lo(xv.x), acc[i]);
+          acc[i] = fmaf(w8[1], bf16hi(xv.x), acc[i]);
+          acc[i] = fmaf(w8[2], bf16lo(xv.y), acc[i]);
+          acc[i] = fmaf(w8[3], bf16hi(xv.y), acc[i]);
+          acc[i] = fmaf(w8[4], bf16lo(xv.z), acc[i]);
+          acc[i] = fmaf(w8[5], bf16hi(xv.z), acc[i]);
+          acc[i] = fmaf(w8[6], bf16lo(xv.w), acc[i]);
+          acc[i] = fmaf(w8[7], bf16hi(xv.w), acc[i]);
+        }
+      }
+    }
+  }
+#pragma unroll
+  for (int i = 0; i < BMAX; ++i) {
+    float v = acc[i];
+#pragma unroll
+    for (int d = 16; d > 0; d >>= 1) v += __shfl_down_sync(0xFFFFFFFFu, v, d);
+    if (lane == 0 && i < B) Y[(long long)i * ldy + o] = f32_to_bf16_rne(act_f(act, v));
   }
 }
 
@@ -524,6 +575,14 @@ cudaError_t launch_attention(const float* q, const float* kcache, const float* v
                              int npos, int cache_ld_pos, uint16_t* o_bf16, cudaStream_t s, int terms) {
   return launch_pdl(k_attention, dim3(B * nh), dim3(128), 0, s, q, kcache, vcache, D, nh, npos, cache_ld_pos, o_bf16,
                     terms, B);
+}
+
+cudaError_t launch_gemv_bf16(const uint16_t* X, int ldx, const uint16_t* W, int B, int O, int K, int act,
+                             uint16_t* Y, int ldy, cudaStream_t s) {
+  if (!gemv_bf16_ok(B, K)) return cudaErrorInvalidValue;
+  const int warps = 4;
+  return launch_pdl(k_gemv_bf16<kGemvBf16MaxRows>, dim3((O + warps - 1) / warps), dim3(warps * 32),
+                    (size_t)B * K * 2, s, X, ldx, W, B, O, K, act, Y, ldy);
 }
 
 cudaError_t launch_gemv_f32(const float* X, int ldx, const float* W, int B, int O, int K, int act, float* Y, int ldy,

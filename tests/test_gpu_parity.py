@@ -203,6 +203,9 @@ SMALL = {
                                 head_d_model=512, head_d_hidden=256, head_d_rank=256),
     "mlp2": synth.with_sizes(synth.WORKLOADS["qwen3_0p6b"], B=3, n=6, V=2000,
                              head_d_model=128, head_d_hidden=192, head_d_rank=192),
+    # more requests than the CUDA-core path takes: tensor-core products + reductions
+    "mlp2_b9": synth.with_sizes(synth.WORKLOADS["qwen3_0p6b"], B=9, n=5, V=2000,
+                                head_d_model=128, head_d_hidden=192, head_d_rank=192),
     "xfmr": synth.with_sizes(synth.WORKLOADS["qwen3_4b"], B=2, n=5, V=1536,
                              head_d_model=256, head_d_hidden=512, head_d_rank=256, head_n_heads=4,
                              head_max_pos=8),
