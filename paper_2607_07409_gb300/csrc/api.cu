@@ -235,6 +235,28 @@ bool plan_store(Gemm& g, int B, int O, const void* X0, const void* W0, int K0, c
   return true;
 }
 
+// Splits for `tiles` output tiles when the items (tiles x splits) may take
+// more than one wave: the split count with the shortest makespan in item
+// time, ceil(tiles s / sms) / s, plus 2 % per split for the partials written
+// and re-read (80 tiles on 152 SMs: 5 splits, 0.6 of one tile's time, where
+// one split left 72 SMs idle).
+int splits_balanced(int O, int n_tile, int K, int sms) {
+  const int tiles = (O + n_tile - 1) / n_tile;
+  const int nch = (K + 63) / 64;
+  const int smax = std::min(nch, 32);
+  int best = 1;
+  double best_cost = 1e30;
+  for (int sp = 1; sp <= smax; ++sp) {
+    const long long waves = ((long long)tiles * sp + sms - 1) / std::max(1, sms);
+    const double cost = (double)waves / sp + 0.02 * sp;
+    if (cost < best_cost - 1e-9) {
+      best_cost = cost;
+      best = sp;
+    }
+  }
+  return best;
+}
+
 // Splits so that tiles x splits roughly fills the GPU once.
 int splits_for(int O, int n_tile, int K, int sms) {
   const int tiles = (O + n_tile - 1) / n_tile;
@@ -458,10 +480,10 @@ DraftLayout draft_layout(const dels_local_head* hd, int B, int n, int V) {
       L.q = c.take((size_t)B * D * 4);
       L.kc = c.take((size_t)B * P * D * 4);
       L.vc = c.take((size_t)B * P * D * 4);
-      L.xs_qkv = splits_for(D, 128, D, sms);
-      L.xs_o = splits_for(D, 128, D, sms);
-      L.xs_1 = splits_for(F, 128, D, sms);
-      L.xs_2 = splits_for(D, 128, F, sms);
+      L.xs_qkv = splits_balanced(D, 128, D, sms);
+      L.xs_o = splits_balanced(D, 128, D, sms);
+      L.xs_1 = splits_balanced(F, 128, D, sms);
+      L.xs_2 = splits_balanced(D, 128, F, sms);
       const int smax = std::max(std::max(L.xs_qkv, L.xs_o), std::max(L.xs_1, L.xs_2));
       L.xpart = c.take((size_t)smax * T * B * std::max(D, F) * 4);
       // the k and v products of a position have their own partials, so that
@@ -515,6 +537,7 @@ int validate_head(const dels_local_head* h, int n) {
         if (!h->w[i]) return DELS_ERR_NULL_POINTER;
       if (!dim_ok(h->d_model) || !dim_ok(h->d_hidden) || h->d_rank != h->d_model) return DELS_ERR_BAD_SHAPE;
       if (h->n_heads < 1 || h->d_model % h->n_heads != 0 || h->max_pos < n) return DELS_ERR_BAD_SHAPE;
+      if (h->d_model / h->n_heads > 8192) return DELS_ERR_UNSUPPORTED;   // q of one head in shared memory
       return DELS_OK;
     case DELS_HEAD_MARKOV:
       if (!dim_ok(h->d_rank)) return DELS_ERR_BAD_SHAPE;

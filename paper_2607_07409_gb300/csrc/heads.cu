@@ -321,37 +321,64 @@ __global__ void k_xfmr_embed(const uint16_t* __restrict__ e_rows, const uint16_t
   if (threadIdx.x == 0) pdl_trigger();
   pdl_wait();
   const long long off = (long long)blockIdx.x * D;
+  const int nv = D / 8;   // 8-value vectors (D is a multiple of 16)
+  const uint4* e4 = reinterpret_cast<const uint4*>(e_rows + off);
+  const uint4* p4 = reinterpret_cast<const uint4*>(pos_table + (long long)pos * D);
+  float4* t4 = reinterpret_cast<float4*>(t_out + off);
   float ss = 0.f;
-  for (int i = threadIdx.x; i < D; i += blockDim.x) {
-    const float t = bf16_to_f(e_rows[off + i]) + bf16_to_f(pos_table[(long long)pos * D + i]);
-    t_out[off + i] = t;
-    ss += t * t;
+  for (int v = threadIdx.x; v < nv; v += blockDim.x) {
+    const uint4 e = e4[v], pp = __ldg(p4 + v);
+    const float4 a = make_float4(bf16lo(e.x) + bf16lo(pp.x), bf16hi(e.x) + bf16hi(pp.x),
+                                 bf16lo(e.y) + bf16lo(pp.y), bf16hi(e.y) + bf16hi(pp.y));
+    const float4 c = make_float4(bf16lo(e.z) + bf16lo(pp.z), bf16hi(e.z) + bf16hi(pp.z),
+                                 bf16lo(e.w) + bf16lo(pp.w), bf16hi(e.w) + bf16hi(pp.w));
+    t4[2 * v] = a;
+    t4[2 * v + 1] = c;
+    ss += a.x * a.x + a.y * a.y + a.z * a.z + a.w * a.w + c.x * c.x + c.y * c.y + c.z * c.z + c.w * c.w;
   }
-  ss = block_sum(ss);
+  ss = block_sum(ss);   // also orders this CTA's t writes before the reads below
   const float inv = rsqrtf(ss / (float)D + 1e-6f);
-  for (int i = threadIdx.x; i < D; i += blockDim.x)
-    store_bf16_terms(a_bf16, terms, B, blockIdx.x, D, i, t_out[off + i] * inv);
+  for (int v = threadIdx.x; v < nv; v += blockDim.x) {
+    const float4 a = t4[2 * v], c = t4[2 * v + 1];
+    const float t8[8] = {a.x, a.y, a.z, a.w, c.x, c.y, c.z, c.w};
+#pragma unroll
+    for (int i = 0; i < 8; ++i) store_bf16_terms(a_bf16, terms, B, blockIdx.x, D, 8 * v + i, t8[i] * inv);
+  }
 }
 
 // Causal attention of the newest position over positions 0..npos-1 of the
 // block: one CTA per (row, head); o = softmax(q k^T / sqrt(dh)) v, stored as
-// `terms` bf16 terms.
+// `terms` bf16 terms. q is staged in shared memory; one warp per position
+// computes a score with four loads of the key in flight; each output element
+// sums over the positions four values at a time.
 __global__ void k_attention(const float* __restrict__ q, const float* __restrict__ kc, const float* __restrict__ vc,
                             int D, int nh, int npos, int cache_ld_pos, uint16_t* __restrict__ o_bf16, int terms,
                             int B) {
+  extern __shared__ float sq[];   // dh
+  __shared__ float w[64];
   if (threadIdx.x == 0) pdl_trigger();
   pdl_wait();
   const int b = blockIdx.x / nh, hd = blockIdx.x % nh;
   const int dh = D / nh;
-  __shared__ float w[64];
-  const float* qv = q + (long long)b * D + hd * dh;
   const float scale = rsqrtf((float)dh);
-  for (int p = 0; p < npos; ++p) {
+  for (int i = threadIdx.x; i < dh; i += blockDim.x) sq[i] = q[(long long)b * D + hd * dh + i];
+  __syncthreads();
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  for (int p = warp; p < npos; p += nw) {
     const float* kv = kc + ((long long)b * cache_ld_pos + p) * D + hd * dh;
-    float d = 0.f;
-    for (int i = threadIdx.x; i < dh; i += blockDim.x) d += qv[i] * kv[i];
-    d = block_sum(d);
-    if (threadIdx.x == 0) w[p] = d * scale;
+    float d[4] = {0.f, 0.f, 0.f, 0.f};
+    for (int i0 = lane; i0 < dh; i0 += 128) {
+      float k4[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) k4[u] = i0 + 32 * u < dh ? kv[i0 + 32 * u] : 0.f;
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+        if (i0 + 32 * u < dh) d[u] = fmaf(sq[i0 + 32 * u], k4[u], d[u]);
+    }
+    float dd = (d[0] + d[1]) + (d[2] + d[3]);
+#pragma unroll
+    for (int k = 16; k > 0; k >>= 1) dd += __shfl_down_sync(0xFFFFFFFFu, dd, k);
+    if (lane == 0) w[p] = dd * scale;
   }
   __syncthreads();
   if (threadIdx.x == 0) {
@@ -362,10 +389,19 @@ __global__ void k_attention(const float* __restrict__ q, const float* __restrict
     for (int p = 0; p < npos; ++p) w[p] /= s;
   }
   __syncthreads();
+  const long long row0 = (long long)b * cache_ld_pos * D + hd * dh;
   for (int i = threadIdx.x; i < dh; i += blockDim.x) {
-    float o = 0.f;
-    for (int p = 0; p < npos; ++p) o += w[p] * vc[((long long)b * cache_ld_pos + p) * D + hd * dh + i];
-    store_bf16_terms(o_bf16, terms, B, b, D, hd * dh + i, o);
+    float o[4] = {0.f, 0.f, 0.f, 0.f};
+    int p = 0;
+    for (; p + 4 <= npos; p += 4) {
+      float v4[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) v4[u] = vc[row0 + (long long)(p + u) * D + i];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) o[u] = fmaf(w[p + u], v4[u], o[u]);
+    }
+    for (; p < npos; ++p) o[0] = fmaf(w[p], vc[row0 + (long long)p * D + i], o[0]);
+    store_bf16_terms(o_bf16, terms, B, b, D, hd * dh + i, (o[0] + o[1]) + (o[2] + o[3]));
   }
 }
 
@@ -568,13 +604,16 @@ cudaError_t launch_rmsnorm_bf16(const float* x, int B, int D, int ld, uint16_t* 
 
 cudaError_t launch_xfmr_embed(const uint16_t* e_rows, const uint16_t* pos_table, int pos, int B, int D,
                               float* t_out, uint16_t* a_bf16, cudaStream_t s, int terms) {
+  if (D % 8 != 0) return cudaErrorInvalidValue;
   return launch_pdl(k_xfmr_embed, dim3(B), dim3(256), 0, s, e_rows, pos_table, pos, D, t_out, a_bf16, terms, B);
 }
 
 cudaError_t launch_attention(const float* q, const float* kcache, const float* vcache, int B, int D, int nh,
                              int npos, int cache_ld_pos, uint16_t* o_bf16, cudaStream_t s, int terms) {
-  return launch_pdl(k_attention, dim3(B * nh), dim3(128), 0, s, q, kcache, vcache, D, nh, npos, cache_ld_pos, o_bf16,
-                    terms, B);
+  if (npos < 1 || npos > 64) return cudaErrorInvalidValue;
+  const int dh = D / nh;
+  return launch_pdl(k_attention, dim3(B * nh), dim3(256), (size_t)dh * 4, s, q, kcache, vcache, D, nh, npos,
+                    cache_ld_pos, o_bf16, terms, B);
 }
 
 cudaError_t launch_gemv_bf16(const uint16_t* X, int ldx, const uint16_t* W, int B, int O, int K, int act,
