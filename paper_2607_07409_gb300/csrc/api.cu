@@ -420,7 +420,7 @@ struct DraftLayout {
   size_t u = 0, mpart = 0, h1 = 0, h2 = 0;
   int mlp_s1 = 0, mlp_s2 = 0;
   // XFMR
-  size_t ex = 0, t = 0, ab = 0, q = 0, kc = 0, vc = 0, xpart = 0, xpk = 0, xpv = 0, ob = 0, uu = 0, anb = 0, fb = 0,
+  size_t ex = 0, t = 0, ab = 0, q = 0, kc = 0, vc = 0, xpart = 0, wqkv = 0, xpqkv = 0, ob = 0, uu = 0, anb = 0, fb = 0,
          y = 0, feat = 0;
   int xs_qkv = 0, xs_o = 0, xs_1 = 0, xs_2 = 0;
   // MARKOV
@@ -480,16 +480,17 @@ DraftLayout draft_layout(const dels_local_head* hd, int B, int n, int V) {
       L.q = c.take((size_t)B * D * 4);
       L.kc = c.take((size_t)B * P * D * 4);
       L.vc = c.take((size_t)B * P * D * 4);
-      L.xs_qkv = splits_balanced(D, 128, D, sms);
+      L.xs_qkv = splits_balanced(3 * D, 128, D, sms);
       L.xs_o = splits_balanced(D, 128, D, sms);
       L.xs_1 = splits_balanced(F, 128, D, sms);
       L.xs_2 = splits_balanced(D, 128, F, sms);
       const int smax = std::max(std::max(L.xs_qkv, L.xs_o), std::max(L.xs_1, L.xs_2));
       L.xpart = c.take((size_t)smax * T * B * std::max(D, F) * 4);
-      // the k and v products of a position have their own partials, so that
-      // the q, k and v products run back to back before one reduction
-      L.xpk = c.take((size_t)L.xs_qkv * T * B * D * 4);
-      L.xpv = c.take((size_t)L.xs_qkv * T * B * D * 4);
+      // W_q, W_k and W_v stacked as one [3 d_model, d_model] matrix (copied
+      // here unless the caller's three matrices are already contiguous): the
+      // three products of a position are one launch, with their partials
+      L.wqkv = c.take((size_t)3 * D * D * 2);
+      L.xpqkv = c.take((size_t)L.xs_qkv * T * B * 3 * D * 4);
       L.ob = c.take((size_t)T * B * D * 2);
       L.uu = c.take((size_t)B * D * 4);
       L.anb = c.take((size_t)T * B * D * 2);
@@ -1584,8 +1585,16 @@ int draft_block_impl(const dels_local_head* head, const void* long_logits, dels_
       float* kc = at<float>(workspace, L.kc);
       float* vc = at<float>(workspace, L.vc);
       float* xpart = at<float>(workspace, L.xpart);
-      float* xpk = at<float>(workspace, L.xpk);
-      float* xpv = at<float>(workspace, L.xpv);
+      float* xpqkv = at<float>(workspace, L.xpqkv);
+      const uint16_t* wq = static_cast<const uint16_t*>(head->w[1]);
+      const uint16_t* wqkv = wq;
+      const size_t dd = (size_t)D * D;
+      if (static_cast<const uint16_t*>(head->w[2]) != wq + dd || static_cast<const uint16_t*>(head->w[3]) != wq + 2 * dd) {
+        uint16_t* packed = at<uint16_t>(workspace, L.wqkv);
+        for (int k = 0; k < 3; ++k)
+          DELS_CUDA(cudaMemcpyAsync(packed + k * dd, head->w[1 + k], dd * 2, cudaMemcpyDeviceToDevice, s));
+        wqkv = packed;
+      }
       uint16_t* ob = at<uint16_t>(workspace, L.ob);
       float* uu = at<float>(workspace, L.uu);
       uint16_t* anb = at<uint16_t>(workspace, L.anb);
@@ -1598,33 +1607,30 @@ int draft_block_impl(const dels_local_head* head, const void* long_logits, dels_
       r = draft_position0(long_logits, logit_dtype, B, n, V, partials, L.partial_ld, status, mb, sms, s);
       if (r != DELS_OK || n == 1) return r;
       constexpr int T = kXfmrTerms;
-      RowBlocks gq, gk, gvv, go, g1, g2;
+      RowBlocks gqkv, go, g1, g2;
       Gemm gv;
-      bool ok = plan_store_rows(gq, T * B, D, ab, head->w[1], D, L.xs_qkv, xpart, status, sms) &&
-                plan_store_rows(gk, T * B, D, ab, head->w[2], D, L.xs_qkv, xpk, status, sms) &&
-                plan_store_rows(gvv, T * B, D, ab, head->w[3], D, L.xs_qkv, xpv, status, sms) &&
+      bool ok = plan_store_rows(gqkv, T * B, 3 * D, ab, wqkv, D, L.xs_qkv, xpqkv, status, sms) &&
                 plan_store_rows(go, T * B, D, ob, head->w[4], D, L.xs_o, xpart, status, sms) &&
                 plan_store_rows(g1, T * B, F, anb, head->w[5], D, L.xs_1, xpart, status, sms) &&
                 plan_store_rows(g2, T * B, D, fb, head->w[6], F, L.xs_2, xpart, status, sms) &&
                 plan_combine(gv, B, V, n, feat, D, head->w_vocab, long_logits, logit_dtype, log_prior, alpha, beta,
                              partials, L.partial_ld, status, sms);
       if (!ok) return DELS_ERR_CUDA;
-      const int Sq = gq.g[0].a.total_splits, Sk = gk.g[0].a.total_splits, Sv = gvv.g[0].a.total_splits;
+      const int Sqkv = gqkv.g[0].a.total_splits;
       const int So = go.g[0].a.total_splits, S1 = g1.g[0].a.total_splits, S2 = g2.g[0].a.total_splits;
       const uint16_t* pos = static_cast<const uint16_t*>(head->w[0]);
       for (int j = 1; j < n; ++j) {
         const int p = j - 1;   // position of the newest drafted token x_{j-1}
         { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_xfmr_embed(ex, pos, p, B, D, t, ab, s, T)); }
-        { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run_rows(gq, s)); }
-        { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run_rows(gk, s)); }
-        { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run_rows(gvv, s)); }
+        { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run_rows(gqkv, s)); }
         {
+          // q, and the k / v cache rows of position p, from the stacked partials
           SplitkJobs3 jq{};
-          jq.j[0] = SplitkJob{xpart, Sq, q, (long long)D};
-          jq.j[1] = SplitkJob{xpk, Sk, kc + (size_t)p * D, (long long)P * D};
-          jq.j[2] = SplitkJob{xpv, Sv, vc + (size_t)p * D, (long long)P * D};
+          jq.j[0] = SplitkJob{xpqkv, Sqkv, 0, q, (long long)D};
+          jq.j[1] = SplitkJob{xpqkv, Sqkv, D, kc + (size_t)p * D, (long long)P * D};
+          jq.j[2] = SplitkJob{xpqkv, Sqkv, 2 * D, vc + (size_t)p * D, (long long)P * D};
           PROF(DELS_KCLASS_HEAD_MISC);
-          DELS_CUDA(launch_splitk_finish3(jq, 3, B, D, T, s));
+          DELS_CUDA(launch_splitk_finish3(jq, 3, B, D, 3 * D, T, s));
         }
         { PROF(DELS_KCLASS_HEAD_MISC); DELS_CUDA(launch_attention(q, kc, vc, B, D, NH, p + 1, P, ob, s, T)); }
         { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run_rows(go, s)); }

@@ -329,17 +329,21 @@ cudaError_t launch_splitk_finish(const float* part, int S, int B, int O, const f
                                  float* out_f32, int ld_f32, uint16_t* out_bf16, int ld_bf16, cudaStream_t s,
                                  int in_terms = 1, int out_terms = 1);
 cudaError_t launch_rmsnorm_bf16(const float* x, int B, int D, int ld, uint16_t* out, cudaStream_t s, int terms = 1);
-// Up to three split-K reductions (float32 outputs, own row pitches) in one launch.
+// Up to three split-K reductions (float32 outputs, own row pitches) in one
+// launch: job k sums columns col0 .. col0 + O - 1 of partials
+// [S][in_terms * B][ldp].
 struct SplitkJob {
-  const float* part;   // [S][in_terms * B][O]
+  const float* part;
   int S;
+  int col0;
   float* out;          // row b at out + b * ld
   long long ld;
 };
 struct SplitkJobs3 {
   SplitkJob j[3];
 };
-cudaError_t launch_splitk_finish3(const SplitkJobs3& jobs, int njobs, int B, int O, int in_terms, cudaStream_t s);
+cudaError_t launch_splitk_finish3(const SplitkJobs3& jobs, int njobs, int B, int O, int ldp, int in_terms,
+                                  cudaStream_t s);
 // Split-K reduction + residual (out_f32) and RMSNorm of each row as `terms`
 // bf16 terms (norm_bf16, row pitch D); a cluster of kNormCluster CTAs per row.
 constexpr int kNormCluster = 8;

@@ -222,18 +222,21 @@ __global__ void k_splitk_finish(const float* __restrict__ part, int S, int B, in
 }
 
 // Up to three split-K reductions in one launch (blockIdx.y = job): the same
-// sum as k_splitk_finish with in_terms-term partials, no residual, no
-// activation, float32 output with its own row pitch (the transformer head's
-// q, k and v of the newest position).
-__global__ void k_splitk_finish3(SplitkJobs3 jobs, int B, int O, int in_terms) {
+// sum as k_splitk_finish with in_terms-term partials of row pitch ldp (job k
+// reads columns col0 .. col0 + O - 1), no residual, no activation, float32
+// output with its own row pitch (the transformer head's q, k and v of the
+// newest position, from the partials of their stacked product).
+__global__ void k_splitk_finish3(SplitkJobs3 jobs, int B, int O, int ldp, int in_terms) {
   if (threadIdx.x == 0) pdl_trigger();
   pdl_wait();
   const SplitkJob& jb = jobs.j[blockIdx.y];
   const long long total = (long long)B * O;
+  const long long term_stride = (long long)B * ldp;
   for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < total;
        e += (long long)gridDim.x * blockDim.x) {
     const int b = (int)(e / O), o = (int)(e % O);
-    jb.out[(long long)b * jb.ld + o] = splitk_sum(jb.part, jb.S, in_terms, total, e);
+    jb.out[(long long)b * jb.ld + o] =
+        splitk_sum(jb.part, jb.S, in_terms, term_stride, (long long)b * ldp + jb.col0 + o);
   }
 }
 
@@ -583,9 +586,10 @@ cudaError_t launch_splitk_finish(const float* part, int S, int B, int O, const f
                     act, out_f32, ld_f32, out_bf16, ld_bf16, in_terms, out_terms);
 }
 
-cudaError_t launch_splitk_finish3(const SplitkJobs3& jobs, int njobs, int B, int O, int in_terms, cudaStream_t s) {
+cudaError_t launch_splitk_finish3(const SplitkJobs3& jobs, int njobs, int B, int O, int ldp, int in_terms,
+                                  cudaStream_t s) {
   if (njobs < 1 || njobs > 3) return cudaErrorInvalidValue;
-  return launch_pdl(k_splitk_finish3, dim3(grid_for((long long)B * O, 256), njobs), dim3(256), 0, s, jobs, B, O,
+  return launch_pdl(k_splitk_finish3, dim3(grid_for((long long)B * O, 256), njobs), dim3(256), 0, s, jobs, B, O, ldp,
                     in_terms);
 }
 
