@@ -191,8 +191,9 @@ size_t dels_draft_workspace_bytes(const dels_local_head* head, int B, int n, int
  * out_top2_gap [device] [B, n] float32 top-1 minus top-2 fused value; may be NULL.
  * Limits: 1 <= B <= 128, 1 <= n <= 32, 8 <= V < 2^31, V % 8 == 0; bf16 heads
  * need d_model, d_hidden, d_rank multiples of 16 (d_rank <= 4096); the
- * transformer head needs n <= max_pos, d_model % n_heads == 0 and a head
- * width d_model / n_heads <= 8192 (DELS_ERR_UNSUPPORTED otherwise).
+ * transformer head needs n <= max_pos, d_model % n_heads == 0, d_model <=
+ * 32768 and a head width d_model / n_heads <= 8192 (DELS_ERR_UNSUPPORTED
+ * otherwise).
  * B == 0 is a no-op.
  */
 int dels_draft_block(const dels_local_head* head, const void* long_logits, dels_dtype logit_dtype,

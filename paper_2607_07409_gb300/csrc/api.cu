@@ -539,6 +539,7 @@ int validate_head(const dels_local_head* h, int n) {
       if (!dim_ok(h->d_model) || !dim_ok(h->d_hidden) || h->d_rank != h->d_model) return DELS_ERR_BAD_SHAPE;
       if (h->n_heads < 1 || h->d_model % h->n_heads != 0 || h->max_pos < n) return DELS_ERR_BAD_SHAPE;
       if (h->d_model / h->n_heads > 8192) return DELS_ERR_UNSUPPORTED;   // q of one head in shared memory
+      if (h->d_model > 32768) return DELS_ERR_UNSUPPORTED;               // RMSNorm rows: 8 CTAs x 4096 values
       return DELS_OK;
     case DELS_HEAD_MARKOV:
       if (!dim_ok(h->d_rank)) return DELS_ERR_BAD_SHAPE;
