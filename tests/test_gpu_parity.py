@@ -58,9 +58,10 @@ def _combine(long, short, prior, alpha, beta):
     (1, 151936, "bf16", 1.0),
     (33, 5000, "f32", 0.0),
     (3, 1004, "f32", 0.5),         # V = 4 mod 8: element-wise path
-    (5, 16392, "bf16", 0.5),       # streamed rows: the shortest streamed V, rows cut between CTAs
-    (40, 32000, "f32", 0.3),       # streamed rows, f32
-    (150, 20000, "bf16", 1.0),     # streamed rows, about one row per CTA
+    (5, 16392, "bf16", 0.5),       # rows cut between many CTAs
+    (40, 32000, "f32", 0.3),       # one wave of resident CTAs
+    (150, 20000, "bf16", 1.0),     # about one row per CTA
+    (1217, 16000, "bf16", 0.5),    # more rows than one wave: two rows per CTA, an odd last pair
 ])
 def test_combine_matches_oracle(rows, V, dtype, w):
     d = synth.make_combine_inputs(rows, V, dtype, seed=rows * 31 + V, device=DEV)
