@@ -148,6 +148,19 @@ typedef struct {
 size_t dels_selftest_timeout_bytes(void);
 int dels_selftest_timeout(void* workspace, size_t workspace_bytes, dels_stream_t stream);
 
+/* ---- self test of the Gumbel transform ---------------------------------- */
+
+/*
+ * Writes g[i] = the device's Gumbel variate of the 32-bit Philox output word
+ * bits[i]: u = (floor(bits / 2^9) + 1/2) / 2^23, g = -ln(-ln u), computed as
+ * every temperature-1 kernel of the library computes it (a test hook for
+ * its error against the exact transform; the paper has no counterpart).
+ * `bits` [device, n uint32] and `g` [device, n float32], caller-owned.
+ * Asynchronous on `stream`. Returns DELS_OK, DELS_ERR_BAD_SHAPE for n < 0,
+ * DELS_ERR_NULL_POINTER for a missing pointer with n > 0, or DELS_ERR_CUDA.
+ */
+int dels_selftest_gumbel(const uint32_t* bits, float* g, long long n, dels_stream_t stream);
+
 /* ---- GRU input table (head preparation, once per set of weights) -------- */
 
 /*

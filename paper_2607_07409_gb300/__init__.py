@@ -31,7 +31,7 @@ __all__ = [
     "dels_read_status", "dels_prior_from_counts", "dels_status_string", "dels_version",
     "dels_profile_enable", "dels_profile_reset", "dels_profile_read", "KCLASS",
     "dels_gru_input_table_bytes", "dels_gru_build_input_table", "gru_input_table",
-    "dels_selftest_timeout_bytes", "dels_selftest_timeout",
+    "dels_selftest_timeout_bytes", "dels_selftest_timeout", "dels_selftest_gumbel",
     "dels_prior_workspace_bytes", "dels_prior_count", "dels_prior_log", "dels_prior_estimate", "estimate_prior",
     "make_head", "Drafter", "dtype_code",
 ]
@@ -66,6 +66,7 @@ class LocalHead(ctypes.Structure):
 _SIGS = {
     "dels_selftest_timeout_bytes": (_sz, []),
     "dels_selftest_timeout": (_i, [_vp, _sz, _vp]),
+    "dels_selftest_gumbel": (_i, [_vp, _vp, ctypes.c_longlong, _vp]),
     "dels_gru_input_table_bytes": (_sz, [ctypes.POINTER(LocalHead), _i]),
     "dels_gru_build_input_table": (_i, [ctypes.POINTER(LocalHead), _i, _vp, _sz, _vp, _sz, _vp]),
     "dels_draft_workspace_bytes": (_sz, [ctypes.POINTER(LocalHead), _i, _i, _i]),
@@ -191,6 +192,10 @@ def dels_selftest_timeout_bytes() -> int:
 
 def dels_selftest_timeout(workspace, workspace_bytes: int, stream=None) -> int:
     return lib().dels_selftest_timeout(_ptr(workspace), workspace_bytes, _stream(stream))
+
+
+def dels_selftest_gumbel(bits, g, n: int, stream=None) -> int:
+    return lib().dels_selftest_gumbel(_ptr(bits), _ptr(g), n, _stream(stream))
 
 
 def dels_gru_input_table_bytes(head: LocalHead, V: int) -> int:

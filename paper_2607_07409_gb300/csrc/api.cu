@@ -1093,6 +1093,15 @@ int dels_verify_block(const int32_t* draft_tokens, const void* target_logits, de
 
 // ------------------------------------------------------------ self test
 
+int dels_selftest_gumbel(const uint32_t* bits, float* g, long long n, dels_stream_t stream) {
+  if (n < 0) return DELS_ERR_BAD_SHAPE;
+  if (n > 0 && (!bits || !g)) return DELS_ERR_NULL_POINTER;
+  const int sms = device_sm_count();
+  if (sms <= 0) return DELS_ERR_CUDA;
+  DELS_CUDA(launch_selftest_gumbel(bits, g, n, sms, reinterpret_cast<cudaStream_t>(stream)));
+  return DELS_OK;
+}
+
 size_t dels_selftest_timeout_bytes(void) { return kHeaderBytes + 4096; }
 
 int dels_selftest_timeout(void* workspace, size_t workspace_bytes, dels_stream_t stream) {

@@ -131,6 +131,8 @@ struct SampleRowsArgs {
   int partial_ld;
 };
 cudaError_t launch_sample_rows(const SampleRowsArgs& a, bool f32, cudaStream_t s);
+// The Gumbel transform of Philox words, element-wise (test hook).
+cudaError_t launch_selftest_gumbel(const uint32_t* bits, float* g, long long n, int sms, cudaStream_t s);
 
 // Verification of a temperature-1 block by lossless speculative sampling.
 constexpr int kMaxSampledBlock = 32;

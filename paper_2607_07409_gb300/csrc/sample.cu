@@ -11,6 +11,8 @@
 //   drawn from max(0, p_a - q_a) (normalised), and after n acceptances from
 //   p_n. q_a is rebuilt from the drafting's kept state: the fused row
 //   l_L + alpha_a W_vocab r_a - beta_a l_P and its LSE.
+#include <algorithm>
+
 #include "dels_device.cuh"
 
 namespace dels {
@@ -240,7 +242,21 @@ __global__ void __launch_bounds__(256) k_residual_merge(VerifySampledArgs a) {
   }
 }
 
+__global__ void __launch_bounds__(256) k_selftest_gumbel(const uint32_t* __restrict__ bits, float* __restrict__ g,
+                                                        long long n) {
+  const long long stride = (long long)gridDim.x * blockDim.x;
+  for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride)
+    g[i] = gumbel_from_bits(bits[i]);
+}
+
 }  // namespace
+
+cudaError_t launch_selftest_gumbel(const uint32_t* bits, float* g, long long n, int sms, cudaStream_t s) {
+  if (n == 0) return cudaSuccess;
+  const long long blocks = std::min<long long>((n + 255) / 256, (long long)sms * 8);
+  k_selftest_gumbel<<<(unsigned)blocks, 256, 0, s>>>(bits, g, n);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_verify_accept(const VerifySampledArgs& a, cudaStream_t s) {
   return launch_pdl(k_verify_accept, dim3((unsigned)a.B), dim3(256), 0, s, a);

@@ -316,14 +316,10 @@ __device__ __forceinline__ bool mma_run(const Ctx& c, const Phase& p, MmaState& 
 // then top-1/top-2 and the online log-sum-exp. `lrow` is this row's 128-byte
 // line of the logits box holding the chunk, `half` selects the chunk's
 // 64-byte half (bf16) and `ptile` the prior of the chunk's columns.
-// SAMPLE (temperature 1): the top-2 runs over the keys k = f + g, g the
-// drafting-stream Gumbel variates of (row b, position j, column), and the
-// sum over exp(f - k_max) (see write_decode_sampled).
-template <bool SAMPLE = false>
 __device__ __forceinline__ void combine_chunk(const float (&acc)[32], const uint8_t* lrow, int half, int swz,
                                               bool long_f32, const float* ptile, int cbase, int V, float alpha,
                                               float nbeta, float& best, float& second, int& idx, float& m,
-                                              float& ssum, const TcGemmArgs* sa = nullptr, int b = 0) {
+                                              float& ssum) {
   float f[32];
   if (!long_f32) {
 #pragma unroll
@@ -356,29 +352,64 @@ __device__ __forceinline__ void combine_chunk(const float (&acc)[32], const uint
     for (int i = 0; i < 32; ++i)
       if (cbase + i >= V) f[i] = -INFINITY;
   }
-  if (SAMPLE) {
-    // cbase is a multiple of 32: four Philox blocks of 8 columns
 #pragma unroll
-    for (int t = 0; t < 4; ++t) {
-      float g[8];
-      gumbel8(sa->seed, sa->step, b, sa->j, kStreamDraft, (cbase >> 3) + t, g);
-      // keys at or below the runner-up change neither the top-1 nor the top-2
-      float k[8], km = -INFINITY;
-#pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        k[i] = f[t * 8 + i] + g[i];
-        km = fmaxf(km, k[i]);
-      }
-      if (km > second) {
-#pragma unroll
-        for (int i = 0; i < 8; ++i) top2_push(k[i], cbase + t * 8 + i, best, second, idx);
-      }
-    }
-  } else {
-#pragma unroll
-    for (int i = 0; i < 32; ++i) top2_push(f[i], cbase + i, best, second, idx);
-  }
+  for (int i = 0; i < 32; ++i) top2_push(f[i], cbase + i, best, second, idx);
   lse_chunk_ex2<32>(f, best, m, ssum);
+}
+
+// Temperature 1 (Algorithm 1 with Decode = a draw from the softmax, by
+// Gumbel-max): one 32-column chunk, in four groups of 8 columns (one pair
+// of Philox blocks each). The top-2 runs over the keys k = f + g, g the
+// drafting-stream Gumbel variates of (row b, position j, column), and the
+// sum over exp(f - k_max) (see write_decode_sampled). The group loop stays
+// rolled: unrolled, the chunk's code outgrows the instruction cache and
+// the warps stall on instruction fetch.
+__device__ __forceinline__ void sample_chunk(uint32_t taddr, const uint8_t* lrow, int half, int swz, bool long_f32,
+                                             const float* ptile, int cbase, const TcGemmArgs& a, int b, float& best,
+                                             float& second, int& idx, float& m, float& ssum) {
+  const float alpha = a.alpha, nbeta = -a.beta;
+#pragma unroll 1
+  for (int t = 0; t < 4; ++t) {
+    float acc[8], l[8], f[8];
+    tmem_ld_32x32b_x8(taddr + (uint32_t)(t * 8), acc);
+    tmem_ld_wait();
+    if (!long_f32) {
+      // bf16: group t is 16-byte word t of the chunk's 64-byte half
+      const uint4 w = *reinterpret_cast<const uint4*>(lrow + (((half * 4 + t) ^ swz) << 4));
+      l[0] = bf16lo(w.x); l[1] = bf16hi(w.x); l[2] = bf16lo(w.y); l[3] = bf16hi(w.y);
+      l[4] = bf16lo(w.z); l[5] = bf16hi(w.z); l[6] = bf16lo(w.w); l[7] = bf16hi(w.w);
+    } else {
+      // f32: group t is 16-byte words 2t, 2t + 1 of the chunk's line
+      const float4 w0 = *reinterpret_cast<const float4*>(lrow + (((2 * t) ^ swz) << 4));
+      const float4 w1 = *reinterpret_cast<const float4*>(lrow + (((2 * t + 1) ^ swz) << 4));
+      l[0] = w0.x; l[1] = w0.y; l[2] = w0.z; l[3] = w0.w; l[4] = w1.x; l[5] = w1.y; l[6] = w1.z; l[7] = w1.w;
+    }
+    const float4 p0 = *reinterpret_cast<const float4*>(ptile + t * 8);
+    const float4 p1 = *reinterpret_cast<const float4*>(ptile + t * 8 + 4);
+    const float pr[8] = {p0.x, p0.y, p0.z, p0.w, p1.x, p1.y, p1.z, p1.w};
+#pragma unroll
+    for (int i = 0; i < 8; ++i) f[i] = fmaf(nbeta, pr[i], fmaf(alpha, acc[i], l[i]));
+    const int c0 = cbase + t * 8;
+    if (c0 + 8 > a.V) {
+#pragma unroll
+      for (int i = 0; i < 8; ++i)
+        if (c0 + i >= a.V) f[i] = -INFINITY;
+    }
+    float g[8];
+    gumbel8(a.seed, a.step, b, a.j, kStreamDraft, c0 >> 3, g);
+    float k[8], km = -INFINITY;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      k[i] = f[i] + g[i];
+      km = fmaxf(km, k[i]);
+    }
+    // keys at or below the runner-up change neither the top-1 nor the top-2
+    if (km > second) {
+#pragma unroll
+      for (int i = 0; i < 8; ++i) top2_push(k[i], c0 + i, best, second, idx);
+    }
+    lse_chunk_ex2<8>(f, best, m, ssum);
+  }
 }
 
 struct EpiState {
@@ -446,15 +477,25 @@ __device__ __forceinline__ bool epi_run(const Ctx& c, const Phase& p, EpiState& 
       auto run_chunk = [&](const float (&acc)[32], int cc) {
         if (!a.long_f32) {
           // bf16 boxes of 64 columns: chunk cc is half (cc & 1) of box (cc >> 1)
-          combine_chunk<SAMPLE>(acc, lbuf + (cc >> 1) * box_bytes + br * 128, cc & 1, swz, false, ptile + cc * 32,
-                                it.o0 + cc * 32, a.V, alpha, nbeta, best, second, idx, m, ssum, &a, b);
+          combine_chunk(acc, lbuf + (cc >> 1) * box_bytes + br * 128, cc & 1, swz, false, ptile + cc * 32,
+                        it.o0 + cc * 32, a.V, alpha, nbeta, best, second, idx, m, ssum);
         } else {
           // f32 boxes of 32 columns: chunk cc is box cc
-          combine_chunk<SAMPLE>(acc, lbuf + cc * box_bytes + br * 128, 0, swz, true, ptile + cc * 32,
-                                it.o0 + cc * 32, a.V, alpha, nbeta, best, second, idx, m, ssum, &a, b);
+          combine_chunk(acc, lbuf + cc * box_bytes + br * 128, 0, swz, true, ptile + cc * 32,
+                        it.o0 + cc * 32, a.V, alpha, nbeta, best, second, idx, m, ssum);
         }
       };
-      if (c1 < nchunk) {
+      if constexpr (SAMPLE) {
+#pragma unroll 1
+        for (int cc = c0; cc < nchunk; cc += workers) {
+          if (!a.long_f32)
+            sample_chunk(tbase + (uint32_t)(cc * 32), lbuf + (cc >> 1) * box_bytes + br * 128, cc & 1, swz, false,
+                         ptile + cc * 32, it.o0 + cc * 32, a, b, best, second, idx, m, ssum);
+          else
+            sample_chunk(tbase + (uint32_t)(cc * 32), lbuf + cc * box_bytes + br * 128, 0, swz, true,
+                         ptile + cc * 32, it.o0 + cc * 32, a, b, best, second, idx, m, ssum);
+        }
+      } else if (c1 < nchunk) {
         float acc0[32], acc1[32];
         tmem_ld_32x32b_x32(tbase + (uint32_t)(c0 * 32), acc0);
         tmem_ld_32x32b_x32(tbase + (uint32_t)(c1 * 32), acc1);

@@ -159,3 +159,25 @@ def test_sampled_verify_rejection_at_position_zero(name):
     assert np.all(acc == 0) and np.all(bonus != tok[:, 0])
     tol = LP_TOL_F32 if w.head.wdtype == "f32" else LP_TOL_BF16
     print(name, _check_verify(w, d, W, a, b, tok, acc, bonus, bgap, target, seed, step, tol))
+
+
+def test_gumbel_transform_error_over_every_uniform():
+    """The device's g = -ln(-ln u) for every one of the 2^23 uniforms a Philox
+    word can give (u = (2k + 1) 2^-24), against the float64 transform: the
+    largest absolute error stays below 4e-6 (the exponential variate E = -ln u
+    carries a relative error of ~1.5e-6 at most, which g inherits as an
+    absolute error, plus the fast outer logarithm's)."""
+    k = torch.arange(1 << 23, dtype=torch.int64)
+    w = k << 9                                   # the word's top 23 bits select k
+    bits = torch.where(w >= 2 ** 31, w - 2 ** 32, w).to(torch.int32).to(DEV)   # same 32 bits, as int32
+    g = torch.empty(1 << 23, dtype=torch.float32, device=DEV)
+    assert dels.dels_selftest_gumbel(bits, g, 1 << 23) == 0
+    torch.cuda.synchronize()
+    u = (2.0 * np.arange(1 << 23, dtype=np.float64) + 1.0) / 2.0 ** 24
+    exact = -np.log(-np.log(u))
+    err = np.abs(g.cpu().numpy().astype(np.float64) - exact)
+    worst = int(np.argmax(err))
+    print(f"gumbel transform: max |error| {err[worst]:.3g} at u = {u[worst]:.9f}, mean {err.mean():.3g}")
+    assert err[worst] < 4e-6
+    assert dels.dels_selftest_gumbel(bits, g, -1) == dels.DELS_ERR_BAD_SHAPE
+    assert dels.dels_selftest_gumbel(None, g, 1) == dels.DELS_ERR_NULL_POINTER
