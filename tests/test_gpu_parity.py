@@ -62,6 +62,9 @@ def _combine(long, short, prior, alpha, beta):
     (40, 32000, "f32", 0.3),       # one wave of resident CTAs
     (150, 20000, "bf16", 1.0),     # about one row per CTA
     (1217, 16000, "bf16", 0.5),    # more rows than one wave: two rows per CTA, an odd last pair
+    (400, 50000, "bf16", 0.5),     # one wave of whole rows, a third of the slots idle
+    (200, 50000, "f32", 0.0),      # the same at two CTAs per SM, exact ties
+    (1023, 40000, "bf16", 1.0),    # one wave of row pairs, an odd last pair
 ])
 def test_combine_matches_oracle(rows, V, dtype, w):
     d = synth.make_combine_inputs(rows, V, dtype, seed=rows * 31 + V, device=DEV)
@@ -107,6 +110,22 @@ def test_combine_masked_and_nonfinite_rows(V):
     rt, rl, rg = oracle.combine_argmax(long[:1], None, None, 0.0, 0.0)
     assert tok[0] == rt[0] and abs(lp[0] - rl[0]) < 1e-5
     assert tok[1] == -1 and tok[2] == -1 and tok[3] == -1
+
+
+def test_combine_nonfinite_rows_among_many():
+    """A NaN, an all-masked row and an infinite entry among 400 rows each give
+    token -1 and the status flag; the other rows match the oracle."""
+    rows, V = 400, 50000
+    long = torch.randn(rows, V, device=DEV) * 3
+    long[7, 1234] = float("nan")
+    long[8, :] = -float("inf")
+    long[300, V - 1] = float("inf")
+    tok, lp, gap, st = _combine(long, None, None, 0.0, 0.0)
+    assert st & dels.DELS_STATUS_NONFINITE
+    assert tok[7] == -1 and tok[8] == -1 and tok[300] == -1
+    keep = [r for r in range(rows) if r not in (7, 8, 300)]
+    rt, rl, rg = oracle.combine_argmax(long[keep], None, None, 0.0, 0.0)
+    check_rows(tok[keep], lp[keep], gap[keep], rt, rl, rg, exact_ties=True)
 
 
 def test_combine_zero_rows_is_noop():
