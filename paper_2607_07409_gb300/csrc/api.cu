@@ -268,7 +268,7 @@ int splits_for(int O, int n_tile, int K, int sms) {
 // Vocabulary projection fused with the combine (l_L tile of position j).
 bool plan_combine(Gemm& g, int B, int V, int n, const void* X, int K, const void* Wv, const void* longp,
                   dels_dtype ldt, const float* prior, float alpha, float beta, void* partials, int partial_ld,
-                  int* status, int sms) {
+                  int* status, int sms, bool pair_stages) {
   TcGemmArgs& a = g.a;
   const int n_tile = 128;
   a.B = B;
@@ -316,7 +316,21 @@ bool plan_combine(Gemm& g, int B, int V, int n, const void* X, int K, const void
   } else {
     a.stages = pick_stages(a, 128 * 128 + n_tile * 128, l_fixed);
   }
-  if (!map_x(&g.mA0, X, B, K, a.a_box_rows) || !map_w(&g.mB0, Wv, V, K, n_tile)) return false;
+  // Resident activations and an even number of K chunks: each weight stage
+  // holds two consecutive chunks, loaded as one 3-D box (the weight rows'
+  // 256-byte spans in one request; 8B-shaped launch 29.2 -> 26.8 us).
+  if (pair_stages && a.a_resident && a.seg_chunks[0] % 2 == 0) {
+    a.b_chunks = 2;
+    a.stages = std::max(2, a.stages / 2);
+  }
+  if (!map_x(&g.mA0, X, B, K, a.a_box_rows)) return false;
+  if (a.b_chunks == 2) {
+    if (!encode_tmap_3d(&g.mB0, Wv, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, 64, (uint64_t)V, (uint64_t)(K / 64),
+                        (uint64_t)K * 2, 128, 64, (uint32_t)n_tile, 2, CU_TENSOR_MAP_SWIZZLE_128B))
+      return false;
+  } else if (!map_w(&g.mB0, Wv, V, K, n_tile)) {
+    return false;
+  }
   if (!encode_tmap_3d(&g.mL, longp, a.long_f32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16,
                       es, (uint64_t)V, (uint64_t)n, (uint64_t)B, (uint64_t)V * es, (uint64_t)n * V * es,
                       (uint32_t)a.l_box_cols, 1, (uint32_t)a.l_box_rows, CU_TENSOR_MAP_SWIZZLE_128B))
@@ -1236,7 +1250,7 @@ int draft_block_impl(const dels_local_head* head, const void* long_logits, dels_
             !plan_store(gr, B, R, hb, head->w[2], H, nullptr, nullptr, 0, 32, 1, 0, ACT_SILU, nullptr,
                         static_cast<uint16_t*>(rr), R, status, sms) ||
             !plan_combine(gv, B, V, n, rr, R, head->w_vocab, long_logits, logit_dtype, log_prior, alpha, beta,
-                          partials, L.partial_ld, status, sms))
+                          partials, L.partial_ld, status, sms, false))
           return DELS_ERR_CUDA;
         PersistGruArgs P{};
         P.B = B; P.n = n; P.V = V; P.D = D; P.H = H; P.R = R;
@@ -1305,7 +1319,7 @@ int draft_block_impl(const dels_local_head* head, const void* long_logits, dels_
             !plan_store(gh, B, 3 * H, hb, head->w[1], H, nullptr, nullptr, 0, kHhTile, L.hh_splits, 0, ACT_NONE,
                         gpart, nullptr, 0, status, sms) ||
             !plan_combine(gv, B, V, n, rr, R, head->w_vocab, long_logits, logit_dtype, log_prior, alpha, beta,
-                          partials, L.partial_ld, status, sms))
+                          partials, L.partial_ld, status, sms, false))
           return DELS_ERR_CUDA;
         // the rank product's K splits form one cluster per output tile
         gr.a.cluster_k = gr.a.total_splits;
@@ -1386,7 +1400,7 @@ int draft_block_impl(const dels_local_head* head, const void* long_logits, dels_
             !plan_store(gh, B, 3 * H, hb, head->w[1], H, nullptr, nullptr, 0, kHhTile, L.hh_splits, 0, ACT_NONE,
                         gpart, nullptr, 0, status, sms) ||
             !plan_combine(gv, B, V, n, rr, R, head->w_vocab, long_logits, logit_dtype, log_prior, alpha, beta,
-                          partials, L.partial_ld, status, sms))
+                          partials, L.partial_ld, status, sms, true))
           return DELS_ERR_CUDA;
         // The rank product's K splits reduce inside a cluster (one cluster per
         // output tile, no partials in HBM); its SiLU needs the whole sum.
@@ -1458,7 +1472,7 @@ int draft_block_impl(const dels_local_head* head, const void* long_logits, dels_
                         static_cast<uint16_t*>(rr), R, status, sms))
           return DELS_ERR_CUDA;
         if (!plan_combine(gv, B, V, n, rr, R, head->w_vocab, long_logits, logit_dtype, log_prior, alpha, beta,
-                          partials, L.partial_ld, status, sms))
+                          partials, L.partial_ld, status, sms, true))
           return DELS_ERR_CUDA;
         for (int j = 1; j < n; ++j) {
           { PROF(DELS_KCLASS_HEAD_GEMM); DELS_CUDA(run(gg, s)); }
@@ -1526,7 +1540,7 @@ int draft_block_impl(const dels_local_head* head, const void* long_logits, dels_
                         nullptr, 0, status, sms))
           return DELS_ERR_CUDA;
         if (!plan_combine(gv, B, V, n, feat, Hd, head->w_vocab, long_logits, logit_dtype, log_prior, alpha, beta,
-                          partials, L.partial_ld, status, sms))
+                          partials, L.partial_ld, status, sms, true))
           return DELS_ERR_CUDA;
         // a few requests: each layer is one CUDA-core launch (product, GELU and
         // bf16 rounding together) instead of a split-K product plus its reduction
@@ -1624,7 +1638,7 @@ int draft_block_impl(const dels_local_head* head, const void* long_logits, dels_
                 plan_store_rows(g1, T * B, F, anb, head->w[5], D, L.xs_1, xpart, status, sms) &&
                 plan_store_rows(g2, T * B, D, fb, head->w[6], F, L.xs_2, xpart, status, sms) &&
                 plan_combine(gv, B, V, n, feat, D, head->w_vocab, long_logits, logit_dtype, log_prior, alpha, beta,
-                             partials, L.partial_ld, status, sms);
+                             partials, L.partial_ld, status, sms, true);
       if (!ok) return DELS_ERR_CUDA;
       const int Sqkv = gqkv.g[0].a.total_splits;
       const int So = go.g[0].a.total_splits, S1 = g1.g[0].a.total_splits, S2 = g2.g[0].a.total_splits;
@@ -1674,7 +1688,7 @@ int draft_block_impl(const dels_local_head* head, const void* long_logits, dels_
       if (r != DELS_OK || n == 1) return r;
       Gemm gv;
       if (bf && !plan_combine(gv, B, V, n, feat, R, head->w_vocab, long_logits, logit_dtype, log_prior, alpha, beta,
-                              partials, L.partial_ld, status, sms))
+                              partials, L.partial_ld, status, sms, true))
         return DELS_ERR_CUDA;
       const int nch = std::max(1, std::min(L.partial_ld, (V + 255) / 256));
       for (int j = 1; j < n; ++j) {

@@ -7,7 +7,9 @@
 // (both operands K-major). Four roles run it, each on its own thread(s):
 //
 //  * producer (one thread): TMA loads of weight tiles (B operand) and
-//    activation tiles (A operand) into a ring of S stages. Weight tiles do not
+//    activation tiles (A operand) into a ring of S stages (with resident
+//    activations a stage may hold two consecutive K chunks of the weights,
+//    loaded as one 3-D box: b_chunks = 2). Weight tiles do not
 //    depend on anything computed earlier, so `prod_prefetch` issues the next
 //    phase's first weight stages early (their barriers get the weight bytes as
 //    expected transactions; the arrival, with any activation bytes, comes from
@@ -97,7 +99,11 @@ __device__ __forceinline__ Item get_item(const TcGemmArgs& a, int i) {
   it.kb = ls * per;
   it.ke = min(nch, it.kb + per);
   const int len = it.ke - it.kb;
-  it.rot = len > 0 ? ot % len : 0;
+  // two chunks per stage: the rotation keeps pairs of consecutive chunks
+  if (a.b_chunks == 2)
+    it.rot = len >= 2 ? (ot % (len >> 1)) * 2 : 0;
+  else
+    it.rot = len > 0 ? ot % len : 0;
   return it;
 }
 
@@ -148,14 +154,26 @@ struct ProdState {
   int afull_uses = 0;
 };
 
+// Weights of the stage that starts at visit index i of the item: one 2-D box
+// (one K chunk), or one 3-D box of C consecutive K chunks.
+template <int C>
+__device__ __forceinline__ void load_w(const Ctx& c, const Phase& p, const Item& it, int i, int s, uint64_t pol_w) {
+  const CUtensorMap* mB = it.seg ? p.mB1 : p.mB0;
+  if constexpr (C > 1)
+    tma_load_3d(c.sB + s * c.b_stage_bytes, mB, &c.full[s], 0, it.o0, it.chunk(i), pol_w);
+  else
+    tma_load_2d(c.sB + s * c.b_stage_bytes, mB, &c.full[s], it.chunk(i) * kBlockK, it.o0, pol_w);
+}
+
 // Issue the weight tiles of the phase's first stages (up to S) ahead of the
 // activations. Only waits for stages freed by already-issued MMAs.
-__device__ __forceinline__ bool prod_prefetch(const Ctx& c, const Phase& p, ProdState& st, uint64_t pol_w) {
+template <int C>
+__device__ __forceinline__ bool prod_prefetch_c(const Ctx& c, const Phase& p, ProdState& st, uint64_t pol_w) {
   const TcGemmArgs& a = *p.a;
-  const uint32_t b_bytes = (uint32_t)a.n_tile * 128u;
+  const uint32_t b_bytes = (uint32_t)a.n_tile * 128u * (uint32_t)C;
   int f = max(st.fills, st.pre_end);
   int t = 0;
-  int done = f - st.fills;   // already prefetched for this phase
+  int done = f - st.fills;   // stages already prefetched for this phase
   // skip the chunks already prefetched
   Item it = p.count > 0 ? get_item(a, p.first) : Item{0, 0, 0, 0, 0, 0};
   int i = 0;   // chunk index within the item (visit order)
@@ -166,7 +184,7 @@ __device__ __forceinline__ bool prod_prefetch(const Ctx& c, const Phase& p, Prod
       i = 0;
       continue;
     }
-    ++i;
+    i += C;
     --skip;
   }
   while (f - st.fills < c.S && t < p.count) {
@@ -179,19 +197,23 @@ __device__ __forceinline__ bool prod_prefetch(const Ctx& c, const Phase& p, Prod
     const int s = f % c.S;
     if (!mbar_wait(&c.empty[s], ((f / c.S) & 1) ^ 1, c.deadline, c.abort_flag)) return false;
     mbar_expect_tx(&c.full[s], b_bytes);
-    tma_load_2d(c.sB + s * c.b_stage_bytes, it.seg ? p.mB1 : p.mB0, &c.full[s], it.chunk(i) * kBlockK, it.o0, pol_w);
+    load_w<C>(c, p, it, i, s, pol_w);
     ++f;
-    ++i;
+    i += C;
   }
   st.pre_end = f;
   return true;
 }
+__device__ __forceinline__ bool prod_prefetch(const Ctx& c, const Phase& p, ProdState& st, uint64_t pol_w) {
+  return p.a->b_chunks == 2 ? prod_prefetch_c<2>(c, p, st, pol_w) : prod_prefetch_c<1>(c, p, st, pol_w);
+}
 
 // Load the activations (and the remaining weights) of the phase.
-__device__ __forceinline__ bool prod_run(const Ctx& c, const Phase& p, ProdState& st, uint64_t pol_w,
-                                         uint64_t pol_act) {
+template <int C>   // > 1 only with resident activations
+__device__ __forceinline__ bool prod_run_c(const Ctx& c, const Phase& p, ProdState& st, uint64_t pol_w,
+                                           uint64_t pol_act) {
   const TcGemmArgs& a = *p.a;
-  const uint32_t b_bytes = (uint32_t)a.n_tile * 128u;
+  const uint32_t b_bytes = (uint32_t)a.n_tile * 128u * (uint32_t)C;
   const uint32_t a_copy_bytes = (uint32_t)a.a_box_rows * 128u;
   const uint32_t a_bytes = a_copy_bytes * (uint32_t)a.a_copies;
   if (a.a_resident && p.count > 0) {
@@ -209,8 +231,7 @@ __device__ __forceinline__ bool prod_run(const Ctx& c, const Phase& p, ProdState
   for (int t = 0; t < p.count; ++t) {
     const Item it = get_item(a, p.first + t * p.stride);
     const CUtensorMap* mA = it.seg ? p.mA1 : p.mA0;
-    const CUtensorMap* mB = it.seg ? p.mB1 : p.mB0;
-    for (int i = 0; i < it.ke - it.kb; ++i, ++f) {
+    for (int i = 0; i < it.ke - it.kb; i += C, ++f) {
       const int kc = it.chunk(i);
       const int s = f % c.S;
       if (f < st.pre_end) {
@@ -231,12 +252,16 @@ __device__ __forceinline__ bool prod_run(const Ctx& c, const Phase& p, ProdState
       if (!a.a_resident)
         for (int cp = 0; cp < a.a_copies; ++cp)
           tma_load_2d(c.sA + s * c.a_stage_bytes + cp * a_copy_bytes, mA, &c.full[s], kc * kBlockK, 0, pol_act);
-      tma_load_2d(c.sB + s * c.b_stage_bytes, mB, &c.full[s], kc * kBlockK, it.o0, pol_w);
+      load_w<C>(c, p, it, i, s, pol_w);
     }
   }
   st.fills = f;
   st.pre_end = max(st.pre_end, f);
   return true;
+}
+__device__ __forceinline__ bool prod_run(const Ctx& c, const Phase& p, ProdState& st, uint64_t pol_w,
+                                         uint64_t pol_act) {
+  return p.a->b_chunks == 2 ? prod_run_c<2>(c, p, st, pol_w, pol_act) : prod_run_c<1>(c, p, st, pol_w, pol_act);
 }
 
 // ------------------------------------------------------------- logits producer
@@ -276,7 +301,8 @@ struct MmaState {
   int afull_uses = 0;
 };
 
-__device__ __forceinline__ bool mma_run(const Ctx& c, const Phase& p, MmaState& st) {
+template <int C>
+__device__ __forceinline__ bool mma_run_c(const Ctx& c, const Phase& p, MmaState& st) {
   const TcGemmArgs& a = *p.a;
   const uint32_t idesc = idesc_bf16_f32(128, a.n_tile);
   if (a.a_resident && p.count > 0) {
@@ -289,18 +315,21 @@ __device__ __forceinline__ bool mma_run(const Ctx& c, const Phase& p, MmaState& 
     if (!mbar_wait(&c.acce[buf], ((st.tiles >> 1) & 1) ^ 1, c.deadline, c.abort_flag)) return false;
     tc_fence_after();
     const uint32_t d_tmem = c.tmem_base + (uint32_t)(buf * a.n_tile);
-    for (int i = 0; i < it.ke - it.kb; ++i, ++st.fills) {
-      const int kc = it.chunk(i);
+    for (int i = 0; i < it.ke - it.kb; i += C, ++st.fills) {
       const int s = st.fills % c.S;
       if (!mbar_wait(&c.full[s], (st.fills / c.S) & 1, c.deadline, c.abort_flag)) return false;
       tc_fence_after();
-      const uint32_t a_addr =
-          smem_u32(a.a_resident ? c.sA + kc * kATileBytes : c.sA + s * c.a_stage_bytes);
-      const uint32_t b_addr = smem_u32(c.sB + s * c.b_stage_bytes);
 #pragma unroll
-      for (int kk = 0; kk < kBlockK / kUmmaK; ++kk) {
-        tc_mma_f16(d_tmem, smem_desc_sw128(a_addr + kk * kUmmaK * 2), smem_desc_sw128(b_addr + kk * kUmmaK * 2), idesc,
-                   (i > 0 || kk > 0) ? 1u : 0u);
+      for (int cc = 0; cc < C; ++cc) {
+        const int kc = it.chunk(i + cc);
+        const uint32_t a_addr =
+            smem_u32(a.a_resident ? c.sA + kc * kATileBytes : c.sA + s * c.a_stage_bytes);
+        const uint32_t b_addr = smem_u32(c.sB + s * c.b_stage_bytes + cc * a.n_tile * 128);
+#pragma unroll
+        for (int kk = 0; kk < kBlockK / kUmmaK; ++kk) {
+          tc_mma_f16(d_tmem, smem_desc_sw128(a_addr + kk * kUmmaK * 2), smem_desc_sw128(b_addr + kk * kUmmaK * 2),
+                     idesc, (i > 0 || cc > 0 || kk > 0) ? 1u : 0u);
+        }
       }
       tc_commit(&c.empty[s]);
     }
@@ -308,6 +337,9 @@ __device__ __forceinline__ bool mma_run(const Ctx& c, const Phase& p, MmaState& 
     ++st.tiles;
   }
   return true;
+}
+__device__ __forceinline__ bool mma_run(const Ctx& c, const Phase& p, MmaState& st) {
+  return p.a->b_chunks == 2 ? mma_run_c<2>(c, p, st) : mma_run_c<1>(c, p, st);
 }
 
 // ----------------------------------------------------------------- epilogue

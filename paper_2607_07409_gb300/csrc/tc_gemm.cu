@@ -51,7 +51,7 @@ __host__ __device__ inline Smem smem_layout(const TcGemmArgs& a) {
   s.a_off = off;
   off += (uint32_t)a_tiles * kATileBytes;
   s.b_off = off;
-  off += (uint32_t)a.stages * b_tile;
+  off += (uint32_t)a.stages * b_tile * (uint32_t)(a.b_chunks > 1 ? a.b_chunks : 1);
   s.l_off = off;
   off += 2u * l_tile;
   s.p_off = off;
@@ -183,7 +183,7 @@ __global__ void __launch_bounds__(kThreads, MODE != 0 ? 1 : 2)
   c.abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   c.S = a.stages;
   c.a_stage_bytes = kATileBytes;
-  c.b_stage_bytes = (uint32_t)a.n_tile * 128u;
+  c.b_stage_bytes = (uint32_t)a.n_tile * 128u * (uint32_t)(a.b_chunks > 1 ? a.b_chunks : 1);
   c.l_buf_bytes = comb ? (uint32_t)(a.l_boxes * a.l_box_rows * 128) : 0u;
   c.deadline = globaltimer_ns() + budget_ns;
   const uint32_t tmem_cols =
