@@ -20,6 +20,10 @@
 //    DFlash-logit tile of each vocabulary tile, double-buffered.
 //  * epilogue (8 warps): TMEM -> registers; either stores (optionally with an
 //    activation, f32 split partials or bf16) or the fused combine.
+//  * noise (8 warps, temperature-1 combine launches only): the Gumbel
+//    variates of each tile, written to a second pair of TMEM buffers ahead
+//    of the epilogue (they depend on nothing computed earlier), so that the
+//    epilogue's work per element is that of temperature 0 plus one add.
 //
 // Every role keeps running counters across phases so mbarrier parities stay
 // consistent when one CTA runs many phases (the persistent kernel).
@@ -51,6 +55,9 @@ struct Ctx {
   uint64_t* lfull;          // [2]
   uint64_t* lempty;         // [2]
   uint64_t* afull;          // [1] resident activations
+  uint64_t* nfull;          // [2] noise buffers written (temperature-1 launches)
+  uint64_t* nempty;         // [2] noise buffers read
+  uint32_t noise_col;       // TMEM column of noise buffer 0 (buffer 1 follows at n_tile)
   uint32_t tmem_base;
   int S;
   uint32_t a_stage_bytes;   // pitch of the activation stages (>= the rows actually loaded; the MMA
@@ -348,10 +355,11 @@ __device__ __forceinline__ bool mma_run(const Ctx& c, const Phase& p, MmaState& 
 // then top-1/top-2 and the online log-sum-exp. `lrow` is this row's 128-byte
 // line of the logits box holding the chunk, `half` selects the chunk's
 // 64-byte half (bf16) and `ptile` the prior of the chunk's columns.
+template <bool KEYS = false>
 __device__ __forceinline__ void combine_chunk(const float (&acc)[32], const uint8_t* lrow, int half, int swz,
                                               bool long_f32, const float* ptile, int cbase, int V, float alpha,
                                               float nbeta, float& best, float& second, int& idx, float& m,
-                                              float& ssum) {
+                                              float& ssum, const float (&g)[32]) {
   float f[32];
   if (!long_f32) {
 #pragma unroll
@@ -384,70 +392,85 @@ __device__ __forceinline__ void combine_chunk(const float (&acc)[32], const uint
     for (int i = 0; i < 32; ++i)
       if (cbase + i >= V) f[i] = -INFINITY;
   }
-#pragma unroll
-  for (int i = 0; i < 32; ++i) top2_push(f[i], cbase + i, best, second, idx);
-  lse_chunk_ex2<32>(f, best, m, ssum);
-}
-
-// Temperature 1 (Algorithm 1 with Decode = a draw from the softmax, by
-// Gumbel-max): one 32-column chunk, in four groups of 8 columns (one pair
-// of Philox blocks each). The top-2 runs over the keys k = f + g, g the
-// drafting-stream Gumbel variates of (row b, position j, column), and the
-// sum over exp(f - k_max) (see write_decode_sampled). The group loop stays
-// rolled: unrolled, the chunk's code outgrows the instruction cache and
-// the warps stall on instruction fetch.
-__device__ __forceinline__ void sample_chunk(uint32_t taddr, const uint8_t* lrow, int half, int swz, bool long_f32,
-                                             const float* ptile, int cbase, const TcGemmArgs& a, int b, float& best,
-                                             float& second, int& idx, float& m, float& ssum) {
-  const float alpha = a.alpha, nbeta = -a.beta;
-#pragma unroll 1
-  for (int t = 0; t < 4; ++t) {
-    float acc[8], l[8], f[8];
-    tmem_ld_32x32b_x8(taddr + (uint32_t)(t * 8), acc);
-    tmem_ld_wait();
-    if (!long_f32) {
-      // bf16: group t is 16-byte word t of the chunk's 64-byte half
-      const uint4 w = *reinterpret_cast<const uint4*>(lrow + (((half * 4 + t) ^ swz) << 4));
-      l[0] = bf16lo(w.x); l[1] = bf16hi(w.x); l[2] = bf16lo(w.y); l[3] = bf16hi(w.y);
-      l[4] = bf16lo(w.z); l[5] = bf16hi(w.z); l[6] = bf16lo(w.w); l[7] = bf16hi(w.w);
-    } else {
-      // f32: group t is 16-byte words 2t, 2t + 1 of the chunk's line
-      const float4 w0 = *reinterpret_cast<const float4*>(lrow + (((2 * t) ^ swz) << 4));
-      const float4 w1 = *reinterpret_cast<const float4*>(lrow + (((2 * t + 1) ^ swz) << 4));
-      l[0] = w0.x; l[1] = w0.y; l[2] = w0.z; l[3] = w0.w; l[4] = w1.x; l[5] = w1.y; l[6] = w1.z; l[7] = w1.w;
-    }
-    const float4 p0 = *reinterpret_cast<const float4*>(ptile + t * 8);
-    const float4 p1 = *reinterpret_cast<const float4*>(ptile + t * 8 + 4);
-    const float pr[8] = {p0.x, p0.y, p0.z, p0.w, p1.x, p1.y, p1.z, p1.w};
-#pragma unroll
-    for (int i = 0; i < 8; ++i) f[i] = fmaf(nbeta, pr[i], fmaf(alpha, acc[i], l[i]));
-    const int c0 = cbase + t * 8;
-    if (c0 + 8 > a.V) {
-#pragma unroll
-      for (int i = 0; i < 8; ++i)
-        if (c0 + i >= a.V) f[i] = -INFINITY;
-    }
-    float g[8];
-    gumbel8(a.seed, a.step, b, a.j, kStreamDraft, c0 >> 3, g);
-    float k[8], km = -INFINITY;
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      k[i] = f[i] + g[i];
-      km = fmaxf(km, k[i]);
-    }
+  if constexpr (KEYS) {
+    // temperature 1: the top-2 over the keys f + g (g: the Gumbel variates);
     // keys at or below the runner-up change neither the top-1 nor the top-2
-    if (km > second) {
 #pragma unroll
-      for (int i = 0; i < 8; ++i) top2_push(k[i], c0 + i, best, second, idx);
+    for (int t = 0; t < 4; ++t) {
+      float k[8], km = -INFINITY;
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        k[i] = f[t * 8 + i] + g[t * 8 + i];
+        km = fmaxf(km, k[i]);
+      }
+      if (km > second) {
+#pragma unroll
+        for (int i = 0; i < 8; ++i) top2_push(k[i], cbase + t * 8 + i, best, second, idx);
+      }
     }
-    lse_chunk_ex2<8>(f, best, m, ssum);
+  } else {
+#pragma unroll
+    for (int i = 0; i < 32; ++i) top2_push(f[i], cbase + i, best, second, idx);
   }
+  lse_chunk_ex2<32>(f, best, m, ssum);
 }
 
 struct EpiState {
   int tiles = 0;      // accumulator tiles consumed
   int ltiles = 0;     // logits tiles consumed
+  int ntiles = 0;     // noise tiles consumed (temperature 1)
 };
+
+// The epilogue's quadrant / copy / worker mapping of a combine phase (see
+// epi_run): the noise warps write exactly the values the epilogue reads.
+struct EpiMap {
+  int q, qpc, cpy, b, workers, quad_live;
+};
+__device__ __forceinline__ EpiMap epi_map(const TcGemmArgs& a, int warp, int lane) {
+  EpiMap m;
+  m.q = warp & 3;
+  m.qpc = (a.a_box_rows + 31) / 32;
+  m.cpy = m.q / m.qpc;
+  m.b = (m.q % m.qpc) * 32 + lane;
+  m.workers = 2 * a.a_copies;
+  m.quad_live = m.cpy < a.a_copies && ((m.q % m.qpc) * 32) < a.B;
+  return m;
+}
+
+// Noise warp of TMEM lane quadrant warp % 4 (temperature-1 combine phases;
+// two per quadrant, g = 0, 1): for every tile of the phase, the Gumbel
+// variates of the columns that epilogue warp g of the quadrant combines,
+// written to noise buffer (tile & 1) once the epilogue has released it.
+__device__ __forceinline__ bool noise_run(const Ctx& c, const Phase& p, int warp, int lane, int g) {
+  const TcGemmArgs& a = *p.a;
+  const EpiMap mp = epi_map(a, warp, lane);
+  const int nchunk = a.n_tile / 32;
+  for (int t = 0; t < p.count; ++t) {
+    const Item it = get_item(a, p.first + t * p.stride);
+    const int nb = t & 1;
+    if (!mbar_wait(&c.nempty[nb], ((t >> 1) & 1) ^ 1, c.deadline, c.abort_flag)) return false;
+    tc_fence_after();
+    if (mp.quad_live) {
+      const uint32_t base = c.tmem_base + ((uint32_t)(mp.q * 32) << 16) + c.noise_col + (uint32_t)(nb * a.n_tile);
+      {
+#pragma unroll 1
+        for (int cc = mp.cpy * 2 + g; cc < nchunk; cc += mp.workers) {
+#pragma unroll 1
+          for (int grp = 0; grp < 4; ++grp) {
+            float gv[8];
+            gumbel8(a.seed, a.step, mp.b, a.j, kStreamDraft, ((it.o0 + cc * 32) >> 3) + grp, gv);
+            tmem_st_32x32b_x8(base + (uint32_t)(cc * 32 + grp * 8), gv);
+          }
+        }
+      }
+      tmem_st_wait();
+    }
+    tc_fence_before();
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&c.nfull[nb]);
+  }
+  return true;
+}
 
 // Stage the prior of this CTA's vocabulary range for a combine phase
 // (called by the 256 epilogue threads; ends with an epilogue-only barrier).
@@ -502,6 +525,13 @@ __device__ __forceinline__ bool epi_run(const Ctx& c, const Phase& p, EpiState& 
       if (!ok) break;
     }
     const uint32_t tbase = c.tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * a.n_tile);
+    const int nbuf = st.ntiles & 1;
+    if constexpr (SAMPLE) {
+      ok = mbar_wait(&c.nfull[nbuf], (st.ntiles >> 1) & 1, c.deadline, c.abort_flag);
+      if (!ok) break;
+      tc_fence_after();
+    }
+    const uint32_t gbase = c.tmem_base + ((uint32_t)(q * 32) << 16) + c.noise_col + (uint32_t)(nbuf * a.n_tile);
     if (quad_live && comb) {
       const uint8_t* lbuf = c.sL + lbuf_i * c.l_buf_bytes;
       const float* ptile = c.sP + t * a.n_tile;
@@ -510,22 +540,26 @@ __device__ __forceinline__ bool epi_run(const Ctx& c, const Phase& p, EpiState& 
         if (!a.long_f32) {
           // bf16 boxes of 64 columns: chunk cc is half (cc & 1) of box (cc >> 1)
           combine_chunk(acc, lbuf + (cc >> 1) * box_bytes + br * 128, cc & 1, swz, false, ptile + cc * 32,
-                        it.o0 + cc * 32, a.V, alpha, nbeta, best, second, idx, m, ssum);
+                        it.o0 + cc * 32, a.V, alpha, nbeta, best, second, idx, m, ssum, acc);
         } else {
           // f32 boxes of 32 columns: chunk cc is box cc
           combine_chunk(acc, lbuf + cc * box_bytes + br * 128, 0, swz, true, ptile + cc * 32,
-                        it.o0 + cc * 32, a.V, alpha, nbeta, best, second, idx, m, ssum);
+                        it.o0 + cc * 32, a.V, alpha, nbeta, best, second, idx, m, ssum, acc);
         }
       };
       if constexpr (SAMPLE) {
 #pragma unroll 1
         for (int cc = c0; cc < nchunk; cc += workers) {
+          float acc[32], g[32];
+          tmem_ld_32x32b_x32(tbase + (uint32_t)(cc * 32), acc);
+          tmem_ld_32x32b_x32(gbase + (uint32_t)(cc * 32), g);
+          tmem_ld_wait();
           if (!a.long_f32)
-            sample_chunk(tbase + (uint32_t)(cc * 32), lbuf + (cc >> 1) * box_bytes + br * 128, cc & 1, swz, false,
-                         ptile + cc * 32, it.o0 + cc * 32, a, b, best, second, idx, m, ssum);
+            combine_chunk<true>(acc, lbuf + (cc >> 1) * box_bytes + br * 128, cc & 1, swz, false, ptile + cc * 32,
+                                it.o0 + cc * 32, a.V, alpha, nbeta, best, second, idx, m, ssum, g);
           else
-            sample_chunk(tbase + (uint32_t)(cc * 32), lbuf + cc * box_bytes + br * 128, 0, swz, true,
-                         ptile + cc * 32, it.o0 + cc * 32, a, b, best, second, idx, m, ssum);
+            combine_chunk<true>(acc, lbuf + cc * box_bytes + br * 128, 0, swz, true, ptile + cc * 32,
+                                it.o0 + cc * 32, a.V, alpha, nbeta, best, second, idx, m, ssum, g);
         }
       } else if (c1 < nchunk) {
         float acc0[32], acc1[32];
@@ -605,9 +639,11 @@ __device__ __forceinline__ bool epi_run(const Ctx& c, const Phase& p, EpiState& 
     if (lane == 0) {
       mbar_arrive(&c.acce[buf]);
       if (comb) mbar_arrive(&c.lempty[lbuf_i]);
+      if (SAMPLE) mbar_arrive(&c.nempty[nbuf]);
     }
     ++st.tiles;
     if (comb) ++st.ltiles;
+    if (SAMPLE) ++st.ntiles;
   }
   if (comb) {
     // merge the workers' states of each row, publish one record per request

@@ -29,6 +29,9 @@ using namespace tce;
 
 constexpr int kWarps = 11;
 constexpr int kThreads = kWarps * 32;
+constexpr int kNoiseWarps = 8;                          // temperature-1 combine launches
+constexpr int kThreadsSample = (kWarps + kNoiseWarps) * 32;
+__host__ __device__ constexpr int threads_for(int mode) { return mode == 2 ? kThreadsSample : kThreads; }
 constexpr int kLWarp = 10;
 
 struct Smem {
@@ -141,11 +144,12 @@ __device__ __forceinline__ void epi_cluster_finish(const Ctx& c, const TcGemmArg
 }
 
 // MODE 1 / 2: combine launches at temperature 0 / 1 (one CTA per SM, the
-// combine epilogue's registers); MODE 0: store launches, compiled separately
+// combine epilogue's registers; MODE 2 adds the 8 noise warps and their two
+// TMEM buffers); MODE 0: store launches, compiled separately
 // with at most 2 x 352 threads' worth of registers per SM, so that a store
 // launch's CTAs can share an SM with the small kernels around them.
 template <int MODE>
-__global__ void __launch_bounds__(kThreads, MODE != 0 ? 1 : 2)
+__global__ void __launch_bounds__(threads_for(MODE), MODE != 0 ? 1 : 2)
     k_tc_gemm(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ CUtensorMap mB0,
               const __grid_constant__ CUtensorMap mA1, const __grid_constant__ CUtensorMap mB1,
               const __grid_constant__ CUtensorMap mL, const __grid_constant__ TcGemmArgs a0,
@@ -178,6 +182,8 @@ __global__ void __launch_bounds__(kThreads, MODE != 0 ? 1 : 2)
   c.lfull = c.acce + 2;
   c.lempty = c.lfull + 2;
   c.afull = c.lempty + 2;
+  c.nfull = bars + 48;    // noise barriers (temperature 1): slots past the others'
+  c.nempty = bars + 50;
   uint64_t* mmadone = c.afull + 1;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mmadone + 1);
   c.abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
@@ -186,8 +192,11 @@ __global__ void __launch_bounds__(kThreads, MODE != 0 ? 1 : 2)
   c.b_stage_bytes = (uint32_t)a.n_tile * 128u * (uint32_t)(a.b_chunks > 1 ? a.b_chunks : 1);
   c.l_buf_bytes = comb ? (uint32_t)(a.l_boxes * a.l_box_rows * 128) : 0u;
   c.deadline = globaltimer_ns() + budget_ns;
-  const uint32_t tmem_cols =
+  // two accumulator buffers; at temperature 1 two noise buffers after them
+  const uint32_t acc_cols =
       (a.n_tile * 2 <= 32) ? 32u : (uint32_t)(a.n_tile * 2 <= 64 ? 64 : (a.n_tile * 2 <= 128 ? 128 : 256));
+  const uint32_t tmem_cols = MODE == 2 ? 2u * acc_cols : acc_cols;
+  c.noise_col = acc_cols;
 
   if (threadIdx.x == 0) {
     pdl_trigger();
@@ -203,6 +212,12 @@ __global__ void __launch_bounds__(kThreads, MODE != 0 ? 1 : 2)
     }
     mbar_init(c.afull, 1);
     mbar_init(mmadone, 1);
+    if (MODE == 2) {
+      for (int i = 0; i < 2; ++i) {
+        mbar_init(&c.nfull[i], kNoiseWarps);
+        mbar_init(&c.nempty[i], kEpiWarps);
+      }
+    }
     *c.abort_flag = 0;
     fence_mbarrier_init();
   }
@@ -280,6 +295,9 @@ __global__ void __launch_bounds__(kThreads, MODE != 0 ? 1 : 2)
       volatile int dummy = 0;
       mbar_wait(mmadone, 0, globaltimer_ns() + 100000000ull, &dummy);
     }
+  } else if (MODE == 2 && warp >= kWarps) {
+    // the variates depend on the arguments only: no wait for the predecessor
+    noise_run(c, p, warp, lane, (warp - kWarps) >> 2);
   } else {
     if (comb) epi_stage_prior(c, p, threadIdx.x - 64);   // an input: no wait needed
     pdl_wait();
@@ -326,6 +344,7 @@ cudaError_t launch_tc_gemm(const TcGemmArgs& a, const CUtensorMap* mA0, const CU
   if (two && (second->a->epi == EPI_COMBINE) != comb) return cudaErrorInvalidValue;
   const int mode = comb ? (a.sample ? 2 : 1) : 0;
   auto kern = mode == 2 ? k_tc_gemm<2> : mode == 1 ? k_tc_gemm<1> : k_tc_gemm<0>;
+  const int threads = threads_for(mode);
   cudaError_t e = ensure_dynamic_smem(reinterpret_cast<const void*>(kern), smem_bytes);
   if (e != cudaSuccess) return e;
   const uint64_t budget = a.debug_skip_producer ? 100000000ull : kWaitBudgetNs;
@@ -335,9 +354,9 @@ cudaError_t launch_tc_gemm(const TcGemmArgs& a, const CUtensorMap* mA0, const CU
   const int ck = std::max(a.cluster_k, two ? second->a->cluster_k : 1);
   if (ck > 1 && (g0 % ck != 0 || (two && second->grid % ck != 0))) return cudaErrorInvalidValue;
   if (two)
-    return launch_pdl_cluster(kern, dim3(g0 + second->grid), dim3(kThreads), smem_bytes, s, ck, *mA0, *mB0,
+    return launch_pdl_cluster(kern, dim3(g0 + second->grid), dim3(threads), smem_bytes, s, ck, *mA0, *mB0,
                               *mA1, *mB1, *mL, a, *second->mA, *second->mB, *second->a, g0, budget);
-  return launch_pdl_cluster(kern, dim3(g0), dim3(kThreads), smem_bytes, s, ck, *mA0, *mB0, *mA1, *mB1, *mL, a,
+  return launch_pdl_cluster(kern, dim3(g0), dim3(threads), smem_bytes, s, ck, *mA0, *mB0, *mA1, *mB1, *mL, a,
                             *mA0, *mB0, a, g0, budget);
 }
 
