@@ -561,18 +561,16 @@ __device__ __forceinline__ bool epi_run(const Ctx& c, const Phase& p, EpiState& 
             combine_chunk<true>(acc, lbuf + cc * box_bytes + br * 128, 0, swz, true, ptile + cc * 32,
                                 it.o0 + cc * 32, a.V, alpha, nbeta, best, second, idx, m, ssum, g);
         }
-      } else if (c1 < nchunk) {
-        float acc0[32], acc1[32];
-        tmem_ld_32x32b_x32(tbase + (uint32_t)(c0 * 32), acc0);
-        tmem_ld_32x32b_x32(tbase + (uint32_t)(c1 * 32), acc1);
-        tmem_ld_wait();
-        run_chunk(acc0, c0);
-        run_chunk(acc1, c1);
-      } else if (c0 < nchunk) {
-        float acc0[32];
-        tmem_ld_32x32b_x32(tbase + (uint32_t)(c0 * 32), acc0);
-        tmem_ld_wait();
-        run_chunk(acc0, c0);
+      } else {
+        // one call site per type: the unrolled chunk is large, and more
+        // copies of it cost instruction-cache misses
+#pragma unroll 1
+        for (int cc = c0; cc < nchunk; cc += workers) {
+          float acc0[32];
+          tmem_ld_32x32b_x32(tbase + (uint32_t)(cc * 32), acc0);
+          tmem_ld_wait();
+          run_chunk(acc0, cc);
+        }
       }
     } else if (quad_live) {
       for (int cc = g; cc < nchunk; cc += 2) {
