@@ -316,10 +316,11 @@ bool plan_combine(Gemm& g, int B, int V, int n, const void* X, int K, const void
   } else {
     a.stages = pick_stages(a, 128 * 128 + n_tile * 128, l_fixed);
   }
-  // Resident activations and an even number of K chunks: each weight stage
-  // holds two consecutive chunks, loaded as one 3-D box (the weight rows'
-  // 256-byte spans in one request; 8B-shaped launch 29.2 -> 26.8 us).
-  if (pair_stages && a.a_resident && a.seg_chunks[0] % 2 == 0) {
+  // An even number of K chunks: each pipeline stage holds two consecutive
+  // chunks, the weights' as one 3-D box (8B-shaped launch 29.2 -> 26.8 us;
+  // with staged activations, 0.6B-shaped 59.6 -> 53.9 us, 4B-shaped
+  // 130.9 -> 126.5 us).
+  if (pair_stages && a.seg_chunks[0] % 2 == 0) {
     a.b_chunks = 2;
     a.stages = std::max(2, a.stages / 2);
   }

@@ -205,7 +205,7 @@ struct TcGemmArgs {
   int total_splits;
   int epi;
   int a_resident;                // A (activations) loaded once per CTA
-  int b_chunks;                  // weight K chunks per pipeline stage: 2 (one 3-D box, resident A only); 0 or 1: one
+  int b_chunks;                  // K chunks per pipeline stage: 2 (the weights' as one 3-D box); 0 or 1: one
   int stages;
   int max_items_per_cta;         // EPI_COMBINE: sizes the per-CTA prior slice in smem
   int a_box_rows;                // activation rows per TMA box (the map's box height)

@@ -7,9 +7,9 @@
 // (both operands K-major). Four roles run it, each on its own thread(s):
 //
 //  * producer (one thread): TMA loads of weight tiles (B operand) and
-//    activation tiles (A operand) into a ring of S stages (with resident
-//    activations a stage may hold two consecutive K chunks of the weights,
-//    loaded as one 3-D box: b_chunks = 2). Weight tiles do not
+//    activation tiles (A operand) into a ring of S stages (a stage may hold
+//    two consecutive K chunks, the weights' loaded as one 3-D box:
+//    b_chunks = 2). Weight tiles do not
 //    depend on anything computed earlier, so `prod_prefetch` issues the next
 //    phase's first weight stages early (their barriers get the weight bytes as
 //    expected transactions; the arrival, with any activation bytes, comes from
@@ -216,7 +216,7 @@ __device__ __forceinline__ bool prod_prefetch(const Ctx& c, const Phase& p, Prod
 }
 
 // Load the activations (and the remaining weights) of the phase.
-template <int C>   // > 1 only with resident activations
+template <int C>
 __device__ __forceinline__ bool prod_run_c(const Ctx& c, const Phase& p, ProdState& st, uint64_t pol_w,
                                            uint64_t pol_act) {
   const TcGemmArgs& a = *p.a;
@@ -241,13 +241,17 @@ __device__ __forceinline__ bool prod_run_c(const Ctx& c, const Phase& p, ProdSta
     for (int i = 0; i < it.ke - it.kb; i += C, ++f) {
       const int kc = it.chunk(i);
       const int s = f % c.S;
+      // staged activations: chunk kc + cc of the stage at sA + s * a_stage_bytes + cc * kATileBytes
       if (f < st.pre_end) {
         if (a.a_resident) {
           mbar_arrive(&c.full[s]);
         } else {
-          mbar_arrive_expect_tx(&c.full[s], a_bytes);
-          for (int cp = 0; cp < a.a_copies; ++cp)
-            tma_load_2d(c.sA + s * c.a_stage_bytes + cp * a_copy_bytes, mA, &c.full[s], kc * kBlockK, 0, pol_act);
+          mbar_arrive_expect_tx(&c.full[s], (uint32_t)C * a_bytes);
+#pragma unroll
+          for (int cc = 0; cc < C; ++cc)
+            for (int cp = 0; cp < a.a_copies; ++cp)
+              tma_load_2d(c.sA + s * c.a_stage_bytes + cc * kATileBytes + cp * a_copy_bytes, mA, &c.full[s],
+                          (kc + cc) * kBlockK, 0, pol_act);
         }
         continue;
       }
@@ -255,10 +259,14 @@ __device__ __forceinline__ bool prod_run_c(const Ctx& c, const Phase& p, ProdSta
         st.fills = f;
         return false;
       }
-      mbar_arrive_expect_tx(&c.full[s], b_bytes + (a.a_resident ? 0u : a_bytes));
-      if (!a.a_resident)
-        for (int cp = 0; cp < a.a_copies; ++cp)
-          tma_load_2d(c.sA + s * c.a_stage_bytes + cp * a_copy_bytes, mA, &c.full[s], kc * kBlockK, 0, pol_act);
+      mbar_arrive_expect_tx(&c.full[s], b_bytes + (a.a_resident ? 0u : (uint32_t)C * a_bytes));
+      if (!a.a_resident) {
+#pragma unroll
+        for (int cc = 0; cc < C; ++cc)
+          for (int cp = 0; cp < a.a_copies; ++cp)
+            tma_load_2d(c.sA + s * c.a_stage_bytes + cc * kATileBytes + cp * a_copy_bytes, mA, &c.full[s],
+                        (kc + cc) * kBlockK, 0, pol_act);
+      }
       load_w<C>(c, p, it, i, s, pol_w);
     }
   }
@@ -330,7 +338,7 @@ __device__ __forceinline__ bool mma_run_c(const Ctx& c, const Phase& p, MmaState
       for (int cc = 0; cc < C; ++cc) {
         const int kc = it.chunk(i + cc);
         const uint32_t a_addr =
-            smem_u32(a.a_resident ? c.sA + kc * kATileBytes : c.sA + s * c.a_stage_bytes);
+            smem_u32(a.a_resident ? c.sA + kc * kATileBytes : c.sA + s * c.a_stage_bytes + cc * kATileBytes);
         const uint32_t b_addr = smem_u32(c.sB + s * c.b_stage_bytes + cc * a.n_tile * 128);
 #pragma unroll
         for (int kk = 0; kk < kBlockK / kUmmaK; ++kk) {

@@ -49,7 +49,7 @@ __host__ __device__ inline Smem smem_layout(const TcGemmArgs& a) {
   const int b_tile = a.n_tile * 128;
   const bool comb = a.epi == EPI_COMBINE;
   const int l_tile = comb ? a.l_boxes * a.l_box_rows * 128 : 0;
-  const int a_tiles = a.a_resident ? a.seg_chunks[0] : a.stages;
+  const int a_tiles = a.a_resident ? a.seg_chunks[0] : a.stages * (a.b_chunks > 1 ? a.b_chunks : 1);
   uint32_t off = 0;
   s.a_off = off;
   off += (uint32_t)a_tiles * kATileBytes;
@@ -188,7 +188,7 @@ __global__ void __launch_bounds__(threads_for(MODE), MODE != 0 ? 1 : 2)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mmadone + 1);
   c.abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   c.S = a.stages;
-  c.a_stage_bytes = kATileBytes;
+  c.a_stage_bytes = kATileBytes * (uint32_t)(a.b_chunks > 1 ? a.b_chunks : 1);
   c.b_stage_bytes = (uint32_t)a.n_tile * 128u * (uint32_t)(a.b_chunks > 1 ? a.b_chunks : 1);
   c.l_buf_bytes = comb ? (uint32_t)(a.l_boxes * a.l_box_rows * 128) : 0u;
   c.deadline = globaltimer_ns() + budget_ns;
