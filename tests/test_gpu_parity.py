@@ -221,6 +221,9 @@ SMALL = {
                             head_d_model=256, head_d_hidden=128, head_d_rank=64),
     "gru_b64": synth.with_sizes(synth.WORKLOADS["qwen3_8b_batched"], B=64, n=4, V=4096,
                                 head_d_model=512, head_d_hidden=256, head_d_rank=256),
+    # more than 64 requests: one 128-row copy of the activations, all four TMEM lane quadrants live
+    "gru_b100": synth.with_sizes(synth.WORKLOADS["qwen3_8b_batched"], B=100, n=3, V=2048,
+                                 head_d_model=256, head_d_hidden=128, head_d_rank=128),
     "mlp2": synth.with_sizes(synth.WORKLOADS["qwen3_0p6b"], B=3, n=6, V=2000,
                              head_d_model=128, head_d_hidden=192, head_d_rank=192),
     # more requests than the CUDA-core path takes: tensor-core products + reductions

@@ -35,7 +35,8 @@ def _sampled(name, seed=17, step=3, weights="learned"):
     return w, d, W, a, b, tok.cpu().numpy(), lp.cpu().numpy(), gap.cpu().numpy(), state
 
 
-@pytest.mark.parametrize("name,seed,step", [("gru", 17, 3), ("gru_b64", 17, 3), ("mlp2", 17, 3), ("xfmr", 17, 3),
+@pytest.mark.parametrize("name,seed,step", [("gru", 17, 3), ("gru_b64", 17, 3), ("gru_b100", 17, 3), ("mlp2", 17, 3),
+                                            ("xfmr", 17, 3),
                                             ("markov", 17, 3), ("gru_f32", 17, 3), ("tiny", 17, 3),
                                             ("gru", 0xFEDCBA9876543210, 2 ** 32 - 1)])
 def test_sampled_draft_matches_oracle(name, seed, step):
