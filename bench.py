@@ -853,7 +853,8 @@ def run_sampled(args):
             "roofline": {"bound": "hbm", "kernel": "k_tc_gemm<sample> (vocab projection + Gumbel-max)",
                          "achieved": vbytes_alg / (us_v * 1e-6) / 1e9, "peak": peak, "unit": "GB/s",
                          "frac": vbytes_alg / (us_v * 1e-6) / 1e9 / peak, "peak_source": peak_kind,
-                         "us_per_launch": us_v},
+                         "us_per_launch": us_v, "algorithmic_bytes_per_launch": vbytes_alg,
+                         "traffic": ncu_traffic("vocab_sample_qwen3_8b_batched.md")},
             "clocks": clk.summary()}), flush=True)
     replicas.barrier()
     return 0
